@@ -1,0 +1,83 @@
+/*
+ * pced_oracle.h -- CPU oracle of one Parallel Context-of-Experts Decoding
+ * (PCED) step.  TEST INFRASTRUCTURE ONLY: the tests, the smoke check and the
+ * benchmark's CPU-baseline leg call it; the decoding library never does.
+ *
+ * Plain fp64 statement of what the decode step computes (paper Sec. 3,
+ * "Parallel Context-of-Experts" and "Retrieval-aware contrastive decoding",
+ * Eq. 2 and Eq. 3), written for checkability rather than speed.  bf16
+ * tensors are passed as raw uint16 bit patterns.
+ */
+#ifndef PCED_ORACLE_H
+#define PCED_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* exact value of a bf16 bit pattern */
+double oracle_bf16_value(uint16_t bits);
+/* nearest bf16 to x, ties to even (x finite, |x| < 3e38) */
+uint16_t oracle_round_bf16(double x);
+/* y = x / sqrt(mean(x^2) + eps) */
+void oracle_rmsnorm(const double* x, int32_t n, double eps, double* y);
+
+/* One layer of decode attention for S sequences.
+ * q: bf16 [S][Hq][D].  kc/vc: one layer's cache region; the slab of
+ * (sequence s, kv-head h) starts at element kv_off[s] + h*cap[s]*D and its
+ * first len[s] rows of D elements are the keys/values attended to.
+ * Query head hq reads kv-head hq / (Hq/Hkv) (grouped-query attention).
+ * out: fp64 [S][Hq][D] = softmax(scale * q K^T) V.  Returns 0, or -1 on bad
+ * arguments. */
+int32_t oracle_attention(const uint16_t* q, const uint16_t* kc, const uint16_t* vc, const int64_t* kv_off,
+                         const int32_t* cap, const int32_t* len, int32_t S, int32_t Hq, int32_t Hkv, int32_t D,
+                         double scale, double* out, int32_t nthreads);
+
+/* Unembedding + log-softmax: z[s][v] = sum_i h[s][i] * W[v][i];
+ * lse[s] = log sum_v exp(z[s][v]); lp[s][v] = z[s][v] - lse[s].
+ * h: bf16 [S][d], W: bf16 [V][d]; lp: fp64 [S][V]; lse: fp64 [S]. */
+int32_t oracle_lm_head_logprobs(const uint16_t* h, const uint16_t* w, int32_t S, int32_t d, int32_t V, double* lp,
+                                double* lse, int32_t nthreads);
+
+/* Eq. 2 + Eq. 3 on log-probabilities lp [S][V] (row b*(N+1) is query b's
+ * amateur, rows b*(N+1)+k, k = 1..N, its contextual experts).
+ *   shat_k(v) = (1 + beta[b][k-1]) lp_k(v) - beta[b][k-1] lp_0(v) + gamma log r~[b][k-1],
+ *   r~ = min(max(r, 1e-8), 1 - 1e-8),
+ *   token[b] = argmax_v max_k shat_k(v), expert[b] = the maximising k (1-based).
+ * Exact ties: highest score, then lowest token id, then lowest expert.
+ * token_gap[b] = score - max_{v != token} max_k shat_k(v);
+ * expert_gap[b] = score - max_{k != expert} shat_k(token)  (+inf when N = 1). */
+int32_t oracle_contrastive_select(const double* lp, const float* beta, const float* r, double gamma, int32_t B,
+                                  int32_t N, int32_t V, int32_t* token, int32_t* expert, double* score,
+                                  double* token_gap, double* expert_gap);
+
+typedef struct oracle_dims {
+  int32_t B, N, L, Hq, Hkv, D, V; /* S = B*(N+1), d = Hq*D, requires 2*Hkv <= Hq */
+  double gamma;                   /* retrieval-prior weight of Eq. 2 */
+  double rms_eps;                 /* RMSNorm epsilon */
+  double attn_scale;              /* softmax scale, 1/sqrt(D) */
+} oracle_dims;
+
+/* One full decode step of the synthetic PCED model.
+ *   x_0[s]    = emb_rows[b]            (embedding of query b's previous token)
+ *   per layer l:  u = bf16(rmsnorm(x_l[s]));  K_l[s][h][len] = u[h], V_l[s][h][len] = u[Hkv + h]
+ *                 (h < Hkv, appended at the old length; the length grows by one per step)
+ *                 x_{l+1}[s] = x_l[s] + attention(u as [Hq][D], K_l, V_l)
+ *   h[s]      = bf16(rmsnorm(x_L[s]))
+ *   then the unembedding/log-softmax and Eq. 2 + Eq. 3 selection.
+ * kc/vc span L layers of layer_elems elements (slab layout as in
+ * oracle_attention); len[S] is updated in place; h_out (bf16 [S][d]) and
+ * lse_out ([S]) may be NULL.  Returns 0, -1 on bad arguments, -2 when a
+ * cache is full. */
+int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, int64_t layer_elems,
+                           const int64_t* kv_off, const int32_t* cap, int32_t* len, const uint16_t* emb_rows,
+                           const uint16_t* w, const float* beta, const float* r, int32_t* token, int32_t* expert,
+                           double* score, double* token_gap, double* expert_gap, uint16_t* h_out, double* lse_out,
+                           int32_t nthreads);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PCED_ORACLE_H */
