@@ -1,0 +1,182 @@
+/*
+ * pced.h -- C ABI of the GB300 (sm_103a) implementation of one decode step of
+ * Parallel Context-of-Experts Decoding (PCED, arXiv 2601.08670).
+ *
+ * The paper (Sec. 3, "Parallel Context-of-Experts") runs N+1 streams in one
+ * batched pass: an amateur with no document (model prior) and N contextual
+ * experts, each attending over its own independently encoded KV cache.  Each
+ * step turns every expert's hidden state into log-probabilities s_k, scores
+ *   shat_k = (1 + beta) s_k - beta s_0 + gamma log r_k          (Eq. 2)
+ * and picks  y_t = argmax_v max_{k in 1..N} shat_k(v)            (Eq. 3),
+ * then appends y_t to the shared history of all experts.
+ *
+ * Conventions shared by every entry point
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the
+ *     library allocates nothing and never synchronises.  `stream` is a
+ *     cudaStream_t (NULL = legacy default stream).
+ *   - bf16 tensors are raw bf16 arrays (2 bytes per element).
+ *   - Sequences are query-major: sequence s = b*(N+1) + j belongs to query b;
+ *     j = 0 is the amateur, j = 1..N are the contextual experts.
+ *   - KV-cache slabs: for layer l, sequence s and kv-head h the keys (values)
+ *     are cap[s] rows of D elements starting at element
+ *         l*layer_elems + kv_offset[s] + h*cap[s]*D
+ *     of k_cache (v_cache); rows [0, seq_len[s]) are live.
+ *   - Every call validates its host-visible arguments before launching and
+ *     returns a pced_status; nothing is launched on failure.  Conditions only
+ *     visible on the device (a length above its capacity, a token outside the
+ *     vocabulary, a full cache, a bounded wait that ran out) set bits of the
+ *     32-bit device status word at byte 0 of the caller's workspace; the
+ *     library only ORs bits into it, so the caller zeroes it once and reads it
+ *     when convenient.
+ *   - Workspaces must be 256-byte aligned and at least as large as the
+ *     matching *_workspace_size() result.
+ */
+#ifndef PCED_H
+#define PCED_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum pced_status {
+  PCED_OK = 0,
+  PCED_ERR_INVALID_ARG = 1, /* null pointer, inconsistent or out-of-range size */
+  PCED_ERR_WORKSPACE = 2,   /* workspace too small or misaligned */
+  PCED_ERR_UNSUPPORTED = 3, /* shape the kernels do not implement (see each call) */
+  PCED_ERR_CUDA = 4,        /* a CUDA runtime/driver call failed */
+  PCED_ERR_NO_DEVICE = 5    /* no usable sm_103 device */
+} pced_status;
+
+/* device status word bits (byte 0 of the workspace) */
+#define PCED_DEV_BAD_LENGTH 0x1u  /* seq_len outside [1, cap] */
+#define PCED_DEV_CACHE_FULL 0x2u  /* pced_step found no room for the new token */
+#define PCED_DEV_TIMEOUT 0x4u     /* a bounded in-kernel wait expired */
+#define PCED_DEV_BAD_TOKEN 0x8u   /* history token outside [0, V) */
+#define PCED_DEV_STEP_LIMIT 0x10u /* step counter reached max_steps */
+
+/* Static description of a status code (host). */
+const char* pced_status_string(int32_t status);
+/* Detail of the last failing call on this host thread (host, static storage). */
+const char* pced_last_error(void);
+
+typedef struct pced_dims {
+  int32_t B;   /* independent queries */
+  int32_t N;   /* contextual experts per query; the amateur is extra, S = B*(N+1) */
+  int32_t L;   /* layers */
+  int32_t Hq;  /* query heads */
+  int32_t Hkv; /* kv heads (grouped-query attention, Hq % Hkv == 0) */
+  int32_t D;   /* head dim; hidden size d = Hq*D */
+  int32_t V;   /* vocabulary size */
+} pced_dims;
+
+/* ------------------------------------------------------------------------
+ * pced_decode_attention -- one layer of decode attention for all S
+ * sequences, each over its own cache (Sec. 3: each expert keeps its own KV
+ * cache and attends only to it; grouped-query heads).
+ *   q        bf16 [S][Hq][D]   query of the token being decoded
+ *   k_cache, v_cache           bf16 cache region of THIS layer: slab (s, h)
+ *                              at kv_offset[s] + h*cap[s]*D, cache_elems
+ *                              elements in total
+ *   kv_offset int64 [S], cap int32 [S], seq_len int32 [S] (device; the token
+ *                              being decoded is already appended, so it is
+ *                              row seq_len[s]-1 and attends to itself)
+ *   total_cap                  host upper bound of sum(seq_len) (e.g. sum(cap));
+ *                              sizes the grid only
+ *   scale                      softmax scale, usually 1/sqrt(D)
+ *   out      fp32 [S][Hq][D]   o = softmax(scale q K^T) V
+ * Query head hq reads kv-head hq / (Hq/Hkv).  Supports D in {64, 128},
+ * Hq/Hkv <= 8, cache_elems/D < 2^31, 16-byte aligned caches.
+ * ------------------------------------------------------------------------ */
+size_t pced_decode_attention_workspace_size(int32_t S, int32_t Hq, int32_t Hkv, int32_t D);
+pced_status pced_decode_attention(const void* q, const void* k_cache, const void* v_cache, int64_t cache_elems,
+                                  const int64_t* kv_offset, const int32_t* cap, const int32_t* seq_len, int32_t S,
+                                  int32_t Hq, int32_t Hkv, int32_t D, int64_t total_cap, float scale, float* out,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * pced_lm_head_logprobs -- per-expert log-probabilities s_k over the
+ * vocabulary (Sec. 3: "per-expert logits s_k in R^|V|"; read as
+ * log-softmax outputs, the scale Eq. 2 mixes).
+ *   hidden    bf16 [S][d]   final normalised hidden states
+ *   w_unembed bf16 [V][d]   unembedding matrix (row v = token v)
+ *   logprobs  fp32 [S][V]   z - lse with z = hidden W^T
+ *   lse       fp32 [S]      log sum_v exp(z[s][v])
+ * Supports 1 <= S <= 512, d % 64 == 0, d <= 16384, 16-byte aligned rows.
+ * ------------------------------------------------------------------------ */
+size_t pced_lm_head_workspace_size(int32_t S, int32_t V);
+pced_status pced_lm_head_logprobs(const void* hidden, const void* w_unembed, int32_t S, int32_t d, int32_t V,
+                                  float* logprobs, float* lse, void* workspace, size_t workspace_bytes,
+                                  void* stream);
+
+/* ------------------------------------------------------------------------
+ * pced_contrastive_select -- Eq. 2 and Eq. 3 on materialised log-probs.
+ *   logprobs fp32 [S][V], S = B*(N+1), query-major, amateur first
+ *   beta     fp32 [B][N]  contrastive strength of each expert (a broadcast beta_0)
+ *   r        fp32 [B][N]  relevance scores, clipped on the device to [1e-8, 1]
+ *   gamma                 weight of the retrieval prior
+ *   token    int32 [B]    argmax_v max_k shat_k(v)
+ *   expert   int32 [B]    maximising expert, 1-based
+ *   score    fp32 [B]     the maximal shat
+ * Exact ties go to the lowest token id, then the lowest expert index.
+ * ------------------------------------------------------------------------ */
+size_t pced_contrastive_select_workspace_size(int32_t B, int32_t N, int32_t V);
+pced_status pced_contrastive_select(const float* logprobs, const float* beta, const float* r, float gamma, int32_t B,
+                                    int32_t N, int32_t V, int32_t* token, int32_t* expert, float* score,
+                                    void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * pced_step -- one full greedy decode step of all B queries (Sec. 3,
+ * Eq. 2, Eq. 3 and the shared-history append) on the weight-free layer
+ * chain used for synthetic workloads:
+ *   x_0     = embed[y_{t-1}]           (y_{-1} = bos_token; shared by all experts of a query)
+ *   layer l: u = bf16(rmsnorm(x_l));  append K row u[0:Hkv) and V row u[Hkv:2Hkv) (as heads)
+ *            at position seq_len (then seq_len+1 rows are live)
+ *            x_{l+1} = x_l + attention(u as [Hq][D], own cache of layer l)   (fp32)
+ *   h       = bf16(rmsnorm(x_L))
+ *   token   = Eq. 3 over Eq. 2 of log_softmax(h W^T); appended to history[b][t]
+ * The step index t, lengths and history live on the device, so a captured
+ * CUDA graph of one call can be replayed step after step.  Each call adds
+ * one to *step and to every seq_len[s].  Requires 2*Hkv <= Hq plus the limits
+ * of the three calls above.
+ * ------------------------------------------------------------------------ */
+typedef struct pced_step_args {
+  pced_dims dims;
+  const void* embed;        /* bf16 [V][d] token embedding */
+  const void* w_unembed;    /* bf16 [V][d] */
+  void* k_cache;            /* bf16, L regions of layer_elems elements */
+  void* v_cache;
+  int64_t layer_elems;
+  const int64_t* kv_offset; /* [S] */
+  const int32_t* cap;       /* [S] rows per slab */
+  int64_t total_cap;        /* host: sum of cap */
+  int32_t* seq_len;         /* [S] live rows; +1 per step */
+  int32_t* step;            /* [1] step counter t; +1 per step */
+  int32_t* history;         /* [B][max_steps] chosen tokens */
+  int32_t* expert_trace;    /* [B][max_steps] winning expert (1-based), may be NULL */
+  float* score_trace;       /* [B][max_steps] winning score, may be NULL */
+  int32_t max_steps;
+  const float* beta;        /* [B][N] */
+  const float* r;           /* [B][N] relevance scores */
+  float gamma;
+  float attn_scale;         /* usually 1/sqrt(D) */
+  float rms_eps;            /* usually 1e-6 */
+  int32_t bos_token;
+  void* hidden_out;         /* optional bf16 [S][d]: h of this step */
+  float* lse_out;           /* optional fp32 [S]: log-sum-exp of each row of h W^T */
+  void* workspace;
+  size_t workspace_bytes;
+} pced_step_args;
+
+size_t pced_step_workspace_size(const pced_dims* dims);
+pced_status pced_step(const pced_step_args* args, void* stream);
+
+/* Number of kernel launches one pced_step call makes for these dimensions. */
+int32_t pced_step_launch_count(const pced_dims* dims);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PCED_H */

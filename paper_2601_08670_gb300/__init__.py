@@ -1,0 +1,234 @@
+"""GB300 (sm_103a) decode step of Parallel Context-of-Experts Decoding.
+
+Thin ctypes binding of ``libpced.so`` (C ABI declared in ``include/pced.h``):
+argument marshalling only, every step of the computation runs in the
+library's CUDA kernels.  PyTorch supplies device memory and streams.  There is
+no CPU fallback: if the library is not built, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "_lib", "libpced.so")
+
+PCED_DEV_BAD_LENGTH = 0x1
+PCED_DEV_CACHE_FULL = 0x2
+PCED_DEV_TIMEOUT = 0x4
+PCED_DEV_BAD_TOKEN = 0x8
+PCED_DEV_STEP_LIMIT = 0x10
+
+
+class PcedError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(msg)
+        self.status = status
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("N", ctypes.c_int32), ("L", ctypes.c_int32), ("Hq", ctypes.c_int32),
+                ("Hkv", ctypes.c_int32), ("D", ctypes.c_int32), ("V", ctypes.c_int32)]
+
+
+class StepArgs(ctypes.Structure):
+    _fields_ = [("dims", Dims), ("embed", ctypes.c_void_p), ("w_unembed", ctypes.c_void_p),
+                ("k_cache", ctypes.c_void_p), ("v_cache", ctypes.c_void_p), ("layer_elems", ctypes.c_int64),
+                ("kv_offset", ctypes.c_void_p), ("cap", ctypes.c_void_p), ("total_cap", ctypes.c_int64),
+                ("seq_len", ctypes.c_void_p), ("step", ctypes.c_void_p), ("history", ctypes.c_void_p),
+                ("expert_trace", ctypes.c_void_p), ("score_trace", ctypes.c_void_p), ("max_steps", ctypes.c_int32),
+                ("beta", ctypes.c_void_p), ("r", ctypes.c_void_p), ("gamma", ctypes.c_float),
+                ("attn_scale", ctypes.c_float), ("rms_eps", ctypes.c_float), ("bos_token", ctypes.c_int32),
+                ("hidden_out", ctypes.c_void_p), ("lse_out", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
+                ("workspace_bytes", ctypes.c_size_t)]
+
+
+_lib = None
+
+
+def lib(path: str = LIB_PATH):
+    """Load libpced.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is missing: build it with paper_2601_08670_gb300.build.build()")
+        L = ctypes.CDLL(path)
+        P, I32, I64, SZ, F = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t, ctypes.c_float
+        L.pced_status_string.argtypes = [I32]
+        L.pced_status_string.restype = ctypes.c_char_p
+        L.pced_last_error.argtypes = []
+        L.pced_last_error.restype = ctypes.c_char_p
+        L.pced_decode_attention_workspace_size.argtypes = [I32, I32, I32, I32]
+        L.pced_decode_attention_workspace_size.restype = SZ
+        L.pced_decode_attention.argtypes = [P, P, P, I64, P, P, P, I32, I32, I32, I32, I64, F, P, P, SZ, P]
+        L.pced_decode_attention.restype = I32
+        L.pced_lm_head_workspace_size.argtypes = [I32, I32]
+        L.pced_lm_head_workspace_size.restype = SZ
+        L.pced_lm_head_logprobs.argtypes = [P, P, I32, I32, I32, P, P, P, SZ, P]
+        L.pced_lm_head_logprobs.restype = I32
+        L.pced_contrastive_select_workspace_size.argtypes = [I32, I32, I32]
+        L.pced_contrastive_select_workspace_size.restype = SZ
+        L.pced_contrastive_select.argtypes = [P, P, P, F, I32, I32, I32, P, P, P, P, SZ, P]
+        L.pced_contrastive_select.restype = I32
+        L.pced_step_workspace_size.argtypes = [ctypes.POINTER(Dims)]
+        L.pced_step_workspace_size.restype = SZ
+        L.pced_step.argtypes = [ctypes.POINTER(StepArgs), P]
+        L.pced_step.restype = I32
+        L.pced_step_launch_count.argtypes = [ctypes.POINTER(Dims)]
+        L.pced_step_launch_count.restype = I32
+        _lib = L
+    return _lib
+
+
+def _check(rc: int, what: str):
+    if rc != 0:
+        L = lib()
+        raise PcedError(rc, f"{what}: {L.pced_status_string(rc).decode()}: {L.pced_last_error().decode()}")
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    """Zeroed workspace (the device status word at byte 0 starts clear)."""
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def device_status(ws: torch.Tensor) -> int:
+    """Device status bits the kernels ORed into the workspace (synchronises)."""
+    return int(ws[:4].view(torch.int32).item())
+
+
+# ------------------------------------------------------------------ entry points
+def decode_attention_workspace_size(S, Hq, Hkv, D) -> int:
+    return int(lib().pced_decode_attention_workspace_size(S, Hq, Hkv, D))
+
+
+def decode_attention(q, k_cache, v_cache, kv_offset, cap, seq_len, Hkv: int, total_cap: int, scale=None, out=None,
+                     ws=None, stream=None):
+    """pced_decode_attention: q bf16 [S, Hq, D]; caches bf16 (one layer); returns fp32 [S, Hq, D]."""
+    S, Hq, D = q.shape
+    scale = 1.0 / math.sqrt(D) if scale is None else scale
+    if out is None:
+        out = torch.empty((S, Hq, D), dtype=torch.float32, device=q.device)
+    if ws is None:
+        ws = workspace(decode_attention_workspace_size(S, Hq, Hkv, D), q.device)
+    _check(lib().pced_decode_attention(_ptr(q), _ptr(k_cache), _ptr(v_cache), k_cache.numel(), _ptr(kv_offset),
+                                       _ptr(cap), _ptr(seq_len), S, Hq, Hkv, D, int(total_cap), float(scale),
+                                       _ptr(out), _ptr(ws), ws.numel(), _stream(stream)), "pced_decode_attention")
+    return out
+
+
+def lm_head_workspace_size(S, V) -> int:
+    return int(lib().pced_lm_head_workspace_size(S, V))
+
+
+def lm_head_logprobs(hidden, w_unembed, logprobs=None, lse=None, ws=None, stream=None):
+    """pced_lm_head_logprobs: hidden bf16 [S, d], W bf16 [V, d] -> (fp32 [S, V], fp32 [S])."""
+    S, d = hidden.shape
+    V = w_unembed.shape[0]
+    if logprobs is None:
+        logprobs = torch.empty((S, V), dtype=torch.float32, device=hidden.device)
+    if lse is None:
+        lse = torch.empty(S, dtype=torch.float32, device=hidden.device)
+    if ws is None:
+        ws = workspace(lm_head_workspace_size(S, V), hidden.device)
+    _check(lib().pced_lm_head_logprobs(_ptr(hidden), _ptr(w_unembed), S, d, V, _ptr(logprobs), _ptr(lse), _ptr(ws),
+                                       ws.numel(), _stream(stream)), "pced_lm_head_logprobs")
+    return logprobs, lse
+
+
+def contrastive_select_workspace_size(B, N, V) -> int:
+    return int(lib().pced_contrastive_select_workspace_size(B, N, V))
+
+
+def contrastive_select(logprobs, beta, r, gamma: float, ws=None, stream=None):
+    """pced_contrastive_select: returns (token [B] int32, expert [B] int32, score [B] fp32)."""
+    B, N = beta.shape
+    V = logprobs.shape[1]
+    dev = logprobs.device
+    token = torch.empty(B, dtype=torch.int32, device=dev)
+    expert = torch.empty(B, dtype=torch.int32, device=dev)
+    score = torch.empty(B, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(contrastive_select_workspace_size(B, N, V), dev)
+    _check(lib().pced_contrastive_select(_ptr(logprobs), _ptr(beta), _ptr(r), float(gamma), B, N, V, _ptr(token),
+                                         _ptr(expert), _ptr(score), _ptr(ws), ws.numel(), _stream(stream)),
+           "pced_contrastive_select")
+    return token, expert, score
+
+
+def dims(B, N, L, Hq, Hkv, D, V) -> Dims:
+    return Dims(B, N, L, Hq, Hkv, D, V)
+
+
+def step_workspace_size(dm: Dims) -> int:
+    return int(lib().pced_step_workspace_size(ctypes.byref(dm)))
+
+
+def step_launch_count(dm: Dims) -> int:
+    return int(lib().pced_step_launch_count(ctypes.byref(dm)))
+
+
+class Decoder:
+    """Device-resident PCED decoding state and the pced_step call.
+
+    Holds references to the caller's caches and weights, and owns the step
+    counter, the generated history, the expert trace and the workspace.  Each
+    ``step()`` is one pced_step call (asynchronous on the current stream)."""
+
+    def __init__(self, dm: Dims, *, embed, w_unembed, k_cache, v_cache, layer_elems: int, kv_offset, cap, seq_len,
+                 beta, r, gamma: float, max_steps: int, total_cap: int, bos: int = 0, attn_scale=None,
+                 rms_eps: float = 1e-6, keep_hidden: bool = False):
+        dev = k_cache.device
+        self.dm = dm
+        B, S, d = dm.B, dm.B * (dm.N + 1), dm.Hq * dm.D
+        self.step_t = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.history = torch.zeros((B, max_steps), dtype=torch.int32, device=dev)
+        self.expert_trace = torch.zeros((B, max_steps), dtype=torch.int32, device=dev)
+        self.score_trace = torch.zeros((B, max_steps), dtype=torch.float32, device=dev)
+        self.hidden = torch.zeros((S, d), dtype=torch.bfloat16, device=dev) if keep_hidden else None
+        self.lse = torch.zeros(S, dtype=torch.float32, device=dev)
+        self.ws = workspace(step_workspace_size(dm), dev)
+        self._keep = (embed, w_unembed, k_cache, v_cache, kv_offset, cap, seq_len, beta, r)
+        self.seq_len = seq_len
+        self.beta, self.r = beta, r
+        self.args = StepArgs(
+            dm, _ptr(embed), _ptr(w_unembed), _ptr(k_cache), _ptr(v_cache), int(layer_elems), _ptr(kv_offset),
+            _ptr(cap), int(total_cap), _ptr(seq_len), _ptr(self.step_t), _ptr(self.history),
+            _ptr(self.expert_trace), _ptr(self.score_trace), int(max_steps), _ptr(beta), _ptr(r), float(gamma),
+            float(1.0 / math.sqrt(dm.D) if attn_scale is None else attn_scale), float(rms_eps), int(bos),
+            _ptr(self.hidden), _ptr(self.lse), _ptr(self.ws), self.ws.numel())
+        self.max_steps = max_steps
+
+    def step(self, stream=None):
+        _check(lib().pced_step(ctypes.byref(self.args), _stream(stream)), "pced_step")
+
+    def launches_per_step(self) -> int:
+        return step_launch_count(self.dm)
+
+    def status(self) -> int:
+        return device_status(self.ws)
+
+
+def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos: int = 0, keep_hidden=False,
+                        attn_scale=None, rms_eps: float = 1e-6) -> Decoder:
+    """Decoder over a dict of device tensors with the keys k_cache, v_cache,
+    kv_offset, cap, seq_len, embed, w_unembed, beta, r, and the host layout
+    values layer_elems / total_cap (or a `layout` object carrying them)."""
+    lay = t.get("layout")
+    layer_elems = t["layer_elems"] if "layer_elems" in t else lay.layer_elems
+    total_cap = t["total_cap"] if "total_cap" in t else int(lay.cap.astype("int64").sum())
+    return Decoder(dm, embed=t["embed"], w_unembed=t["w_unembed"], k_cache=t["k_cache"], v_cache=t["v_cache"],
+                   layer_elems=layer_elems, kv_offset=t["kv_offset"], cap=t["cap"], seq_len=t["seq_len"],
+                   beta=t["beta"], r=t["r"], gamma=gamma, max_steps=max_steps, total_cap=total_cap, bos=bos,
+                   attn_scale=attn_scale, rms_eps=rms_eps, keep_hidden=keep_hidden)

@@ -1,0 +1,448 @@
+// lm_head.cu -- per-expert vocabulary scores (paper Sec. 3, "per-expert logits
+// s_k"; Eq. 2 mixes them as log-probabilities) on the 5th-generation tensor
+// cores.
+//
+// Swap-AB skinny GEMM: Z^T[V x S] = W[V x d] * H^T[d x S].  The vocabulary is
+// the UMMA M dimension (128-row tiles), the S hidden rows are the N dimension,
+// so the bf16 unembedding matrix streams from HBM exactly once per step while
+// the tiny H operand is re-read from L2.  Persistent CTAs, one per SM:
+//   warp 0  TMA producer (W tile 128x64 + H slab S_pad x 64 per stage, 128B swizzle)
+//   warp 1  TMEM allocator and single-thread tcgen05.mma issuer (fp32 accumulators
+//           in TMEM, double-buffered when 2*S_pad <= 512 columns)
+//   warps 2-5 epilogue: tcgen05.ld of the 128 x S accumulator; per column the tile's
+//           (max, sum exp) for the log-softmax and, for each contextual expert k of
+//           query b, the tile's max and argmax of u_k(v) = (1+beta_k) z_k(v) - beta_k z_0(v).
+// Because shat_k(v) = u_k(v) + c_k with c_k = -(1+beta_k) L_k + beta_k L_0 + gamma log r_k
+// constant in v, Eq. 3 only needs these per-tile maxima and the log-sum-exps L:
+// the [S x V] logits never reach HBM on the fused path.
+#include <math.h>
+
+#include "lm_head.cuh"
+
+namespace pced {
+
+constexpr int LM_A_BYTES = LM_TILE_V * LM_TILE_K * 2;  // 16 KB
+constexpr size_t LM_SMEM_BUDGET = 227 * 1024;
+
+bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
+  if (S < 1 || S > LM_MAX_S || d < LM_TILE_K || d % LM_TILE_K != 0 || V < 1) return false;
+  g->S = S;
+  g->d = d;
+  g->V = V;
+  g->nchunk = (S + 255) / 256;
+  const int per = (S + g->nchunk - 1) / g->nchunk;
+  g->chunk_n = ((per < 16 ? 16 : per) + 15) / 16 * 16;
+  g->S_pad = g->nchunk * g->chunk_n;
+  if (g->S_pad > 512) return false;
+  g->acc_bufs = 2 * g->S_pad <= 512 ? 2 : 1;
+  uint32_t cols = 32;
+  while (cols < (uint32_t)(g->acc_bufs * g->S_pad)) cols <<= 1;
+  g->tmem_cols = cols;
+  g->ntiles = (V + LM_TILE_V - 1) / LM_TILE_V;
+  g->nks = d / LM_TILE_K;
+  const size_t stage = LM_A_BYTES + (size_t)g->S_pad * 128;
+  const size_t fixed = 1024 + 64 * 8 + 16 + (size_t)2 * 4 * g->S_pad * sizeof(float2);
+  int st = (int)((LM_SMEM_BUDGET - fixed) / stage);
+  if (st > 8) st = 8;
+  if (st < 2) return false;
+  g->stages = st;
+  g->smem = fixed + (size_t)st * stage;
+  int sms = pced_host::num_sms();
+  g->grid = g->ntiles < sms ? g->ntiles : sms;
+  if (g->grid < 1) g->grid = 1;
+  return true;
+}
+
+__global__ void __launch_bounds__(LM_THREADS, 1)
+    lm_head_kernel(const __grid_constant__ CUtensorMap wmap, const __grid_constant__ CUtensorMap hmap, LmArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t b_bytes = (uint32_t)a.S_pad * 128u;
+  const uint32_t st_bytes = LM_A_BYTES + b_bytes;
+  const int stages = a.stages;
+  // layout: stages | full | empty | tfull[2] | tempty[2] | epi | drain | tmem slot | scratch
+  const uint32_t bar_full = base + stages * st_bytes;
+  const uint32_t bar_empty = bar_full + 8 * stages;
+  const uint32_t bar_tfull = bar_empty + 8 * stages;
+  const uint32_t bar_tempty = bar_tfull + 16;
+  const uint32_t bar_epi = bar_tempty + 16;
+  const uint32_t bar_drain = bar_epi + 8;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + (bar_drain + 8 - base));
+  float2* wst = reinterpret_cast<float2*>(gbase + (bar_drain + 8 - base) + 16);  // [4][S_pad]
+  float2* wag = wst + 4 * a.S_pad;                                                // [4][S_pad]
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int i = 0; i < stages; ++i) {
+      mbar_init(bar_full + 8 * i, 1);
+      mbar_init(bar_empty + 8 * i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar_tfull + 8 * i, 1);
+      mbar_init(bar_tempty + 8 * i, 128);
+    }
+    mbar_init(bar_epi, 128);
+    mbar_init(bar_drain, 1);
+    mbar_fence_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&wmap);
+    tma_prefetch_desc(&hmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), a.tmem_cols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int ntiles = a.ntiles, nks = a.nks;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
+      uint32_t it = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+        for (int ks = 0; ks < nks; ++ks, ++it) {
+          const uint32_t st = it % stages, ph = (it / stages) & 1u;
+          if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = bar_full + 8 * st;
+          const uint32_t sa = base + st * st_bytes, sb = sa + LM_A_BYTES;
+          mbar_arrive_expect_tx(fb, st_bytes);
+          tma_load_2d(sa, &wmap, fb, ks * LM_TILE_K, tile * LM_TILE_V, pol_w);
+          for (int c = 0; c < a.nchunk; ++c)
+            tma_load_2d(sb + c * a.chunk_n * 128, &hmap, fb, ks * LM_TILE_K, c * a.chunk_n, pol_h);
+        }
+      }
+      if (!ok) {
+        for (uint32_t j = (it >= (uint32_t)stages ? it - stages : 0); j < it; ++j)
+          mbar_wait(bar_full + 8 * (j % stages), (j / stages) & 1u, a.status);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA
+    if (lane == 0) {
+      const uint32_t idesc = umma_idesc_bf16(LM_TILE_V, a.chunk_n);
+      uint32_t it = 0, acc = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++acc) {
+        const uint32_t buf = acc % a.acc_bufs, aph = (acc / a.acc_bufs) & 1u;
+        if (!mbar_wait(bar_tempty + 8 * buf, aph ^ 1u, a.status)) break;
+        tc_fence_after();
+        const uint32_t dcol = tmem_base + buf * a.S_pad;
+        for (int ks = 0; ks < nks; ++ks, ++it) {
+          const uint32_t st = it % stages, ph = (it / stages) & 1u;
+          if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = base + st * st_bytes, sb = sa + LM_A_BYTES;
+#pragma unroll
+          for (int k = 0; k < LM_TILE_K / 16; ++k) {
+            const uint64_t ad = umma_desc_sw128(sa + 32 * k);
+            for (int c = 0; c < a.nchunk; ++c)
+              umma_bf16(dcol + c * a.chunk_n, ad, umma_desc_sw128(sb + c * a.chunk_n * 128 + 32 * k), idesc,
+                        (ks | k) != 0);
+          }
+          umma_commit(bar_empty + 8 * st);
+        }
+        if (!ok) break;
+        umma_commit(bar_tfull + 8 * buf);
+      }
+      // all issued MMAs complete before TMEM is released
+      umma_commit(bar_drain);
+      mbar_wait(bar_drain, 0, a.status);
+    }
+    __syncwarp();
+  } else {
+    // ----------------------------------------------------------- epilogue
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int etid = tid - 64;
+    const int S = a.S, S_pad = a.S_pad, n1 = a.N + 1;
+    uint32_t acc = 0, ephase = 0;
+    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++acc) {
+      const uint32_t buf = acc % a.acc_bufs, aph = (acc / a.acc_bufs) & 1u;
+      if (!mbar_wait(bar_tfull + 8 * buf, aph, a.status)) break;
+      tc_fence_after();
+      const int v = tile * LM_TILE_V + 32 * q + lane;
+      const bool valid = v < a.V;
+      const uint32_t trow = tmem_base + ((uint32_t)(32 * q) << 16) + buf * S_pad;
+      float z_am = 0.f;
+      for (int cb = 0; cb < S_pad / 16; ++cb) {
+        float vals[16];
+        tmem_ld16(trow + cb * 16, vals);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int col = cb * 16 + i;
+          if (col >= S) break;
+          const float z = valid ? vals[i] : -INFINITY;
+          if (a.mode == 0 && valid) a.logits[(int64_t)col * a.V + v] = z;
+          const float mw = warp_max(z);
+          const float e = valid ? __expf(z - mw) : 0.f;
+          const float sw = warp_sum(e);
+          if (lane == 0) wst[q * S_pad + col] = make_float2(mw, sw);
+          if (a.mode == 1) {
+            const int j = col % n1;
+            if (j == 0) {
+              z_am = vals[i];
+            } else {
+              const int b = col / n1;
+              const float bt = a.beta[b * a.N + j - 1];
+              float u = valid ? (1.f + bt) * vals[i] - bt * z_am : -INFINITY;
+              int vi = v;
+              warp_argmax(u, vi);
+              if (lane == 0) wag[q * S_pad + col] = make_float2(u, __int_as_float(vi));
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(bar_tempty + 8 * buf);
+      if (!bar_sync_bounded(bar_epi, ephase, a.status)) break;
+      for (int col = etid; col < S; col += 128) {
+        float M = -INFINITY, sum = 0.f;
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) {
+          const float2 r = wst[qq * S_pad + col];
+          lse_merge(M, sum, r.x, r.y);
+        }
+        a.rec_stats[(int64_t)col * ntiles + tile] = make_float2(M, sum);
+        if (a.mode == 1 && col % n1 != 0) {
+          float bu = -INFINITY;
+          int bv = 0x7fffffff;
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq) {
+            const float2 r = wag[qq * S_pad + col];
+            argmax_merge(bu, bv, r.x, __float_as_int(r.y));
+          }
+          a.rec_arg[(int64_t)col * ntiles + tile] = make_float2(bu, __int_as_float(bv));
+        }
+      }
+      if (!bar_sync_bounded(bar_epi, ephase, a.status)) break;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, a.tmem_cols);
+  }
+}
+
+cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, const LmGeom& g, const LmArgs& a,
+                           cudaStream_t stream) {
+  static size_t configured = 0;
+  if (configured < g.smem) {
+    cudaError_t e = cudaFuncSetAttribute(lm_head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)LM_SMEM_BUDGET);
+    if (e != cudaSuccess) return e;
+    configured = LM_SMEM_BUDGET;
+  }
+  lm_head_kernel<<<g.grid, LM_THREADS, g.smem, stream>>>(wmap, hmap, a);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------ mode-0 finish
+__global__ void __launch_bounds__(256) lm_lse_finalize_kernel(float* logits, const float2* rec_stats, float* lse,
+                                                              int32_t V, int32_t ntiles) {
+  const int s = blockIdx.x, tid = threadIdx.x;
+  __shared__ float2 red[8];
+  __shared__ float Ls;
+  float M = -INFINITY, sum = 0.f;
+  for (int t = tid; t < ntiles; t += 256) {
+    const float2 r = rec_stats[(int64_t)s * ntiles + t];
+    lse_merge(M, sum, r.x, r.y);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, M, o), s2 = __shfl_xor_sync(0xffffffffu, sum, o);
+    lse_merge(M, sum, m2, s2);
+  }
+  if ((tid & 31) == 0) red[tid >> 5] = make_float2(M, sum);
+  __syncthreads();
+  if (tid == 0) {
+    float m = -INFINITY, su = 0.f;
+    for (int w = 0; w < 8; ++w) lse_merge(m, su, red[w].x, red[w].y);
+    Ls = m + logf(su);
+    lse[s] = Ls;
+  }
+  __syncthreads();
+  const float L = Ls;
+  float* row = logits + (int64_t)s * V;
+  for (int v = tid; v < V; v += 256) row[v] -= L;
+}
+
+cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float* lse, int32_t S, int32_t V,
+                                   int32_t ntiles, cudaStream_t stream) {
+  lm_lse_finalize_kernel<<<S, 256, 0, stream>>>(logits, rec_stats, lse, V, ntiles);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------- Eq. 2 + Eq. 3 from tile records
+// Per query: L_j for its N+1 rows from the (max, sum) records; for each expert
+// k the best tile record of u_k; score_k = u_k* + c_k; the best (score desc,
+// token asc, expert asc) wins.
+__global__ void __launch_bounds__(256) select_from_records_kernel(SelectArgs a) {
+  const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int N = a.N, n1 = N + 1, s0 = b * n1, T = a.ntiles;
+  __shared__ float Ls[LM_MAX_N1];
+  __shared__ float ksc[LM_MAX_N1];
+  __shared__ int ktok[LM_MAX_N1];
+  __shared__ int t_step;
+  if (tid == 0) t_step = a.step ? *a.step : 0;
+  for (int j = warp; j < n1; j += 8) {
+    const int s = s0 + j;
+    float M = -INFINITY, sum = 0.f;
+    for (int t = lane; t < T; t += 32) {
+      const float2 r = a.rec_stats[(int64_t)s * T + t];
+      lse_merge(M, sum, r.x, r.y);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, M, o), s2 = __shfl_xor_sync(0xffffffffu, sum, o);
+      lse_merge(M, sum, m2, s2);
+    }
+    if (lane == 0) {
+      Ls[j] = M + logf(sum);
+      if (a.lse_out) a.lse_out[s] = Ls[j];
+    }
+  }
+  __syncthreads();
+  for (int k = 1 + warp; k <= N; k += 8) {
+    const int s = s0 + k;
+    float bu = -INFINITY;
+    int bv = 0x7fffffff;
+    for (int t = lane; t < T; t += 32) {
+      const float2 r = a.rec_arg[(int64_t)s * T + t];
+      argmax_merge(bu, bv, r.x, __float_as_int(r.y));
+    }
+    warp_argmax(bu, bv);
+    if (lane == 0) {
+      const float bt = a.beta[b * N + k - 1];
+      const float rr = fminf(fmaxf(a.r[b * N + k - 1], 1e-8f), 1.0f);
+      const float c = -(1.f + bt) * Ls[k] + bt * Ls[0] + a.gamma * logf(rr);
+      ksc[k - 1] = bu + c;
+      ktok[k - 1] = bv;
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    float bs = -INFINITY;
+    int bt = 0x7fffffff, bk = 0x7fffffff;
+    for (int k = lane; k < N; k += 32) {
+      const float sc = ksc[k];
+      const int tk = ktok[k];
+      if (sc > bs || (sc == bs && (tk < bt || (tk == bt && k < bk)))) {
+        bs = sc;
+        bt = tk;
+        bk = k;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float s2 = __shfl_xor_sync(0xffffffffu, bs, o);
+      const int t2 = __shfl_xor_sync(0xffffffffu, bt, o), k2 = __shfl_xor_sync(0xffffffffu, bk, o);
+      if (s2 > bs || (s2 == bs && (t2 < bt || (t2 == bt && k2 < bk)))) {
+        bs = s2;
+        bt = t2;
+        bk = k2;
+      }
+    }
+    if (lane == 0) {
+      if (a.token) a.token[b] = bt;
+      if (a.expert) a.expert[b] = bk + 1;
+      if (a.score) a.score[b] = bs;
+      if (a.step) {
+        const int t = t_step;
+        if (t >= 0 && t < a.max_steps) {
+          a.history[(int64_t)b * a.max_steps + t] = bt;
+          if (a.expert_trace) a.expert_trace[(int64_t)b * a.max_steps + t] = bk + 1;
+          if (a.score_trace) a.score_trace[(int64_t)b * a.max_steps + t] = bs;
+        } else {
+          dev_flag(a.status, PCED_DEV_STEP_LIMIT);
+        }
+        __threadfence();
+        if (atomicAdd(a.done_counter, 1) == a.B - 1) {
+          *a.step = t + 1;
+          *a.done_counter = 0;
+          __threadfence();
+        }
+      }
+    }
+  }
+}
+
+cudaError_t select_from_records_launch(const SelectArgs& a, cudaStream_t stream) {
+  select_from_records_kernel<<<a.B, 256, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace pced
+
+// ------------------------------------------------------------------ C ABI
+using namespace pced;
+using namespace pced_host;
+
+extern "C" size_t pced_lm_head_workspace_size(int32_t S, int32_t V) {
+  if (S < 1 || V < 1) return 0;
+  const int64_t ntiles = (V + LM_TILE_V - 1) / LM_TILE_V;
+  Carver c(nullptr);
+  c.take<float2>((size_t)(S * ntiles));
+  return 256 + c.used();
+}
+
+extern "C" pced_status pced_lm_head_logprobs(const void* hidden, const void* w_unembed, int32_t S, int32_t d,
+                                             int32_t V, float* logprobs, float* lse, void* workspace,
+                                             size_t workspace_bytes, void* stream) {
+  if (!hidden || !w_unembed || !logprobs || !lse || !workspace)
+    return fail(PCED_ERR_INVALID_ARG, "pced_lm_head_logprobs: null pointer");
+  if (S < 1 || d < 1 || V < 1) return fail(PCED_ERR_INVALID_ARG, "pced_lm_head_logprobs: bad sizes");
+  LmGeom g;
+  if (!lm_geometry(S, d, V, &g) || d > 16384)
+    return fail(PCED_ERR_UNSUPPORTED, "pced_lm_head_logprobs: S=%d d=%d (need S<=512, d%%64==0, d<=16384)", S, d);
+  if ((((uintptr_t)hidden) | ((uintptr_t)w_unembed)) & 15u)
+    return fail(PCED_ERR_INVALID_ARG, "pced_lm_head_logprobs: operands must be 16-byte aligned");
+  if (((uintptr_t)workspace) & 255u || workspace_bytes < pced_lm_head_workspace_size(S, V))
+    return fail(PCED_ERR_WORKSPACE, "pced_lm_head_logprobs: workspace too small or misaligned");
+  if (num_sms() <= 0) return fail(PCED_ERR_NO_DEVICE, "pced_lm_head_logprobs: no CUDA device");
+  CUtensorMap wmap, hmap;
+  pced_status st = make_tmap_2d(&wmap, w_unembed, (uint64_t)V, (uint64_t)d, LM_TILE_V, LM_TILE_K, true);
+  if (st != PCED_OK) return st;
+  st = make_tmap_2d(&hmap, hidden, (uint64_t)S, (uint64_t)d, (uint32_t)g.chunk_n, LM_TILE_K, false);
+  if (st != PCED_OK) return st;
+  Carver cv((char*)workspace + 256);
+  LmArgs a = {};
+  a.mode = 0;
+  a.S = S;
+  a.N = 0;
+  a.V = V;
+  a.ntiles = g.ntiles;
+  a.nks = g.nks;
+  a.stages = g.stages;
+  a.acc_bufs = g.acc_bufs;
+  a.S_pad = g.S_pad;
+  a.nchunk = g.nchunk;
+  a.chunk_n = g.chunk_n;
+  a.tmem_cols = g.tmem_cols;
+  a.logits = logprobs;
+  a.rec_stats = cv.take<float2>((size_t)S * g.ntiles);
+  a.rec_arg = nullptr;
+  a.beta = nullptr;
+  a.status = (int*)workspace;
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = lm_head_launch(wmap, hmap, g, a, s);
+  if (e != cudaSuccess) return cuda_status(e, "lm head launch");
+  e = lm_lse_finalize_launch(logprobs, a.rec_stats, lse, S, V, g.ntiles, s);
+  if (e != cudaSuccess) return cuda_status(e, "lse finalize launch");
+  return PCED_OK;
+}

@@ -1,0 +1,62 @@
+// lm_head.cuh -- unembedding GEMM with fused log-softmax statistics and the
+// contrastive per-tile maxima, plus the cross-tile reductions.
+#pragma once
+#include "common.cuh"
+
+namespace pced {
+
+constexpr int LM_THREADS = 192;  // warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-5 epilogue
+constexpr int LM_TILE_V = 128;   // vocabulary rows per tile (UMMA M)
+constexpr int LM_TILE_K = 64;    // hidden elements per stage (one 128-byte swizzle row)
+constexpr int LM_MAX_S = 512;
+constexpr int LM_MAX_N1 = 256;   // experts + amateur per query in the selection kernels
+
+struct LmGeom {
+  int32_t S, S_pad, nchunk, chunk_n, d, V, ntiles, nks, stages, acc_bufs, grid;
+  uint32_t tmem_cols;
+  size_t smem;
+};
+// returns false when the shape is unsupported
+bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g);
+
+struct LmArgs {
+  int mode;  // 0: write logits[S][V]; 1: contrastive tile records (needs N, beta)
+  int32_t S, N, V, ntiles, nks, stages, acc_bufs, S_pad, nchunk, chunk_n;
+  uint32_t tmem_cols;
+  float* logits;      // mode 0
+  float2* rec_stats;  // [S][ntiles] (max z, sum exp(z - max)) of each tile
+  float2* rec_arg;    // [S][ntiles] (max u, argmax v as int bits) for expert columns, mode 1
+  const float* beta;  // [B][N]
+  int* status;
+};
+
+cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, const LmGeom& g, const LmArgs& a,
+                           cudaStream_t stream);
+// mode-0 finish: lse[s] from the tile records, logits -> log-probs in place
+cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float* lse, int32_t S, int32_t V,
+                                   int32_t ntiles, cudaStream_t stream);
+
+// Selection from mode-1 records (Eq. 2 + Eq. 3), one CTA per query.
+struct SelectArgs {
+  const float2* rec_stats;
+  const float2* rec_arg;
+  int32_t B, N, ntiles;
+  const float* beta;
+  const float* r;
+  float gamma;
+  int32_t* token;     // optional [B]
+  int32_t* expert;    // optional [B]
+  float* score;       // optional [B]
+  float* lse_out;     // optional [S]
+  // step bookkeeping (optional): history[b][t] etc. with t = *step, then *step += 1
+  int32_t* step;
+  int32_t* history;
+  int32_t* expert_trace;
+  float* score_trace;
+  int32_t max_steps;
+  int32_t* done_counter;
+  int* status;
+};
+cudaError_t select_from_records_launch(const SelectArgs& a, cudaStream_t stream);
+
+}  // namespace pced

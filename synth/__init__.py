@@ -328,3 +328,38 @@ def dev_fill_matrix(w: Workload, tensor: int, out, stream_ptr, row0: int = 0, ro
                                          normal_scale(sigma), stream_ptr)
     if rc != 0:
         raise RuntimeError(f"synth_dev_fill_matrix failed: cuda error {rc}")
+
+
+T_MISC = 9
+
+
+def host_normal_bf16(n: int, seed: int, sigma: float = 1.0) -> np.ndarray:
+    """n bf16 samples (bit patterns) of an auxiliary stream, for test operands."""
+    out = np.empty(n, dtype=np.uint16)
+    host_lib().synth_fill_matrix(_ptr(out), 0, 1, n, seed, T_MISC, normal_scale(sigma), _threads())
+    return out
+
+
+def device_inputs(w: Workload, device="cuda", extra_steps: int | None = None, stream=None) -> dict:
+    """All inputs of workload `w` as device tensors: caches with generated
+    prefixes (zeros after), embedding, unembedding, lengths, layout tables,
+    beta and r.  Generated on the device with the same bits as the host fills."""
+    import torch
+    stream = torch.cuda.current_stream() if stream is None else stream
+    sp = stream.cuda_stream
+    bl = base_lengths(w)
+    lay = cache_layout(w, bl, extra_steps)
+    k = torch.zeros(lay.total_elems, dtype=torch.bfloat16, device=device)
+    v = torch.zeros(lay.total_elems, dtype=torch.bfloat16, device=device)
+    kv_off = torch.from_numpy(lay.kv_offset).to(device)
+    cap = torch.from_numpy(lay.cap).to(device)
+    base = torch.from_numpy(bl).to(device)
+    ids = torch.arange(w.S, dtype=torch.int32, device=device)
+    dev_fill_caches(w, lay.layer_elems, k, v, kv_off, cap, base, ids, sp)
+    emb = torch.empty((w.V, w.d), dtype=torch.bfloat16, device=device)
+    wu = torch.empty((w.V, w.d), dtype=torch.bfloat16, device=device)
+    dev_fill_matrix(w, T_EMBED, emb, sp)
+    dev_fill_matrix(w, T_UNEMBED, wu, sp)
+    return dict(k_cache=k, v_cache=v, kv_offset=kv_off, cap=cap, seq_len=base.clone(), base_len=bl, layout=lay,
+                embed=emb, w_unembed=wu, beta=torch.from_numpy(betas(w)).to(device),
+                r=torch.from_numpy(retrieval_scores(w)).to(device))
