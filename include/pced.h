@@ -168,6 +168,13 @@ typedef struct pced_step_args {
   float* lse_out;           /* optional fp32 [S]: log-sum-exp of each row of h W^T */
   void* workspace;
   size_t workspace_bytes;
+  /* Optional timing hooks: an array of pced_step_launch_count(&dims) + 1
+   * cudaEvent_t handles (cast to void*).  Event 0 is recorded on `stream`
+   * before the first launch and event i+1 right after launch i, so the time
+   * between consecutive events is the device time of that launch.  NULL (or
+   * fewer events) disables recording. */
+  void* const* stage_events;
+  int32_t n_stage_events;
 } pced_step_args;
 
 size_t pced_step_workspace_size(const pced_dims* dims);
@@ -175,6 +182,9 @@ pced_status pced_step(const pced_step_args* args, void* stream);
 
 /* Number of kernel launches one pced_step call makes for these dimensions. */
 int32_t pced_step_launch_count(const pced_dims* dims);
+/* Kind of launch i of pced_step (0-based): "embed", "attn_split",
+ * "attn_combine", "lm_head" or "select"; NULL when out of range (static storage). */
+const char* pced_step_launch_kind(const pced_dims* dims, int32_t i);
 
 #ifdef __cplusplus
 }

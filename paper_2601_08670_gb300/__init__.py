@@ -43,7 +43,8 @@ class StepArgs(ctypes.Structure):
                 ("beta", ctypes.c_void_p), ("r", ctypes.c_void_p), ("gamma", ctypes.c_float),
                 ("attn_scale", ctypes.c_float), ("rms_eps", ctypes.c_float), ("bos_token", ctypes.c_int32),
                 ("hidden_out", ctypes.c_void_p), ("lse_out", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
-                ("workspace_bytes", ctypes.c_size_t)]
+                ("workspace_bytes", ctypes.c_size_t), ("stage_events", ctypes.c_void_p),
+                ("n_stage_events", ctypes.c_int32)]
 
 
 _lib = None
@@ -79,6 +80,8 @@ def lib(path: str = LIB_PATH):
         L.pced_step.restype = I32
         L.pced_step_launch_count.argtypes = [ctypes.POINTER(Dims)]
         L.pced_step_launch_count.restype = I32
+        L.pced_step_launch_kind.argtypes = [ctypes.POINTER(Dims), I32]
+        L.pced_step_launch_kind.restype = ctypes.c_char_p
         _lib = L
     return _lib
 
@@ -179,6 +182,10 @@ def step_launch_count(dm: Dims) -> int:
     return int(lib().pced_step_launch_count(ctypes.byref(dm)))
 
 
+def step_launch_kinds(dm: Dims) -> list:
+    return [lib().pced_step_launch_kind(ctypes.byref(dm), i).decode() for i in range(step_launch_count(dm))]
+
+
 class Decoder:
     """Device-resident PCED decoding state and the pced_step call.
 
@@ -212,6 +219,23 @@ class Decoder:
 
     def step(self, stream=None):
         _check(lib().pced_step(ctypes.byref(self.args), _stream(stream)), "pced_step")
+
+    def set_stage_events(self, events):
+        """Record one torch.cuda.Event before and after every launch of each
+        subsequent step (None disables)."""
+        if events is None:
+            self._events = None
+            self.args.stage_events = None
+            self.args.n_stage_events = 0
+            return
+        for ev in events:  # torch creates the CUDA event on its first record
+            if ev.cuda_event == 0:
+                ev.record()
+        torch.cuda.synchronize()
+        self._events = events
+        self._event_handles = (ctypes.c_void_p * len(events))(*[ev.cuda_event for ev in events])
+        self.args.stage_events = ctypes.cast(self._event_handles, ctypes.c_void_p)
+        self.args.n_stage_events = len(events)
 
     def launches_per_step(self) -> int:
         return step_launch_count(self.dm)

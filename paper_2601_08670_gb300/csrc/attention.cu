@@ -30,13 +30,13 @@ struct AttCfg {
   static constexpr int BOX_BYTES = ATT_BLOCK_N * 128;   // 64 rows x 128 B
   static constexpr int TILE_BYTES = BOXES * BOX_BYTES;  // K (or V) part of a stage
   static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
-  static constexpr int STAGES = D == 128 ? 5 : 8;
+  static constexpr int STAGES = D == 128 ? 5 : 7;       // odd: consecutive uses of a stage alternate warpgroups
   static constexpr int KSTEPS = D / 16;
   static constexpr int MTILES = D / 16;
   static constexpr int OPAD = 9;  // padded head stride of the merge scratch
   static constexpr int MERGE_FLOATS = 2 * ATT_CONSUMERS * ATT_MAX_G + ATT_CONSUMERS * D * OPAD;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + (2 * STAGES + 1) * 8 + (size_t)MERGE_FLOATS * 4 +
-                                 (ATT_MAX_S + 1) * 8 + ATT_MAX_S * 4 + 128;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + (2 * STAGES + 1) * 8 +
+                                 (size_t)MERGE_FLOATS * 4 + (ATT_MAX_S + 1) * 8 + ATT_MAX_S * 4 + 128;
 };
 
 struct Piece {
@@ -45,24 +45,35 @@ struct Piece {
 
 // (sequence, head, key range) of the piece that starts at global position p
 // and ends at the next segment boundary or at `end`.
-__device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* lens, int32_t S, int64_t p,
+__device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* lens, int32_t S, int64_t T, int64_t p,
                                             int64_t end) {
+  Piece pc;
+  pc.h = (int32_t)(p / T);
+  const int64_t r = p - (int64_t)pc.h * T;
   int32_t lo = 0, hi = S - 1;
   while (lo < hi) {
-    int32_t mid = (lo + hi + 1) >> 1;
-    if (pre[mid] <= p) lo = mid;
+    const int32_t mid = (lo + hi + 1) >> 1;
+    if (pre[mid] <= r) lo = mid;
     else hi = mid - 1;
   }
-  Piece pc;
   pc.s = lo;
-  const int64_t off = p - pre[lo];
-  const int32_t len = lens[lo];
-  pc.h = (int32_t)(off / len);
-  pc.k0 = (int32_t)(off - (int64_t)pc.h * len);
-  const int64_t seg_end = pre[lo] + (int64_t)(pc.h + 1) * len;
+  pc.k0 = (int32_t)(r - pre[lo]);
+  const int64_t seg_end = (int64_t)pc.h * T + pre[lo] + lens[lo];
   const int64_t e = seg_end < end ? seg_end : end;
   pc.k1 = pc.k0 + (int32_t)(e - p);
   return pc;
+}
+
+template <int KSTEPS>
+__device__ __forceinline__ void load_q_frag(uint32_t (&qf)[KSTEPS][2], const AttArgs& a, const Piece& pc, int g,
+                                            int tq, int D) {
+  const bool hv = g < a.G;
+  const __nv_bfloat16* qrow = a.q + ((int64_t)pc.s * a.Hq + (int64_t)pc.h * a.G + (hv ? g : 0)) * D;
+#pragma unroll
+  for (int j = 0; j < KSTEPS; ++j) {
+    qf[j][0] = hv ? *reinterpret_cast<const uint32_t*>(qrow + 16 * j + 2 * tq) : 0u;
+    qf[j][1] = hv ? *reinterpret_cast<const uint32_t*>(qrow + 16 * j + 8 + 2 * tq) : 0u;
+  }
 }
 
 template <int D>
@@ -78,19 +89,19 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   const uint32_t bar_empty = bar_full + C::STAGES * 8;
   const uint32_t bar_merge = bar_empty + C::STAGES * 8;
   float* mscr = reinterpret_cast<float*>(gbase + C::STAGES * C::STAGE_BYTES + (2 * C::STAGES + 1) * 8);
-  float* ms = mscr;                                  // [4][8]
-  float* ls = mscr + ATT_CONSUMERS * ATT_MAX_G;      // [4][8]
-  float* os = mscr + 2 * ATT_CONSUMERS * ATT_MAX_G;  // [4][D][OPAD]
+  float* ms = mscr;                                  // [8][8]
+  float* ls = mscr + ATT_CONSUMERS * ATT_MAX_G;      // [8][8]
+  float* os = mscr + 2 * ATT_CONSUMERS * ATT_MAX_G;  // [8][D][OPAD]
   int64_t* pre = reinterpret_cast<int64_t*>(mscr + C::MERGE_FLOATS);
   int32_t* lens = reinterpret_cast<int32_t*>(pre + ATT_MAX_S + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int32_t S = a.S, Hkv = a.Hkv, G = a.G;
+  const int32_t S = a.S, G = a.G;
 
   if (tid == 0) {
     for (int i = 0; i < C::STAGES; ++i) {
       mbar_init(bar_full + 8 * i, 1);
-      mbar_init(bar_empty + 8 * i, ATT_CONSUMERS);
+      mbar_init(bar_empty + 8 * i, 4);  // one warpgroup consumes each stage
     }
     mbar_init(bar_merge, ATT_CONSUMERS * 32);
     mbar_fence_init();
@@ -109,26 +120,27 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
     lens[i] = L;
   }
   __syncthreads();
-  if (warp == 0) {  // exclusive prefix of Hkv * len
+  if (warp == 0) {  // exclusive prefix of len
     const int chunk = (S + 31) / 32;
     const int b0 = lane * chunk, b1 = min(S, b0 + chunk);
     int64_t sum = 0;
-    for (int i = b0; i < b1; ++i) sum += (int64_t)lens[i] * Hkv;
+    for (int i = b0; i < b1; ++i) sum += lens[i];
     int64_t incl = sum;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      int64_t v = __shfl_up_sync(0xffffffffu, incl, o);
+      const int64_t v = __shfl_up_sync(0xffffffffu, incl, o);
       if (lane >= o) incl += v;
     }
     int64_t run = incl - sum;
     for (int i = b0; i < b1; ++i) {
       pre[i] = run;
-      run += (int64_t)lens[i] * Hkv;
+      run += lens[i];
     }
     if (lane == 31) pre[S] = incl;
   }
   __syncthreads();
-  const int64_t total = pre[S];
+  const int64_t T = pre[S];
+  const int64_t total = T * a.Hkv;
   const int64_t per = (total + gridDim.x - 1) / gridDim.x;
   if (blockIdx.x == 0) {
     for (int i = tid; i <= S; i += ATT_THREADS) a.plan_pre[i] = pre[i];
@@ -144,7 +156,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int64_t p = r_begin; p < r_end && ok;) {
-        const Piece pc = find_piece(pre, lens, S, p, r_end);
+        const Piece pc = find_piece(pre, lens, S, T, p, r_end);
         const int64_t slab_row = a.row_base + (a.kv_offset[pc.s] + (int64_t)pc.h * a.cap[pc.s] * D) / D;
         for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
           const uint32_t st = it % C::STAGES, ph = (it / C::STAGES) & 1u;
@@ -174,41 +186,52 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   }
 
   // -------------------------------------------------------------- consumers
-  const int g = lane >> 2, tq = lane & 3;  // mma group id / thread in group
+  const int wg = warp >> 2, wl = warp & 3;  // warpgroup, warp within the group
+  const int g = lane >> 2, tq = lane & 3;   // mma group id / thread in group
   const int mat = lane >> 3, mr = lane & 7;
+  const int kb = 16 * wl;                   // first key of this warp's slice of a tile
   uint32_t it = 0, mphase = 0;
   bool ok = true;
+  uint32_t qn[C::KSTEPS][2];
+  if (r_begin < r_end) load_q_frag<C::KSTEPS>(qn, a, find_piece(pre, lens, S, T, r_begin, r_end), g, tq, D);
   for (int64_t p = r_begin; p < r_end && ok;) {
-    const Piece pc = find_piece(pre, lens, S, p, r_end);
+    const Piece pc = find_piece(pre, lens, S, T, p, r_end);
     p += pc.k1 - pc.k0;
-    // B operand of S^T = K Q^T: rows = head dim, cols = the G query heads
+    // B operand of S^T = K Q^T (rows: head dim, cols: the G query heads);
+    // the next piece's query is fetched now so its latency overlaps this piece
     uint32_t qf[C::KSTEPS][2];
-    {
-      const bool hv = g < G;
-      const __nv_bfloat16* qrow = a.q + ((int64_t)pc.s * a.Hq + (int64_t)pc.h * G + (hv ? g : 0)) * D;
 #pragma unroll
-      for (int j = 0; j < C::KSTEPS; ++j) {
-        qf[j][0] = hv ? *reinterpret_cast<const uint32_t*>(qrow + 16 * j + 2 * tq) : 0u;
-        qf[j][1] = hv ? *reinterpret_cast<const uint32_t*>(qrow + 16 * j + 8 + 2 * tq) : 0u;
-      }
+    for (int j = 0; j < C::KSTEPS; ++j) {
+      qf[j][0] = qn[j][0];
+      qf[j][1] = qn[j][1];
     }
+    if (p < r_end) load_q_frag<C::KSTEPS>(qn, a, find_piece(pre, lens, S, T, p, r_end), g, tq, D);
+
     float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
     float o[C::MTILES][4];
 #pragma unroll
     for (int i = 0; i < C::MTILES; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
 
     for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
-      const uint32_t st = it % C::STAGES, ph = (it / C::STAGES) & 1u;
+      if ((int)(it & 1u) != wg) continue;
+      const uint32_t use = it / C::STAGES, st = it % C::STAGES, ph = use & 1u;
+      // Consecutive uses of a stage belong to different warpgroups.  Waiting for
+      // the release of the previous use first guarantees that the full barrier
+      // has completed that use's phase, so the parity test below refers to this
+      // tile's phase and not to the older one with the same parity.
+      if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status)) {
+        ok = false;
+        break;
+      }
       if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
         ok = false;
         break;
       }
       const int nvalid = min(ATT_BLOCK_N, pc.k1 - kt);
-      const int kb = 16 * warp;  // first key of this warp's slice
       if (kb < nvalid) {
         const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
-        // ---- scores S^T (16 keys x 8 heads)
-        float sc[4] = {0.f, 0.f, 0.f, 0.f};
+        // ---- scores S^T (16 keys x 8 heads), two independent accumulation chains
+        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
         {
           const int key = kb + (mat & 1) * 8 + mr;
           const uint32_t rowa = sk + key * 128;
@@ -219,14 +242,14 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
             const uint32_t addr = rowa + (chunk >> 3) * C::BOX_BYTES + (((chunk & 7) ^ sw) << 4);
             uint32_t a0, a1, a2, a3;
             ldsm_x4(addr, a0, a1, a2, a3);
-            mma_bf16(sc, a0, a1, a2, a3, qf[j][0], qf[j][1]);
+            mma_bf16((j & 1) ? sb : sa, a0, a1, a2, a3, qf[j][0], qf[j][1]);
           }
         }
         const bool v0 = kb + g < nvalid, v1 = kb + g + 8 < nvalid;
-        const float s0 = v0 ? sc[0] * a.scale_log2 : -INFINITY;
-        const float s1 = v0 ? sc[1] * a.scale_log2 : -INFINITY;
-        const float s2 = v1 ? sc[2] * a.scale_log2 : -INFINITY;
-        const float s3 = v1 ? sc[3] * a.scale_log2 : -INFINITY;
+        const float s0 = v0 ? (sa[0] + sb[0]) * a.scale_log2 : -INFINITY;
+        const float s1 = v0 ? (sa[1] + sb[1]) * a.scale_log2 : -INFINITY;
+        const float s2 = v1 ? (sa[2] + sb[2]) * a.scale_log2 : -INFINITY;
+        const float s3 = v1 ? (sa[3] + sb[3]) * a.scale_log2 : -INFINITY;
         float x0 = fmaxf(s0, s2), x1 = fmaxf(s1, s3);
 #pragma unroll
         for (int off = 4; off < 32; off <<= 1) {
@@ -285,7 +308,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
     }
     if (!ok) break;
 
-    // ---- merge the four warps' partials of this piece and write the record
+    // ---- merge the eight warps' partials of this piece and write the record
 #pragma unroll
     for (int off = 4; off < 32; off <<= 1) {
       l0 += __shfl_xor_sync(0xffffffffu, l0, off);
@@ -307,7 +330,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       ow[d1 * C::OPAD + 2 * tq + 1] = o[i][3];
     }
     if (!bar_sync_bounded(bar_merge, mphase, a.status)) break;
-    const int64_t slot = (int64_t)blockIdx.x + (int64_t)pc.s * Hkv + pc.h;
+    const int64_t slot = (int64_t)blockIdx.x + (int64_t)pc.h * S + pc.s;
     for (int idx = tid; idx < G * D; idx += ATT_CONSUMERS * 32) {
       const int hh = idx / D, dd = idx - hh * D;
       float M = -INFINITY;
@@ -330,67 +353,114 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
 }
 
 // ------------------------------------------------------------------ combine
-constexpr int CMB_THREADS = 256;
-constexpr int CMB_MAX_PER_THREAD = 32;  // d <= 8192
+// One CTA per (kv-head h, sequence s): weights of the records that cover the
+// segment are formed once in shared memory, then every output element sums
+// its records with independent loads.
+constexpr int CMB_THREADS = 128;
+constexpr int CMB_SLOTS = 64;                        // records weighted per pass
+constexpr int CMB_PER_THREAD = ATT_MAX_G * 128 / CMB_THREADS;  // G*D <= 1024 outputs per CTA
 
 __global__ void __launch_bounds__(CMB_THREADS) att_combine_kernel(CombineArgs a) {
-  const int s = blockIdx.x, tid = threadIdx.x;
-  const int32_t Hq = a.Hq, Hkv = a.Hkv, G = a.G, D = a.D, d = Hq * D;
+  const int h = blockIdx.x, s = blockIdx.y, tid = threadIdx.x;
+  const int32_t Hq = a.Hq, Hkv = a.Hkv, G = a.G, D = a.D, S = a.S, d = Hq * D;
+  __shared__ float wts[CMB_SLOTS][ATT_MAX_G];
+  __shared__ float red[CMB_THREADS / 32];
+  __shared__ int last;
   const int64_t per = *a.plan_per;
+  const int64_t T = a.plan_pre[S];
   const int64_t pre_s = a.plan_pre[s];
-  const int64_t len = (a.plan_pre[s + 1] - pre_s) / Hkv;
-  float xv[CMB_MAX_PER_THREAD];
-  float ss = 0.f;
-#pragma unroll
-  for (int j = 0; j < CMB_MAX_PER_THREAD; ++j) {
-    const int idx = tid + j * CMB_THREADS;
-    xv[j] = 0.f;
-    if (idx >= d) continue;
-    const int hq = idx / D, dd = idx - hq * D, h = hq / G, gh = hq - h * G;
-    const int64_t seg = (int64_t)s * Hkv + h;
-    const int64_t pa = pre_s + h * len, pb = pa + len;
-    const int64_t c0 = pa / per, c1 = (pb - 1) / per;
-    float M = -INFINITY;
-    for (int64_t c = c0; c <= c1; ++c) M = fmaxf(M, a.rec_ml[(c + seg) * G + gh].x);
-    float num = 0.f, den = 0.f;
+  const int64_t len = a.plan_pre[s + 1] - pre_s;
+  const int64_t seg = (int64_t)h * S + s;
+  const int64_t pa = (int64_t)h * T + pre_s;
+  const int64_t c0 = pa / per, c1 = (pa + len - 1) / per;
+  const int GD = G * D;
+
+  // global max and total of each head over all records of the segment
+  float Mh = -INFINITY, Lh = 0.f;
+  if (tid < G) {
+    for (int64_t c = c0; c <= c1; ++c) Mh = fmaxf(Mh, a.rec_ml[(c + seg) * G + tid].x);
     for (int64_t c = c0; c <= c1; ++c) {
-      const float2 ml = a.rec_ml[(c + seg) * G + gh];
-      if (ml.x == -INFINITY) continue;
-      const float e = exp2f(ml.x - M);
-      num += a.rec_o[((c + seg) * G + gh) * D + dd] * e;
-      den += ml.y * e;
+      const float2 ml = a.rec_ml[(c + seg) * G + tid];
+      if (ml.x != -INFINITY) Lh += ml.y * exp2f(ml.x - Mh);
     }
-    const float ov = num / den;
-    if (a.mode == 0) {
-      a.out[(int64_t)s * d + idx] = ov;
-    } else {
-      const float x = a.resid[(int64_t)s * d + idx] + ov;
-      a.resid[(int64_t)s * d + idx] = x;
-      xv[j] = x;
+  }
+  __shared__ float Msh[ATT_MAX_G], Lsh[ATT_MAX_G];
+  if (tid < G) {
+    Msh[tid] = Mh;
+    Lsh[tid] = Lh;
+  }
+  float acc[CMB_PER_THREAD];
+#pragma unroll
+  for (int j = 0; j < CMB_PER_THREAD; ++j) acc[j] = 0.f;
+  for (int64_t cb = c0; cb <= c1; cb += CMB_SLOTS) {
+    const int64_t rem = c1 + 1 - cb;
+    const int n = (int)(rem < CMB_SLOTS ? rem : CMB_SLOTS);
+    __syncthreads();
+    for (int i = tid; i < n * G; i += CMB_THREADS) {
+      const int ci = i / G, gh = i - ci * G;
+      const float2 ml = a.rec_ml[(cb + ci + seg) * G + gh];
+      wts[ci][gh] = ml.x == -INFINITY ? 0.f : exp2f(ml.x - Msh[gh]) / Lsh[gh];
+    }
+    __syncthreads();
+    for (int ci = 0; ci < n; ++ci) {
+      const float* ro = a.rec_o + (cb + ci + seg) * GD;
+#pragma unroll
+      for (int j = 0; j < CMB_PER_THREAD; ++j) {
+        const int idx = tid + j * CMB_THREADS;
+        if (idx < GD) acc[j] += wts[ci][idx / D] * ro[idx];
+      }
+    }
+  }
+  if (a.mode == 0) {
+#pragma unroll
+    for (int j = 0; j < CMB_PER_THREAD; ++j) {
+      const int idx = tid + j * CMB_THREADS;
+      if (idx < GD) a.out[(int64_t)s * d + (int64_t)h * GD + idx] = acc[j];
+    }
+    return;
+  }
+  // residual update of this CTA's heads and their sum of squares
+  float ss = 0.f;
+  float* xr = a.resid + (int64_t)s * d + (int64_t)h * GD;
+#pragma unroll
+  for (int j = 0; j < CMB_PER_THREAD; ++j) {
+    const int idx = tid + j * CMB_THREADS;
+    if (idx < GD) {
+      const float x = xr[idx] + acc[j];
+      xr[idx] = x;
       ss += x * x;
     }
   }
-  if (a.mode == 0) return;
-  // RMSNorm of the updated residual stream
-  __shared__ float red[CMB_THREADS / 32];
   ss = warp_sum(ss);
   if ((tid & 31) == 0) red[tid >> 5] = ss;
   __syncthreads();
-  if (tid < 32) {
-    float v = tid < CMB_THREADS / 32 ? red[tid] : 0.f;
-    v = warp_sum(v);
-    if (tid == 0) red[0] = v;
+  if (tid == 0) {
+    float t = 0.f;
+    for (int w = 0; w < CMB_THREADS / 32; ++w) t += red[w];
+    a.part_ss[(int64_t)s * Hkv + h] = t;
+    __threadfence();
+    const int prev = atomicAdd(&a.counters[s], 1);
+    last = prev == Hkv - 1;
+    if (last) a.counters[s] = 0;
   }
   __syncthreads();
-  const float inv = 1.0f / sqrtf(red[0] / (float)d + a.rms_eps);
+  if (!last) return;
+  // last CTA of sequence s: normalise the whole residual row (sums in head order)
+  __threadfence();
+  __shared__ float inv_sh;
+  if (tid == 0) {
+    float t = 0.f;
+    for (int hh = 0; hh < Hkv; ++hh) t += __ldcg(&a.part_ss[(int64_t)s * Hkv + hh]);
+    inv_sh = 1.0f / sqrtf(t / (float)d + a.rms_eps);
+  }
+  __syncthreads();
+  const float inv = inv_sh;
   const int32_t pos = a.seq_len[s] - 1;
   const int32_t capv = a.cap[s];
   const bool can_append = a.append && pos >= 0 && pos < capv;
-#pragma unroll
-  for (int j = 0; j < CMB_MAX_PER_THREAD; ++j) {
-    const int idx = tid + j * CMB_THREADS;
-    if (idx >= d) continue;
-    const __nv_bfloat16 u = __float2bfloat16_rn(xv[j] * inv);
+  const float* xs = a.resid + (int64_t)s * d;
+  for (int idx = tid; idx < d; idx += CMB_THREADS) {
+    const __nv_bfloat16 u = __float2bfloat16_rn(__ldcg(xs + idx) * inv);
     if (a.append) {
       a.q_next[(int64_t)s * d + idx] = u;
       if (can_append && idx < 2 * Hkv * D) {
@@ -449,7 +519,7 @@ cudaError_t att_split_launch(int D, const CUtensorMap& kmap, const CUtensorMap& 
 }
 
 cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream) {
-  att_combine_kernel<<<a.S, CMB_THREADS, 0, stream>>>(a);
+  att_combine_kernel<<<dim3(a.Hkv, a.S), CMB_THREADS, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
@@ -476,8 +546,7 @@ extern "C" pced_status pced_decode_attention(const void* q, const void* k_cache,
   if (D != 64 && D != 128) return fail(PCED_ERR_UNSUPPORTED, "pced_decode_attention: D=%d (supported: 64, 128)", D);
   if (Hq / Hkv > ATT_MAX_G) return fail(PCED_ERR_UNSUPPORTED, "pced_decode_attention: Hq/Hkv > %d", ATT_MAX_G);
   if (S > ATT_MAX_S) return fail(PCED_ERR_UNSUPPORTED, "pced_decode_attention: S > %d", ATT_MAX_S);
-  if (Hq * D > CMB_THREADS * CMB_MAX_PER_THREAD)
-    return fail(PCED_ERR_UNSUPPORTED, "pced_decode_attention: Hq*D > %d", CMB_THREADS * CMB_MAX_PER_THREAD);
+  if (Hq * D > 8192) return fail(PCED_ERR_UNSUPPORTED, "pced_decode_attention: Hq*D > 8192");
   if (cache_elems % D != 0 || cache_elems / D >= (int64_t)1 << 31)
     return fail(PCED_ERR_UNSUPPORTED, "pced_decode_attention: cache of %lld elements", (long long)cache_elems);
   if ((((uintptr_t)k_cache) | ((uintptr_t)v_cache)) & 15u)

@@ -6,25 +6,21 @@
 namespace pced {
 
 constexpr int ATT_BLOCK_N = 64;     // keys per pipeline stage
-constexpr int ATT_CONSUMERS = 4;    // consumer warps; warp w owns keys [16w, 16w+16) of every stage
+constexpr int ATT_CONSUMERS = 8;    // two warpgroups of four warps; warpgroup g takes the CTA's tiles with
+                                    // index = g (mod 2), warp w of a group owns keys [16w, 16w+16) of a tile
 constexpr int ATT_THREADS = (ATT_CONSUMERS + 1) * 32;
 constexpr int ATT_MAX_S = 1024;     // sequences per launch (prefix table lives in shared memory)
 constexpr int ATT_MAX_G = 8;        // query heads per kv-head (mma N = 8)
 constexpr int ATT_MAX_CTAS = 1024;  // upper bound of the grid (sizes the partial-record pool)
 
-// Partition of all (sequence, kv-head, key) positions into equal contiguous
+// Partition of all (kv-head, sequence, key) positions into equal contiguous
 // ranges, one per CTA.  Position of key k of kv-head h of sequence s:
-//   pre[s] + h * len[s] + k,   pre[s] = Hkv * sum_{s' < s} len[s'].
-// A CTA's range is cut into pieces at (s, h) boundaries; the partial result of
-// CTA c over segment seg = s*Hkv + h is stored in record slot c + seg (slots
-// are unique: each step along the position axis crosses either a CTA or a
-// segment boundary).
-struct AttPlan {
-  int64_t total;  // sum over segments of their lengths
-  int64_t per;    // keys per CTA (last CTA may get fewer)
-  int32_t ctas;
-};
-
+//   h * T + pre[s] + k,   pre[s] = sum_{s' < s} len[s'],  T = pre[S].
+// Head-major order spreads short segments (the amateurs) across CTAs.  A
+// CTA's range is cut into pieces at segment boundaries; the partial result of
+// CTA c over segment seg = h*S + s is stored in record slot c + seg (slots are
+// unique: each step along the position axis crosses a CTA boundary or a
+// segment boundary, or both).
 struct AttArgs {
   const __nv_bfloat16* q;     // [S][Hq][D]
   const int64_t* kv_offset;   // [S]
@@ -35,8 +31,8 @@ struct AttArgs {
   float scale_log2;           // softmax scale * log2(e)
   float* rec_o;               // [slots][G][D] unnormalised partial outputs
   float2* rec_ml;             // [slots][G] (running max in log2 units, sum of exp2)
-  int64_t* plan_pre;          // [S+1] written by CTA 0 (prefix of Hkv*len)
-  int64_t* plan_per;          // [1]   written by CTA 0
+  int64_t* plan_pre;          // [S+1] written by CTA 0 (prefix of len)
+  int64_t* plan_per;          // [1]   written by CTA 0: keys per CTA
   int* status;
 };
 
@@ -46,11 +42,12 @@ int att_grid(int64_t total_cap_keys);
 cudaError_t att_split_launch(int D, const CUtensorMap& kmap, const CUtensorMap& vmap, const AttArgs& a, int ctas,
                              cudaStream_t stream);
 
-// Combine partial records of one layer.
+// Combine the partial records of one layer; one CTA per (kv-head, sequence).
 //   mode 0: out[s][hq][dd] = o (fp32)
-//   mode 1: resid[s] += o; u = bf16(rmsnorm(resid[s])); then either write u to
-//           q_next and append K/V rows of layer `next_layer` at seq_len[s]-1,
-//           or (last layer) write u to hidden (and hidden_copy if non-null).
+//   mode 1: resid[s] += o for the CTA's heads; the last CTA of a sequence
+//           then forms u = bf16(rmsnorm(resid[s])) and either writes u to
+//           q_next and appends the next layer's K/V rows at seq_len[s]-1, or
+//           (last layer) writes u to hidden (and hidden_copy if non-null).
 struct CombineArgs {
   int mode;
   int32_t S, Hq, Hkv, G, D;
@@ -61,6 +58,8 @@ struct CombineArgs {
   const int32_t* seq_len;
   float* out;                 // mode 0
   float* resid;               // mode 1 [S][d]
+  float* part_ss;             // mode 1 [S][Hkv] partial sums of squares
+  int32_t* counters;          // mode 1 [S] arrival counters (zero between launches)
   float rms_eps;
   __nv_bfloat16* q_next;      // mode 1, not last layer
   __nv_bfloat16* hidden;      // mode 1, last layer

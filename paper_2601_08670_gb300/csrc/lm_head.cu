@@ -40,12 +40,24 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
   g->tmem_cols = cols;
   g->ntiles = (V + LM_TILE_V - 1) / LM_TILE_V;
   g->nks = d / LM_TILE_K;
-  const size_t stage = LM_A_BYTES + (size_t)g->S_pad * 128;
-  const size_t fixed = 1024 + 64 * 8 + 16 + (size_t)2 * 4 * g->S_pad * sizeof(float2);
+  g->nbeta = S;  // beta has B*N < S entries
+  const size_t slab = LM_A_BYTES + (size_t)g->S_pad * 128;
+  const size_t fixed = 1024 + 64 * 8 + 16 + (size_t)2 * 4 * g->S_pad * sizeof(float2) +
+                       (size_t)2 * g->S_pad * sizeof(float2) + (size_t)g->nbeta * 4 + 64;
+  // several consecutive K-slabs per stage so each row is fetched in longer runs;
+  // keep at least three stages in flight
+  g->slabs = 1;
+  for (int sl = 4; sl >= 2; sl >>= 1)
+    if (g->nks % sl == 0 && fixed + 3 * sl * slab <= LM_SMEM_BUDGET) {
+      g->slabs = sl;
+      break;
+    }
+  const size_t stage = (size_t)g->slabs * slab;
   int st = (int)((LM_SMEM_BUDGET - fixed) / stage);
   if (st > 8) st = 8;
   if (st < 2) return false;
   g->stages = st;
+  g->nst = g->nks / g->slabs;
   g->smem = fixed + (size_t)st * stage;
   int sms = pced_host::num_sms();
   g->grid = g->ntiles < sms ? g->ntiles : sms;
@@ -59,8 +71,9 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
-  const uint32_t b_bytes = (uint32_t)a.S_pad * 128u;
-  const uint32_t st_bytes = LM_A_BYTES + b_bytes;
+  const int SL = a.slabs, S_pad = a.S_pad;
+  const uint32_t b_bytes = (uint32_t)S_pad * 128u;
+  const uint32_t st_bytes = (uint32_t)SL * (LM_A_BYTES + b_bytes);  // SL A slabs, then SL B slabs
   const int stages = a.stages;
   // layout: stages | full | empty | tfull[2] | tempty[2] | epi | drain | tmem slot | scratch
   const uint32_t bar_full = base + stages * st_bytes;
@@ -70,8 +83,11 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
   const uint32_t bar_epi = bar_tempty + 16;
   const uint32_t bar_drain = bar_epi + 8;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + (bar_drain + 8 - base));
-  float2* wst = reinterpret_cast<float2*>(gbase + (bar_drain + 8 - base) + 16);  // [4][S_pad]
-  float2* wag = wst + 4 * a.S_pad;                                                // [4][S_pad]
+  float2* wst = reinterpret_cast<float2*>(gbase + (bar_drain + 8 - base) + 16);  // [4][S_pad] per-warp stats
+  float2* wag = wst + 4 * S_pad;                                                  // [4][S_pad] per-warp argmax
+  float2* cst = wag + 4 * S_pad;   // [S_pad] running (max, sum) over this CTA's tiles
+  float2* carg = cst + S_pad;      // [S_pad] running (max u, argmax)
+  float* sbeta = reinterpret_cast<float*>(carg + S_pad);  // [nbeta]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
@@ -95,11 +111,17 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     tmem_alloc(smem_u32(tmem_slot), a.tmem_cols);
     tmem_relinquish();
   }
+  for (int i = tid; i < S_pad; i += LM_THREADS) {
+    cst[i] = make_float2(-INFINITY, 0.f);
+    carg[i] = make_float2(-INFINITY, __int_as_float(0x7fffffff));
+  }
+  if (a.mode == 1)
+    for (int i = tid; i < a.nbeta; i += LM_THREADS) sbeta[i] = a.beta[i];
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int ntiles = a.ntiles, nks = a.nks;
+  const int ntiles = a.ntiles, nst = a.nst;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA
@@ -108,18 +130,22 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-        for (int ks = 0; ks < nks; ++ks, ++it) {
+        for (int ks = 0; ks < nst; ++ks, ++it) {
           const uint32_t st = it % stages, ph = (it / stages) & 1u;
           if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
             ok = false;
             break;
           }
           const uint32_t fb = bar_full + 8 * st;
-          const uint32_t sa = base + st * st_bytes, sb = sa + LM_A_BYTES;
+          const uint32_t sa = base + st * st_bytes, sb = sa + SL * LM_A_BYTES;
           mbar_arrive_expect_tx(fb, st_bytes);
-          tma_load_2d(sa, &wmap, fb, ks * LM_TILE_K, tile * LM_TILE_V, pol_w);
-          for (int c = 0; c < a.nchunk; ++c)
-            tma_load_2d(sb + c * a.chunk_n * 128, &hmap, fb, ks * LM_TILE_K, c * a.chunk_n, pol_h);
+          // consecutive K-slabs of the same 128 rows back to back: longer runs per row
+          for (int j = 0; j < SL; ++j)
+            tma_load_2d(sa + j * LM_A_BYTES, &wmap, fb, (ks * SL + j) * LM_TILE_K, tile * LM_TILE_V, pol_w);
+          for (int j = 0; j < SL; ++j)
+            for (int c = 0; c < a.nchunk; ++c)
+              tma_load_2d(sb + j * b_bytes + c * a.chunk_n * 128, &hmap, fb, (ks * SL + j) * LM_TILE_K,
+                          c * a.chunk_n, pol_h);
         }
       }
       if (!ok) {
@@ -138,21 +164,23 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
         const uint32_t buf = acc % a.acc_bufs, aph = (acc / a.acc_bufs) & 1u;
         if (!mbar_wait(bar_tempty + 8 * buf, aph ^ 1u, a.status)) break;
         tc_fence_after();
-        const uint32_t dcol = tmem_base + buf * a.S_pad;
-        for (int ks = 0; ks < nks; ++ks, ++it) {
+        const uint32_t dcol = tmem_base + buf * S_pad;
+        for (int ks = 0; ks < nst; ++ks, ++it) {
           const uint32_t st = it % stages, ph = (it / stages) & 1u;
           if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa = base + st * st_bytes, sb = sa + LM_A_BYTES;
+          const uint32_t sa = base + st * st_bytes, sb = sa + SL * LM_A_BYTES;
+          for (int j = 0; j < SL; ++j) {
 #pragma unroll
-          for (int k = 0; k < LM_TILE_K / 16; ++k) {
-            const uint64_t ad = umma_desc_sw128(sa + 32 * k);
-            for (int c = 0; c < a.nchunk; ++c)
-              umma_bf16(dcol + c * a.chunk_n, ad, umma_desc_sw128(sb + c * a.chunk_n * 128 + 32 * k), idesc,
-                        (ks | k) != 0);
+            for (int k = 0; k < LM_TILE_K / 16; ++k) {
+              const uint64_t ad = umma_desc_sw128(sa + j * LM_A_BYTES + 32 * k);
+              for (int c = 0; c < a.nchunk; ++c)
+                umma_bf16(dcol + c * a.chunk_n, ad, umma_desc_sw128(sb + j * b_bytes + c * a.chunk_n * 128 + 32 * k),
+                          idesc, (ks | j | k) != 0);
+            }
           }
           umma_commit(bar_empty + 8 * st);
         }
@@ -168,11 +196,15 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     // ----------------------------------------------------------- epilogue
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int etid = tid - 64;
-    const int S = a.S, S_pad = a.S_pad, n1 = a.N + 1;
+    const int S = a.S, n1 = a.N + 1;
     uint32_t acc = 0, ephase = 0;
+    bool ok = true;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++acc) {
       const uint32_t buf = acc % a.acc_bufs, aph = (acc / a.acc_bufs) & 1u;
-      if (!mbar_wait(bar_tfull + 8 * buf, aph, a.status)) break;
+      if (!mbar_wait(bar_tfull + 8 * buf, aph, a.status)) {
+        ok = false;
+        break;
+      }
       tc_fence_after();
       const int v = tile * LM_TILE_V + 32 * q + lane;
       const bool valid = v < a.V;
@@ -197,7 +229,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
               z_am = vals[i];
             } else {
               const int b = col / n1;
-              const float bt = a.beta[b * a.N + j - 1];
+              const float bt = sbeta[b * a.N + j - 1];
               float u = valid ? (1.f + bt) * vals[i] - bt * z_am : -INFINITY;
               int vi = v;
               warp_argmax(u, vi);
@@ -208,27 +240,41 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       }
       tc_fence_before();
       mbar_arrive(bar_tempty + 8 * buf);
-      if (!bar_sync_bounded(bar_epi, ephase, a.status)) break;
+      if (!bar_sync_bounded(bar_epi, ephase, a.status)) {
+        ok = false;
+        break;
+      }
+      // fold the four warps' results into this CTA's running records
       for (int col = etid; col < S; col += 128) {
-        float M = -INFINITY, sum = 0.f;
+        float2 c = cst[col];
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq) {
           const float2 r = wst[qq * S_pad + col];
-          lse_merge(M, sum, r.x, r.y);
+          lse_merge(c.x, c.y, r.x, r.y);
         }
-        a.rec_stats[(int64_t)col * ntiles + tile] = make_float2(M, sum);
+        cst[col] = c;
         if (a.mode == 1 && col % n1 != 0) {
-          float bu = -INFINITY;
-          int bv = 0x7fffffff;
+          float bu = carg[col].x;
+          int bv = __float_as_int(carg[col].y);
 #pragma unroll
           for (int qq = 0; qq < 4; ++qq) {
             const float2 r = wag[qq * S_pad + col];
             argmax_merge(bu, bv, r.x, __float_as_int(r.y));
           }
-          a.rec_arg[(int64_t)col * ntiles + tile] = make_float2(bu, __int_as_float(bv));
+          carg[col] = make_float2(bu, __int_as_float(bv));
         }
       }
-      if (!bar_sync_bounded(bar_epi, ephase, a.status)) break;
+      if (!bar_sync_bounded(bar_epi, ephase, a.status)) {
+        ok = false;
+        break;
+      }
+    }
+    if (ok) {
+      const int nrec = gridDim.x;
+      for (int col = etid; col < S; col += 128) {
+        a.rec_stats[(int64_t)col * nrec + blockIdx.x] = cst[col];
+        if (a.mode == 1 && col % n1 != 0) a.rec_arg[(int64_t)col * nrec + blockIdx.x] = carg[col];
+      }
     }
   }
   tc_fence_before();
@@ -254,13 +300,13 @@ cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, con
 
 // ------------------------------------------------------------ mode-0 finish
 __global__ void __launch_bounds__(256) lm_lse_finalize_kernel(float* logits, const float2* rec_stats, float* lse,
-                                                              int32_t V, int32_t ntiles) {
+                                                              int32_t V, int32_t nrec) {
   const int s = blockIdx.x, tid = threadIdx.x;
   __shared__ float2 red[8];
   __shared__ float Ls;
   float M = -INFINITY, sum = 0.f;
-  for (int t = tid; t < ntiles; t += 256) {
-    const float2 r = rec_stats[(int64_t)s * ntiles + t];
+  for (int t = tid; t < nrec; t += 256) {
+    const float2 r = rec_stats[(int64_t)s * nrec + t];
     lse_merge(M, sum, r.x, r.y);
   }
 #pragma unroll
@@ -283,8 +329,8 @@ __global__ void __launch_bounds__(256) lm_lse_finalize_kernel(float* logits, con
 }
 
 cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float* lse, int32_t S, int32_t V,
-                                   int32_t ntiles, cudaStream_t stream) {
-  lm_lse_finalize_kernel<<<S, 256, 0, stream>>>(logits, rec_stats, lse, V, ntiles);
+                                   int32_t nrec, cudaStream_t stream) {
+  lm_lse_finalize_kernel<<<S, 256, 0, stream>>>(logits, rec_stats, lse, V, nrec);
   return cudaGetLastError();
 }
 
@@ -294,7 +340,7 @@ cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float
 // token asc, expert asc) wins.
 __global__ void __launch_bounds__(256) select_from_records_kernel(SelectArgs a) {
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int N = a.N, n1 = N + 1, s0 = b * n1, T = a.ntiles;
+  const int N = a.N, n1 = N + 1, s0 = b * n1, T = a.nrec;
   __shared__ float Ls[LM_MAX_N1];
   __shared__ float ksc[LM_MAX_N1];
   __shared__ int ktok[LM_MAX_N1];
@@ -428,6 +474,9 @@ extern "C" pced_status pced_lm_head_logprobs(const void* hidden, const void* w_u
   a.V = V;
   a.ntiles = g.ntiles;
   a.nks = g.nks;
+  a.slabs = g.slabs;
+  a.nst = g.nst;
+  a.nbeta = 0;
   a.stages = g.stages;
   a.acc_bufs = g.acc_bufs;
   a.S_pad = g.S_pad;
@@ -435,14 +484,14 @@ extern "C" pced_status pced_lm_head_logprobs(const void* hidden, const void* w_u
   a.chunk_n = g.chunk_n;
   a.tmem_cols = g.tmem_cols;
   a.logits = logprobs;
-  a.rec_stats = cv.take<float2>((size_t)S * g.ntiles);
+  a.rec_stats = cv.take<float2>((size_t)S * g.grid);
   a.rec_arg = nullptr;
   a.beta = nullptr;
   a.status = (int*)workspace;
   cudaStream_t s = (cudaStream_t)stream;
   cudaError_t e = lm_head_launch(wmap, hmap, g, a, s);
   if (e != cudaSuccess) return cuda_status(e, "lm head launch");
-  e = lm_lse_finalize_launch(logprobs, a.rec_stats, lse, S, V, g.ntiles, s);
+  e = lm_lse_finalize_launch(logprobs, a.rec_stats, lse, S, V, g.grid, s);
   if (e != cudaSuccess) return cuda_status(e, "lse finalize launch");
   return PCED_OK;
 }

@@ -12,7 +12,7 @@ constexpr int LM_MAX_S = 512;
 constexpr int LM_MAX_N1 = 256;   // experts + amateur per query in the selection kernels
 
 struct LmGeom {
-  int32_t S, S_pad, nchunk, chunk_n, d, V, ntiles, nks, stages, acc_bufs, grid;
+  int32_t S, S_pad, nchunk, chunk_n, d, V, ntiles, nks, slabs, nst, stages, acc_bufs, grid, nbeta;
   uint32_t tmem_cols;
   size_t smem;
 };
@@ -20,27 +20,27 @@ struct LmGeom {
 bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g);
 
 struct LmArgs {
-  int mode;  // 0: write logits[S][V]; 1: contrastive tile records (needs N, beta)
-  int32_t S, N, V, ntiles, nks, stages, acc_bufs, S_pad, nchunk, chunk_n;
+  int mode;  // 0: write logits[S][V]; 1: contrastive records (needs N, beta)
+  int32_t S, N, V, ntiles, nks, slabs, nst, stages, acc_bufs, S_pad, nchunk, chunk_n, nbeta;
   uint32_t tmem_cols;
   float* logits;      // mode 0
-  float2* rec_stats;  // [S][ntiles] (max z, sum exp(z - max)) of each tile
-  float2* rec_arg;    // [S][ntiles] (max u, argmax v as int bits) for expert columns, mode 1
+  float2* rec_stats;  // [S][grid] (max z, sum exp(z - max)) over each CTA's tiles
+  float2* rec_arg;    // [S][grid] (max u, argmax v as int bits) for expert columns, mode 1
   const float* beta;  // [B][N]
   int* status;
 };
 
 cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, const LmGeom& g, const LmArgs& a,
                            cudaStream_t stream);
-// mode-0 finish: lse[s] from the tile records, logits -> log-probs in place
+// mode-0 finish: lse[s] from the CTA records, logits -> log-probs in place
 cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float* lse, int32_t S, int32_t V,
-                                   int32_t ntiles, cudaStream_t stream);
+                                   int32_t nrec, cudaStream_t stream);
 
 // Selection from mode-1 records (Eq. 2 + Eq. 3), one CTA per query.
 struct SelectArgs {
   const float2* rec_stats;
   const float2* rec_arg;
-  int32_t B, N, ntiles;
+  int32_t B, N, nrec;  // records per row (the LM-head grid size)
   const float* beta;
   const float* r;
   float gamma;

@@ -111,6 +111,8 @@ struct StepLayout {
   float2* lm_stats;
   float2* lm_arg;
   int32_t* done_counter;
+  float* part_ss;
+  int32_t* seq_counters;
   size_t bytes;
 };
 
@@ -122,6 +124,8 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   pced_host::Carver c(ws);
   L.status = c.take<int>(64);
   L.done_counter = c.take<int32_t>(1);
+  L.seq_counters = c.take<int32_t>((size_t)S);
+  L.part_ss = c.take<float>((size_t)S * dm->Hkv);
   L.resid = c.take<float>((size_t)S * d);
   L.q = c.take<__nv_bfloat16>((size_t)S * d);
   L.h = c.take<__nv_bfloat16>((size_t)S * d);
@@ -147,6 +151,13 @@ extern "C" size_t pced_step_workspace_size(const pced_dims* dm) {
 }
 
 extern "C" int32_t pced_step_launch_count(const pced_dims* dm) { return dm ? 1 + 2 * dm->L + 2 : 0; }
+
+extern "C" const char* pced_step_launch_kind(const pced_dims* dm, int32_t i) {
+  if (!dm || i < 0 || i >= pced_step_launch_count(dm)) return nullptr;
+  if (i == 0) return "embed";
+  if (i <= 2 * dm->L) return (i % 2 == 1) ? "attn_split" : "attn_combine";
+  return i == 2 * dm->L + 1 ? "lm_head" : "select";
+}
 
 extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (!p) return fail(PCED_ERR_INVALID_ARG, "pced_step: null args");
@@ -185,6 +196,20 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (st == PCED_OK) st = make_tmap_2d(&hmap, W.h, (uint64_t)S, (uint64_t)d, (uint32_t)g.chunk_n, LM_TILE_K, false);
   if (st != PCED_OK) return st;
   cudaStream_t s = (cudaStream_t)stream;
+  const bool timed = p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
+  cudaStreamCaptureStatus cap_status = cudaStreamCaptureStatusNone;
+  if (timed && cudaStreamIsCapturing(s, &cap_status) != cudaSuccess) return cuda_status(cudaGetLastError(), "capture query");
+  int mark_i = 0;
+  // inside a stream capture the events become external event-record nodes, so
+  // they can still be timed after each replay
+  auto mark = [&]() -> cudaError_t {
+    if (!timed) return cudaSuccess;
+    cudaEvent_t ev = (cudaEvent_t)p->stage_events[mark_i++];
+    return cap_status == cudaStreamCaptureStatusActive ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal)
+                                                       : cudaEventRecord(ev, s);
+  };
+  cudaError_t e = mark();
+  if (e != cudaSuccess) return cuda_status(e, "stage event");
 
   EmbedArgs ea;
   ea.embed = (const __nv_bfloat16*)p->embed;
@@ -208,7 +233,8 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   ea.rms_eps = p->rms_eps;
   ea.status = W.status;
   step_embed_kernel<<<S, EMB_THREADS, 0, s>>>(ea);
-  cudaError_t e = cudaGetLastError();
+  e = cudaGetLastError();
+  if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "embed launch");
 
   const int ctas = att_grid(p->total_cap * dm.Hkv);
@@ -230,6 +256,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     a.plan_per = W.plan_per;
     a.status = W.status;
     e = att_split_launch(dm.D, kmap, vmap, a, ctas, s);
+    if (e == cudaSuccess) e = mark();
     if (e != cudaSuccess) return cuda_status(e, "attention split launch");
     CombineArgs c = {};
     c.mode = 1;
@@ -244,6 +271,8 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     c.plan_per = W.plan_per;
     c.seq_len = p->seq_len;
     c.resid = W.resid;
+    c.part_ss = W.part_ss;
+    c.counters = W.seq_counters;
     c.rms_eps = p->rms_eps;
     c.k_cache = (__nv_bfloat16*)p->k_cache;
     c.v_cache = (__nv_bfloat16*)p->v_cache;
@@ -260,6 +289,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
       c.hidden_copy = (__nv_bfloat16*)p->hidden_out;
     }
     e = att_combine_launch(c, s);
+    if (e == cudaSuccess) e = mark();
     if (e != cudaSuccess) return cuda_status(e, "attention combine launch");
   }
 
@@ -270,6 +300,9 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.V = dm.V;
   la.ntiles = g.ntiles;
   la.nks = g.nks;
+  la.slabs = g.slabs;
+  la.nst = g.nst;
+  la.nbeta = dm.B * dm.N;
   la.stages = g.stages;
   la.acc_bufs = g.acc_bufs;
   la.S_pad = g.S_pad;
@@ -281,6 +314,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.beta = p->beta;
   la.status = W.status;
   e = lm_head_launch(wmap, hmap, g, la, s);
+  if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "lm head launch");
 
   SelectArgs sa = {};
@@ -288,7 +322,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.rec_arg = W.lm_arg;
   sa.B = dm.B;
   sa.N = dm.N;
-  sa.ntiles = g.ntiles;
+  sa.nrec = g.grid;
   sa.beta = p->beta;
   sa.r = p->r;
   sa.gamma = p->gamma;
@@ -301,6 +335,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.done_counter = W.done_counter;
   sa.status = W.status;
   e = select_from_records_launch(sa, s);
+  if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "select launch");
   return PCED_OK;
 }
