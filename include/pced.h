@@ -97,6 +97,37 @@ pced_status pced_decode_attention(const void* q, const void* k_cache, const void
                                   void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * pced_decode_attention_noalloc -- pced_decode_attention for callers that
+ * cannot allocate device memory when they need it (the paper has no
+ * counterpart; this is a deployment convenience).  Examples: code that runs
+ * while the caller's allocator is locked or shutting down, host callbacks
+ * that must not enter the CUDA allocator, or an embedding runtime whose
+ * memory pool is capped and owned by someone else.  The caller passes only
+ * inputs and outputs; the split-KV partial records live in one fixed device
+ * array inside this library, PCED_NOALLOC_SCRATCH_BYTES large, which every
+ * GPU that loads the library reserves until the process exits.
+ *   Arguments q ... out are those of pced_decode_attention.
+ *   status   optional device int32 word the kernels OR PCED_DEV_* bits into
+ *            (the caller zeroes it); NULL discards device-side conditions.
+ * Sizes: the call needs about (SMs + S*Hkv) * (4*G*D + 8*G) + 8*S bytes of
+ * scratch (G = Hq/Hkv, SMs = multiprocessors of the device); above
+ * PCED_NOALLOC_SCRATCH_BYTES it returns PCED_ERR_UNSUPPORTED with the needed
+ * size in pced_last_error() and launches nothing.  On a 152-SM device with
+ * G = 4 and D = 128 that allows S*Hkv up to about 7900.
+ * The call allocates no memory.  Its first call on a device (with that device
+ * current) looks up the array's device address once, so make that first call
+ * before any stream capture on the device.  Every call shares the one array
+ * and overwrites it: calls that can overlap on the GPU (different streams, or
+ * different host threads) race and give wrong results; serialise them.
+ * Nothing in the array needs to start at zero.
+ * ------------------------------------------------------------------------ */
+#define PCED_NOALLOC_SCRATCH_BYTES (16u << 20)
+pced_status pced_decode_attention_noalloc(const void* q, const void* k_cache, const void* v_cache,
+                                          int64_t cache_elems, const int64_t* kv_offset, const int32_t* cap,
+                                          const int32_t* seq_len, int32_t S, int32_t Hq, int32_t Hkv, int32_t D,
+                                          int64_t total_cap, float scale, float* out, int32_t* status, void* stream);
+
+/* ------------------------------------------------------------------------
  * pced_lm_head_logprobs -- per-expert log-probabilities s_k over the
  * vocabulary (Sec. 3: "per-expert logits s_k in R^|V|"; read as
  * log-softmax outputs, the scale Eq. 2 mixes).

@@ -66,6 +66,8 @@ def lib(path: str = LIB_PATH):
         L.pced_decode_attention_workspace_size.restype = SZ
         L.pced_decode_attention.argtypes = [P, P, P, I64, P, P, P, I32, I32, I32, I32, I64, F, P, P, SZ, P]
         L.pced_decode_attention.restype = I32
+        L.pced_decode_attention_noalloc.argtypes = [P, P, P, I64, P, P, P, I32, I32, I32, I32, I64, F, P, P, P]
+        L.pced_decode_attention_noalloc.restype = I32
         L.pced_lm_head_workspace_size.argtypes = [I32, I32]
         L.pced_lm_head_workspace_size.restype = SZ
         L.pced_lm_head_logprobs.argtypes = [P, P, I32, I32, I32, P, P, P, SZ, P]
@@ -128,6 +130,31 @@ def decode_attention(q, k_cache, v_cache, kv_offset, cap, seq_len, Hkv: int, tot
     _check(lib().pced_decode_attention(_ptr(q), _ptr(k_cache), _ptr(v_cache), k_cache.numel(), _ptr(kv_offset),
                                        _ptr(cap), _ptr(seq_len), S, Hq, Hkv, D, int(total_cap), float(scale),
                                        _ptr(out), _ptr(ws), ws.numel(), _stream(stream)), "pced_decode_attention")
+    return out
+
+
+# fixed size of the library's scratch array behind decode_attention_noalloc
+NOALLOC_SCRATCH_BYTES = 16 << 20
+
+
+def decode_attention_noalloc(q, k_cache, v_cache, kv_offset, cap, seq_len, Hkv: int, total_cap: int, out,
+                             scale=None, status=None, stream=None):
+    """pced_decode_attention_noalloc: decode_attention without a workspace.
+
+    For callers that cannot allocate device memory when they run attention
+    (allocator locked or shutting down, host callbacks, capped memory pools):
+    the partial records live in a fixed library-owned device array, so the
+    caller passes the output buffer ``out`` (fp32 [S, Hq, D]) and, optionally,
+    an int32 device ``status`` word.  Calls share that array: overlapping calls
+    on the GPU race.  The first call on a device should come before any stream
+    capture on it."""
+    S, Hq, D = q.shape
+    scale = 1.0 / math.sqrt(D) if scale is None else scale
+    _check(lib().pced_decode_attention_noalloc(_ptr(q), _ptr(k_cache), _ptr(v_cache), k_cache.numel(),
+                                               _ptr(kv_offset), _ptr(cap), _ptr(seq_len), S, Hq, Hkv, D,
+                                               int(total_cap), float(scale), _ptr(out),
+                                               None if status is None else _ptr(status), _stream(stream)),
+           "pced_decode_attention_noalloc")
     return out
 
 
