@@ -2,23 +2,23 @@
 // (paper Sec. 3: N+1 parallel streams, each with an independently encoded
 // cache; grouped-query heads).
 //
-// Split-KV flash decoding on sm_103a:
-//   * all (sequence, kv-head, key) positions are cut into equal contiguous
+// Split-KV flash decoding on sm_103a, shared by both kernels of this file:
+//   * all (kv-head, sequence, key) positions are cut into equal contiguous
 //     ranges, one per CTA, so ragged caches load-balance without a host plan;
 //   * a producer warp streams 64-key K and V tiles through a multi-stage
 //     shared-memory ring with TMA (2-D tensor copies, 128-byte swizzle),
 //     completion tracked by mbarriers;
-//   * four consumer warps each own 16 keys of every tile and compute, for the
-//     G query heads sharing the kv-head, S^T = K Q^T and O^T += V^T P^T with
-//     bf16 mma.sync (fp32 accumulate), online softmax in base 2 with warp
-//     shuffles; P is split into bf16 hi + lo parts so the PV product keeps
-//     ~16 significant bits;
-//   * per piece, the four warps' partials are merged in shared memory and
-//     written as one unnormalised record (max, sum, o); a combine kernel
-//     merges records across CTAs and either writes o or, on the step path,
-//     updates the residual stream, normalises it and appends the next layer's
-//     K/V rows.
+//   * two warpgroups of consumer warps take alternate tiles; each warp owns 16
+//     keys of a tile and computes, for the G query heads sharing the kv-head,
+//     S^T = K Q^T and O^T += V^T P^T with bf16 mma.sync (fp32 accumulate),
+//     online softmax in base 2 with warp shuffles; P is split into bf16 hi +
+//     lo parts so the PV product keeps ~16 significant bits;
+//   * per piece, the eight warps' partials are merged in shared memory into one
+//     unnormalised record (max, sum, o); records of a segment split across
+//     CTAs are merged by a combine kernel (one layer) or by the last CTA to
+//     finish the segment (whole decode step, see att_step_kernel).
 #include <math.h>
+#include <stdlib.h>
 
 #include "attention.cuh"
 
@@ -33,18 +33,51 @@ struct AttCfg {
   static constexpr int STAGES = D == 128 ? 5 : 7;       // odd: consecutive uses of a stage alternate warpgroups
   static constexpr int KSTEPS = D / 16;
   static constexpr int MTILES = D / 16;
-  static constexpr int OPAD = 9;  // padded head stride of the merge scratch
-  static constexpr int MERGE_FLOATS = 2 * ATT_CONSUMERS * ATT_MAX_G + ATT_CONSUMERS * D * OPAD;
-  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + (2 * STAGES + 1) * 8 +
-                                 (size_t)MERGE_FLOATS * 4 + (ATT_MAX_S + 1) * 8 + ATT_MAX_S * 4 + 128;
+  static constexpr int OPAD = 9;                        // padded head stride of the merge scratch
+  static constexpr int OPT = ATT_MAX_G * D / ATT_CT;   // outputs of a piece per consumer thread (G <= 8)
+  static constexpr int MERGE_FLOATS = 2 * ATT_CONSUMERS * ATT_MAX_G + ATT_CONSUMERS * D * OPAD + ATT_CONSUMERS + 8;
+  static constexpr size_t BARS = (2 * STAGES + 2) * 8;
+  static constexpr size_t SMEM = 1024 + (size_t)STAGES * STAGE_BYTES + BARS + (size_t)MERGE_FLOATS * 4 +
+                                 (ATT_MAX_S + 1) * 8 + ATT_MAX_S * 4 + ATT_MAX_S + 128;
 };
+
+// shared-memory scratch of the consumers (after the stages and barriers)
+struct Scratch {
+  float* ms;      // [8][8] per-warp running max of a piece
+  float* ls;      // [8][8] per-warp sum
+  float* os;      // [8][D][OPAD] per-warp o
+  float* red;     // [8] per-warp partial sums
+  int* flag;      // [8] broadcast flags
+  int64_t* pre;   // [S+1] prefix of the segment extents
+  int32_t* lens;  // [S] live lengths
+  uint8_t* apnd;  // [S] 1 if this step appends a row to sequence s
+};
+
+template <int D>
+__device__ __forceinline__ Scratch carve_scratch(uint8_t* p) {
+  using C = AttCfg<D>;
+  Scratch sc;
+  float* f = reinterpret_cast<float*>(p);
+  sc.ms = f;
+  sc.ls = f + ATT_CONSUMERS * ATT_MAX_G;
+  sc.os = f + 2 * ATT_CONSUMERS * ATT_MAX_G;
+  sc.red = sc.os + ATT_CONSUMERS * D * C::OPAD;
+  sc.flag = reinterpret_cast<int*>(sc.red + ATT_CONSUMERS);
+  sc.pre = reinterpret_cast<int64_t*>(f + C::MERGE_FLOATS);
+  sc.lens = reinterpret_cast<int32_t*>(sc.pre + ATT_MAX_S + 1);
+  sc.apnd = reinterpret_cast<uint8_t*>(sc.lens + ATT_MAX_S);
+  return sc;
+}
 
 struct Piece {
-  int32_t s, h, k0, k1;
+  int32_t s, h, k0, k1;  // real keys [k0, k1) of kv-head h of sequence s (k0 == k1: no keys)
+  int64_t adv;           // positions the piece spans
 };
 
-// (sequence, head, key range) of the piece that starts at global position p
-// and ends at the next segment boundary or at `end`.
+// Piece that starts at global position p and ends at the next segment
+// boundary or at `end`.  Segment (h, s) spans positions
+// [h*T + pre[s], h*T + pre[s+1]); its first lens[s] positions are keys, the
+// rest (if any) only weight the partition.
 __device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* lens, int32_t S, int64_t T, int64_t p,
                                             int64_t end) {
   Piece pc;
@@ -57,25 +90,198 @@ __device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* l
     else hi = mid - 1;
   }
   pc.s = lo;
-  pc.k0 = (int32_t)(r - pre[lo]);
-  const int64_t seg_end = (int64_t)pc.h * T + pre[lo] + lens[lo];
+  const int64_t off = r - pre[lo];
+  const int64_t seg_end = (int64_t)pc.h * T + pre[lo + 1];
   const int64_t e = seg_end < end ? seg_end : end;
-  pc.k1 = pc.k0 + (int32_t)(e - p);
+  pc.adv = e - p;
+  const int64_t len = lens[lo];
+  if (off < len) {
+    const int64_t k1 = off + pc.adv;
+    pc.k0 = (int32_t)off;
+    pc.k1 = (int32_t)(k1 < len ? k1 : len);
+  } else {
+    pc.k0 = pc.k1 = 0;
+  }
   return pc;
 }
 
-template <int KSTEPS>
-__device__ __forceinline__ void load_q_frag(uint32_t (&qf)[KSTEPS][2], const AttArgs& a, const Piece& pc, int g,
-                                            int tq, int D) {
-  const bool hv = g < a.G;
-  const __nv_bfloat16* qrow = a.q + ((int64_t)pc.s * a.Hq + (int64_t)pc.h * a.G + (hv ? g : 0)) * D;
+// exclusive prefix of ext[i] = lens[i] + extra into pre[0..S] (one warp)
+__device__ __forceinline__ void prefix_extents(const int32_t* lens, int32_t S, int32_t extra, int64_t* pre, int lane) {
+  const int chunk = (S + 31) / 32;
+  const int b0 = lane * chunk, b1 = min(S, b0 + chunk);
+  int64_t sum = 0;
+  for (int i = b0; i < b1; ++i) sum += (int64_t)lens[i] + extra;
+  int64_t incl = sum;
 #pragma unroll
-  for (int j = 0; j < KSTEPS; ++j) {
-    qf[j][0] = hv ? *reinterpret_cast<const uint32_t*>(qrow + 16 * j + 2 * tq) : 0u;
-    qf[j][1] = hv ? *reinterpret_cast<const uint32_t*>(qrow + 16 * j + 8 + 2 * tq) : 0u;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int64_t v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  int64_t run = incl - sum;
+  for (int i = b0; i < b1; ++i) {
+    pre[i] = run;
+    run += (int64_t)lens[i] + extra;
+  }
+  if (lane == 31) pre[S] = incl;
+}
+
+// ------------------------------------------------------------ consumer math
+// Online-softmax state of one consumer warp over its keys of a piece.
+template <int D>
+struct WarpAcc {
+  float m0, m1, l0, l1;  // heads 2tq and 2tq+1 of this thread
+  float o[D / 16][4];    // O^T fragments: dims 16i + g (+8), heads 2tq, 2tq+1
+};
+
+template <int D>
+__device__ __forceinline__ void acc_reset(WarpAcc<D>& A) {
+  A.m0 = A.m1 = -INFINITY;
+  A.l0 = A.l1 = 0.f;
+#pragma unroll
+  for (int i = 0; i < D / 16; ++i) A.o[i][0] = A.o[i][1] = A.o[i][2] = A.o[i][3] = 0.f;
+}
+
+// This warp's 16 keys [kb, kb+16) of the 64-key K/V tiles at sk / sv (TMA
+// 128-byte swizzle, D/64 boxes of 64 rows x 128 B); keys at or past nvalid
+// are masked.  qf: B operand of S^T = K Q^T (dims x heads).
+template <int D>
+__device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D / 16][2], uint32_t sk, uint32_t sv,
+                                          int kb, int nvalid, float scale_log2, int lane) {
+  using C = AttCfg<D>;
+  const int g = lane >> 2, tq = lane & 3, mat = lane >> 3, mr = lane & 7;
+  // ---- scores S^T (16 keys x 8 heads), two independent accumulation chains
+  float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+  {
+    const int key = kb + (mat & 1) * 8 + mr;
+    const uint32_t rowa = sk + key * 128;
+    const uint32_t sw = key & 7;
+#pragma unroll
+    for (int j = 0; j < C::KSTEPS; ++j) {
+      const int chunk = 2 * j + (mat >> 1);
+      const uint32_t addr = rowa + (chunk >> 3) * C::BOX_BYTES + (((chunk & 7) ^ sw) << 4);
+      uint32_t a0, a1, a2, a3;
+      ldsm_x4(addr, a0, a1, a2, a3);
+      mma_bf16((j & 1) ? sb : sa, a0, a1, a2, a3, qf[j][0], qf[j][1]);
+    }
+  }
+  const bool v0 = kb + g < nvalid, v1 = kb + g + 8 < nvalid;
+  const float s0 = v0 ? (sa[0] + sb[0]) * scale_log2 : -INFINITY;
+  const float s1 = v0 ? (sa[1] + sb[1]) * scale_log2 : -INFINITY;
+  const float s2 = v1 ? (sa[2] + sb[2]) * scale_log2 : -INFINITY;
+  const float s3 = v1 ? (sa[3] + sb[3]) * scale_log2 : -INFINITY;
+  float x0 = fmaxf(s0, s2), x1 = fmaxf(s1, s3);
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    x0 = fmaxf(x0, __shfl_xor_sync(0xffffffffu, x0, off));
+    x1 = fmaxf(x1, __shfl_xor_sync(0xffffffffu, x1, off));
+  }
+  const float n0 = fmaxf(A.m0, x0), n1 = fmaxf(A.m1, x1);
+  const float u0 = n0 == -INFINITY ? 0.f : n0, u1 = n1 == -INFINITY ? 0.f : n1;
+  const float al0 = exp2f(A.m0 - u0), al1 = exp2f(A.m1 - u1);
+  const float p0 = exp2f(s0 - u0), p1 = exp2f(s1 - u1), p2 = exp2f(s2 - u0), p3 = exp2f(s3 - u1);
+  A.l0 = A.l0 * al0 + p0 + p2;
+  A.l1 = A.l1 * al1 + p1 + p3;
+  A.m0 = n0;
+  A.m1 = n1;
+#pragma unroll
+  for (int i = 0; i < C::MTILES; ++i) {
+    A.o[i][0] *= al0;
+    A.o[i][2] *= al0;
+    A.o[i][1] *= al1;
+    A.o[i][3] *= al1;
+  }
+  // ---- P^T as the B operand (keys x heads), split into bf16 hi + lo
+  const uint32_t h01 = pack_bf16(p0, p1), h23 = pack_bf16(p2, p3);
+  const uint32_t q01 = pack_bf16(p0 - bf16_lo(h01), p1 - bf16_hi(h01));
+  const uint32_t q23 = pack_bf16(p2 - bf16_lo(h23), p3 - bf16_hi(h23));
+  const uint32_t bh0 = movmatrix_t(h01), bh1 = movmatrix_t(h23);
+  const uint32_t bl0 = movmatrix_t(q01), bl1 = movmatrix_t(q23);
+  // ---- O^T += V^T P^T; rows of V past the live length are zeroed
+  const bool partial = kb + 16 > nvalid;
+  const int klo = kb + 2 * tq, khi = klo + 8;
+  const int key = kb + (mat >> 1) * 8 + mr;
+  const uint32_t rowa = sv + key * 128;
+  const uint32_t sw = key & 7;
+#pragma unroll
+  for (int i = 0; i < C::MTILES; ++i) {
+    const int chunk = 2 * i + (mat & 1);
+    const uint32_t addr = rowa + (chunk >> 3) * C::BOX_BYTES + (((chunk & 7) ^ sw) << 4);
+    uint32_t a0, a1, a2, a3;
+    ldsm_x4_t(addr, a0, a1, a2, a3);
+    if (partial) {
+      const uint32_t mlo = (klo < nvalid ? 0xFFFFu : 0u) | (klo + 1 < nvalid ? 0xFFFF0000u : 0u);
+      const uint32_t mhi = (khi < nvalid ? 0xFFFFu : 0u) | (khi + 1 < nvalid ? 0xFFFF0000u : 0u);
+      a0 &= mlo;
+      a1 &= mlo;
+      a2 &= mhi;
+      a3 &= mhi;
+    }
+    mma_bf16(A.o[i], a0, a1, a2, a3, bh0, bh1);
+    mma_bf16(A.o[i], a0, a1, a2, a3, bl0, bl1);
   }
 }
 
+// Merge the eight consumer warps' accumulators of a piece through shared
+// memory.  Afterwards this thread holds, for outputs idx = ctid + k*ATT_CT
+// (idx = hh*D + dd < G*D), the piece's running max mx[k] (log2 units), sum
+// ls[k] and unnormalised output acc[k].  The caller must pass another
+// consumer barrier before the next call (the scratch is reused).
+template <int D>
+__device__ __forceinline__ bool cta_merge(const WarpAcc<D>& A, const Scratch& sc, int G, int warp, int lane, int ctid,
+                                          uint32_t bar, uint32_t& ph, int* status, float (&mx)[AttCfg<D>::OPT],
+                                          float (&ls)[AttCfg<D>::OPT], float (&acc)[AttCfg<D>::OPT]) {
+  using C = AttCfg<D>;
+  const int g = lane >> 2, tq = lane & 3;
+  float l0 = A.l0, l1 = A.l1;
+#pragma unroll
+  for (int off = 4; off < 32; off <<= 1) {
+    l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+  }
+  if (g == 0) {
+    sc.ms[warp * ATT_MAX_G + 2 * tq] = A.m0;
+    sc.ms[warp * ATT_MAX_G + 2 * tq + 1] = A.m1;
+    sc.ls[warp * ATT_MAX_G + 2 * tq] = l0;
+    sc.ls[warp * ATT_MAX_G + 2 * tq + 1] = l1;
+  }
+  float* ow = sc.os + warp * D * C::OPAD;
+#pragma unroll
+  for (int i = 0; i < C::MTILES; ++i) {
+    const int d0 = 16 * i + g, d1 = d0 + 8;
+    ow[d0 * C::OPAD + 2 * tq] = A.o[i][0];
+    ow[d0 * C::OPAD + 2 * tq + 1] = A.o[i][1];
+    ow[d1 * C::OPAD + 2 * tq] = A.o[i][2];
+    ow[d1 * C::OPAD + 2 * tq + 1] = A.o[i][3];
+  }
+  if (!warps_sync(bar, ph, status)) return false;
+#pragma unroll
+  for (int k = 0; k < C::OPT; ++k) {
+    const int idx = ctid + k * ATT_CT;
+    mx[k] = -INFINITY;
+    ls[k] = 0.f;
+    acc[k] = 0.f;
+    if (idx >= G * D) continue;
+    const int hh = idx / D, dd = idx - hh * D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < ATT_CONSUMERS; ++w) M = fmaxf(M, sc.ms[w * ATT_MAX_G + hh]);
+    float a = 0.f, l = 0.f;
+#pragma unroll
+    for (int w = 0; w < ATT_CONSUMERS; ++w) {
+      const float mw = sc.ms[w * ATT_MAX_G + hh];
+      if (mw == -INFINITY) continue;
+      const float e = exp2f(mw - M);
+      a += sc.os[(w * D + dd) * C::OPAD + hh] * e;
+      l += sc.ls[w * ATT_MAX_G + hh] * e;
+    }
+    mx[k] = M;
+    ls[k] = l;
+    acc[k] = a;
+  }
+  return true;
+}
+
+// =================================================================== one layer
 template <int D>
 __global__ void __launch_bounds__(ATT_THREADS, 1)
     att_split_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, AttArgs a) {
@@ -84,16 +290,11 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
-  // layout: stages | full[STAGES] | empty[STAGES] | merge | merge scratch | pre[S+1] | lens[S]
+  // layout: stages | full[STAGES] | empty[STAGES] | consumer barrier | spare | scratch
   const uint32_t bar_full = base + C::STAGES * C::STAGE_BYTES;
   const uint32_t bar_empty = bar_full + C::STAGES * 8;
-  const uint32_t bar_merge = bar_empty + C::STAGES * 8;
-  float* mscr = reinterpret_cast<float*>(gbase + C::STAGES * C::STAGE_BYTES + (2 * C::STAGES + 1) * 8);
-  float* ms = mscr;                                  // [8][8]
-  float* ls = mscr + ATT_CONSUMERS * ATT_MAX_G;      // [8][8]
-  float* os = mscr + 2 * ATT_CONSUMERS * ATT_MAX_G;  // [8][D][OPAD]
-  int64_t* pre = reinterpret_cast<int64_t*>(mscr + C::MERGE_FLOATS);
-  int32_t* lens = reinterpret_cast<int32_t*>(pre + ATT_MAX_S + 1);
+  const uint32_t bar_c = bar_empty + C::STAGES * 8;
+  const Scratch sc = carve_scratch<D>(gbase + C::STAGES * C::STAGE_BYTES + C::BARS);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int32_t S = a.S, G = a.G;
@@ -101,9 +302,9 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   if (tid == 0) {
     for (int i = 0; i < C::STAGES; ++i) {
       mbar_init(bar_full + 8 * i, 1);
-      mbar_init(bar_empty + 8 * i, 4);  // one warpgroup consumes each stage
+      mbar_init(bar_empty + 8 * i, 4);  // the four warps of the consuming warpgroup
     }
-    mbar_init(bar_merge, ATT_CONSUMERS * 32);
+    mbar_init(bar_c, ATT_CONSUMERS);
     mbar_fence_init();
   }
   if (warp == ATT_CONSUMERS && lane == 0) {
@@ -117,28 +318,13 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       dev_flag(a.status, PCED_DEV_BAD_LENGTH);
       L = L < 1 ? 1 : (L > c ? (c < 1 ? 1 : c) : L);
     }
-    lens[i] = L;
+    sc.lens[i] = L;
   }
   __syncthreads();
-  if (warp == 0) {  // exclusive prefix of len
-    const int chunk = (S + 31) / 32;
-    const int b0 = lane * chunk, b1 = min(S, b0 + chunk);
-    int64_t sum = 0;
-    for (int i = b0; i < b1; ++i) sum += lens[i];
-    int64_t incl = sum;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int64_t v = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += v;
-    }
-    int64_t run = incl - sum;
-    for (int i = b0; i < b1; ++i) {
-      pre[i] = run;
-      run += lens[i];
-    }
-    if (lane == 31) pre[S] = incl;
-  }
+  if (warp == 0) prefix_extents(sc.lens, S, 0, sc.pre, lane);
   __syncthreads();
+  const int64_t* pre = sc.pre;
+  const int32_t* lens = sc.lens;
   const int64_t T = pre[S];
   const int64_t total = T * a.Hkv;
   const int64_t per = (total + gridDim.x - 1) / gridDim.x;
@@ -146,7 +332,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
     for (int i = tid; i <= S; i += ATT_THREADS) a.plan_pre[i] = pre[i];
     if (tid == 0) *a.plan_per = per;
   }
-  const int64_t r_begin = (int64_t)blockIdx.x * per;
+  const int64_t r_begin = min(total, (int64_t)blockIdx.x * per);
   const int64_t r_end = min(total, r_begin + per);
 
   if (warp == ATT_CONSUMERS) {
@@ -157,6 +343,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       bool ok = true;
       for (int64_t p = r_begin; p < r_end && ok;) {
         const Piece pc = find_piece(pre, lens, S, T, p, r_end);
+        p += pc.adv;
         const int64_t slab_row = a.row_base + (a.kv_offset[pc.s] + (int64_t)pc.h * a.cap[pc.s] * D) / D;
         for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
           const uint32_t st = it % C::STAGES, ph = (it / C::STAGES) & 1u;
@@ -174,7 +361,6 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
             tma_load_2d(sv + b * C::BOX_BYTES, &vmap, fb, b * 64, row, pol);
           }
         }
-        p += pc.k1 - pc.k0;
       }
       if (!ok) {
         // let copies already in flight land before the CTA exits
@@ -186,32 +372,27 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   }
 
   // -------------------------------------------------------------- consumers
-  const int wg = warp >> 2, wl = warp & 3;  // warpgroup, warp within the group
-  const int g = lane >> 2, tq = lane & 3;   // mma group id / thread in group
-  const int mat = lane >> 3, mr = lane & 7;
-  const int kb = 16 * wl;                   // first key of this warp's slice of a tile
-  uint32_t it = 0, mphase = 0;
+  const int wg = warp >> 2, wl = warp & 3;
+  const int g = lane >> 2, tq = lane & 3;
+  const int kb = 16 * wl;
+  uint32_t it = 0, cph = 0;
   bool ok = true;
-  uint32_t qn[C::KSTEPS][2];
-  if (r_begin < r_end) load_q_frag<C::KSTEPS>(qn, a, find_piece(pre, lens, S, T, r_begin, r_end), g, tq, D);
   for (int64_t p = r_begin; p < r_end && ok;) {
     const Piece pc = find_piece(pre, lens, S, T, p, r_end);
-    p += pc.k1 - pc.k0;
-    // B operand of S^T = K Q^T (rows: head dim, cols: the G query heads);
-    // the next piece's query is fetched now so its latency overlaps this piece
+    p += pc.adv;
     uint32_t qf[C::KSTEPS][2];
+    {
+      const bool hv = g < G;
+      const uint32_t* qrow = reinterpret_cast<const uint32_t*>(
+          a.q + ((int64_t)pc.s * a.Hq + (int64_t)pc.h * G + (hv ? g : 0)) * D);
 #pragma unroll
-    for (int j = 0; j < C::KSTEPS; ++j) {
-      qf[j][0] = qn[j][0];
-      qf[j][1] = qn[j][1];
+      for (int j = 0; j < C::KSTEPS; ++j) {
+        qf[j][0] = hv ? qrow[8 * j + tq] : 0u;
+        qf[j][1] = hv ? qrow[8 * j + 4 + tq] : 0u;
+      }
     }
-    if (p < r_end) load_q_frag<C::KSTEPS>(qn, a, find_piece(pre, lens, S, T, p, r_end), g, tq, D);
-
-    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-    float o[C::MTILES][4];
-#pragma unroll
-    for (int i = 0; i < C::MTILES; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-
+    WarpAcc<D> A;
+    acc_reset(A);
     for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
       if ((int)(it & 1u) != wg) continue;
       const uint32_t use = it / C::STAGES, st = it % C::STAGES, ph = use & 1u;
@@ -229,143 +410,38 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       }
       const int nvalid = min(ATT_BLOCK_N, pc.k1 - kt);
       if (kb < nvalid) {
-        const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
-        // ---- scores S^T (16 keys x 8 heads), two independent accumulation chains
-        float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
-        {
-          const int key = kb + (mat & 1) * 8 + mr;
-          const uint32_t rowa = sk + key * 128;
-          const uint32_t sw = key & 7;
-#pragma unroll
-          for (int j = 0; j < C::KSTEPS; ++j) {
-            const int chunk = 2 * j + (mat >> 1);
-            const uint32_t addr = rowa + (chunk >> 3) * C::BOX_BYTES + (((chunk & 7) ^ sw) << 4);
-            uint32_t a0, a1, a2, a3;
-            ldsm_x4(addr, a0, a1, a2, a3);
-            mma_bf16((j & 1) ? sb : sa, a0, a1, a2, a3, qf[j][0], qf[j][1]);
-          }
-        }
-        const bool v0 = kb + g < nvalid, v1 = kb + g + 8 < nvalid;
-        const float s0 = v0 ? (sa[0] + sb[0]) * a.scale_log2 : -INFINITY;
-        const float s1 = v0 ? (sa[1] + sb[1]) * a.scale_log2 : -INFINITY;
-        const float s2 = v1 ? (sa[2] + sb[2]) * a.scale_log2 : -INFINITY;
-        const float s3 = v1 ? (sa[3] + sb[3]) * a.scale_log2 : -INFINITY;
-        float x0 = fmaxf(s0, s2), x1 = fmaxf(s1, s3);
-#pragma unroll
-        for (int off = 4; off < 32; off <<= 1) {
-          x0 = fmaxf(x0, __shfl_xor_sync(0xffffffffu, x0, off));
-          x1 = fmaxf(x1, __shfl_xor_sync(0xffffffffu, x1, off));
-        }
-        const float n0 = fmaxf(m0, x0), n1 = fmaxf(m1, x1);
-        const float u0 = n0 == -INFINITY ? 0.f : n0, u1 = n1 == -INFINITY ? 0.f : n1;
-        const float al0 = exp2f(m0 - u0), al1 = exp2f(m1 - u1);
-        const float p0 = exp2f(s0 - u0), p1 = exp2f(s1 - u1), p2 = exp2f(s2 - u0), p3 = exp2f(s3 - u1);
-        l0 = l0 * al0 + p0 + p2;
-        l1 = l1 * al1 + p1 + p3;
-        m0 = n0;
-        m1 = n1;
-#pragma unroll
-        for (int i = 0; i < C::MTILES; ++i) {
-          o[i][0] *= al0;
-          o[i][2] *= al0;
-          o[i][1] *= al1;
-          o[i][3] *= al1;
-        }
-        // ---- P^T as the B operand (keys x heads), split into bf16 hi + lo
-        const uint32_t h01 = pack_bf16(p0, p1), h23 = pack_bf16(p2, p3);
-        const uint32_t q01 = pack_bf16(p0 - bf16_lo(h01), p1 - bf16_hi(h01));
-        const uint32_t q23 = pack_bf16(p2 - bf16_lo(h23), p3 - bf16_hi(h23));
-        const uint32_t bh0 = movmatrix_t(h01), bh1 = movmatrix_t(h23);
-        const uint32_t bl0 = movmatrix_t(q01), bl1 = movmatrix_t(q23);
-        // ---- O^T += V^T P^T; rows of V past the live length are zeroed
-        const bool partial = kb + 16 > nvalid;
-        const int klo = kb + 2 * tq, khi = klo + 8;
-        {
-          const int key = kb + (mat >> 1) * 8 + mr;
-          const uint32_t rowa = sv + key * 128;
-          const uint32_t sw = key & 7;
-#pragma unroll
-          for (int i = 0; i < C::MTILES; ++i) {
-            const int chunk = 2 * i + (mat & 1);
-            const uint32_t addr = rowa + (chunk >> 3) * C::BOX_BYTES + (((chunk & 7) ^ sw) << 4);
-            uint32_t a0, a1, a2, a3;
-            ldsm_x4_t(addr, a0, a1, a2, a3);
-            if (partial) {
-              const uint32_t mlo = (klo < nvalid ? 0xFFFFu : 0u) | (klo + 1 < nvalid ? 0xFFFF0000u : 0u);
-              const uint32_t mhi = (khi < nvalid ? 0xFFFFu : 0u) | (khi + 1 < nvalid ? 0xFFFF0000u : 0u);
-              a0 &= mlo;
-              a1 &= mlo;
-              a2 &= mhi;
-              a3 &= mhi;
-            }
-            mma_bf16(o[i], a0, a1, a2, a3, bh0, bh1);
-            mma_bf16(o[i], a0, a1, a2, a3, bl0, bl1);
-          }
-        }
+        const uint32_t sk = base + st * C::STAGE_BYTES;
+        tile_math<D>(A, qf, sk, sk + C::TILE_BYTES, kb, nvalid, a.scale_log2, lane);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_empty + 8 * st);
     }
     if (!ok) break;
-
-    // ---- merge the eight warps' partials of this piece and write the record
-#pragma unroll
-    for (int off = 4; off < 32; off <<= 1) {
-      l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-      l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-    }
-    if (g == 0) {
-      ms[warp * ATT_MAX_G + 2 * tq] = m0;
-      ms[warp * ATT_MAX_G + 2 * tq + 1] = m1;
-      ls[warp * ATT_MAX_G + 2 * tq] = l0;
-      ls[warp * ATT_MAX_G + 2 * tq + 1] = l1;
-    }
-    float* ow = os + warp * D * C::OPAD;
-#pragma unroll
-    for (int i = 0; i < C::MTILES; ++i) {
-      const int d0 = 16 * i + g, d1 = d0 + 8;
-      ow[d0 * C::OPAD + 2 * tq] = o[i][0];
-      ow[d0 * C::OPAD + 2 * tq + 1] = o[i][1];
-      ow[d1 * C::OPAD + 2 * tq] = o[i][2];
-      ow[d1 * C::OPAD + 2 * tq + 1] = o[i][3];
-    }
-    if (!bar_sync_bounded(bar_merge, mphase, a.status)) break;
+    float mx[C::OPT], ls[C::OPT], acc[C::OPT];
+    if (!cta_merge<D>(A, sc, G, warp, lane, tid, bar_c, cph, a.status, mx, ls, acc)) break;
     const int64_t slot = (int64_t)blockIdx.x + (int64_t)pc.h * S + pc.s;
-    for (int idx = tid; idx < G * D; idx += ATT_CONSUMERS * 32) {
-      const int hh = idx / D, dd = idx - hh * D;
-      float M = -INFINITY;
 #pragma unroll
-      for (int w = 0; w < ATT_CONSUMERS; ++w) M = fmaxf(M, ms[w * ATT_MAX_G + hh]);
-      float acc = 0.f, lsum = 0.f;
-#pragma unroll
-      for (int w = 0; w < ATT_CONSUMERS; ++w) {
-        const float mw = ms[w * ATT_MAX_G + hh];
-        if (mw == -INFINITY) continue;
-        const float e = exp2f(mw - M);
-        acc += os[(w * D + dd) * C::OPAD + hh] * e;
-        lsum += ls[w * ATT_MAX_G + hh] * e;
-      }
-      a.rec_o[(slot * G + hh) * D + dd] = acc;
-      if (dd == 0) a.rec_ml[slot * G + hh] = make_float2(M, lsum);
+    for (int k = 0; k < C::OPT; ++k) {
+      const int idx = tid + k * ATT_CT;
+      if (idx >= G * D) continue;
+      a.rec_o[slot * G * D + idx] = acc[k];
+      if (idx % D == 0) a.rec_ml[slot * G + idx / D] = make_float2(mx[k], ls[k]);
     }
-    if (!bar_sync_bounded(bar_merge, mphase, a.status)) break;
+    if (!warps_sync(bar_c, cph, a.status)) break;
   }
 }
 
-// ------------------------------------------------------------------ combine
 // One CTA per (kv-head h, sequence s): weights of the records that cover the
 // segment are formed once in shared memory, then every output element sums
 // its records with independent loads.
 constexpr int CMB_THREADS = 128;
-constexpr int CMB_SLOTS = 64;                        // records weighted per pass
+constexpr int CMB_SLOTS = 64;                                  // records weighted per pass
 constexpr int CMB_PER_THREAD = ATT_MAX_G * 128 / CMB_THREADS;  // G*D <= 1024 outputs per CTA
 
 __global__ void __launch_bounds__(CMB_THREADS) att_combine_kernel(CombineArgs a) {
   const int h = blockIdx.x, s = blockIdx.y, tid = threadIdx.x;
-  const int32_t Hq = a.Hq, Hkv = a.Hkv, G = a.G, D = a.D, S = a.S, d = Hq * D;
+  const int32_t Hq = a.Hq, G = a.G, D = a.D, S = a.S, d = Hq * D;
   __shared__ float wts[CMB_SLOTS][ATT_MAX_G];
-  __shared__ float red[CMB_THREADS / 32];
-  __shared__ int last;
   const int64_t per = *a.plan_per;
   const int64_t T = a.plan_pre[S];
   const int64_t pre_s = a.plan_pre[s];
@@ -411,69 +487,453 @@ __global__ void __launch_bounds__(CMB_THREADS) att_combine_kernel(CombineArgs a)
       }
     }
   }
-  if (a.mode == 0) {
-#pragma unroll
-    for (int j = 0; j < CMB_PER_THREAD; ++j) {
-      const int idx = tid + j * CMB_THREADS;
-      if (idx < GD) a.out[(int64_t)s * d + (int64_t)h * GD + idx] = acc[j];
-    }
-    return;
-  }
-  // residual update of this CTA's heads and their sum of squares
-  float ss = 0.f;
-  float* xr = a.resid + (int64_t)s * d + (int64_t)h * GD;
 #pragma unroll
   for (int j = 0; j < CMB_PER_THREAD; ++j) {
     const int idx = tid + j * CMB_THREADS;
-    if (idx < GD) {
-      const float x = xr[idx] + acc[j];
-      xr[idx] = x;
-      ss += x * x;
+    if (idx < GD) a.out[(int64_t)s * d + (int64_t)h * GD + idx] = acc[j];
+  }
+}
+
+// ============================================================ whole step
+// Tile cursor over a CTA's range through all layers (the producer's order).
+struct TileCursor {
+  int32_t l, kt;
+  int64_t p, row0;  // row0: tensor-map row of key 0 of the current piece
+  Piece pc;
+  bool ok;
+};
+
+__device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
+                                            const int32_t* lens, int64_t T, int64_t cb, int64_t ce, int D) {
+  while (true) {
+    if (c.p >= ce) {
+      if (++c.l >= a.L) {
+        c.ok = false;
+        return;
+      }
+      c.p = cb;
     }
+    c.pc = find_piece(pre, lens, a.S, T, c.p, ce);
+    if (c.pc.k0 < c.pc.k1) {
+      c.kt = c.pc.k0;
+      c.row0 = (int64_t)c.l * a.rows_per_layer + (a.kv_offset[c.pc.s] + (int64_t)c.pc.h * a.cap[c.pc.s] * D) / D;
+      return;
+    }
+    c.p += c.pc.adv;
+  }
+}
+__device__ __forceinline__ void cursor_begin(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
+                                             const int32_t* lens, int64_t T, int64_t cb, int64_t ce, int D) {
+  c.l = 0;
+  c.p = cb;
+  c.ok = cb < ce && a.L > 0;
+  if (c.ok) cursor_seek(c, a, pre, lens, T, cb, ce, D);
+}
+__device__ __forceinline__ void cursor_next(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
+                                            const int32_t* lens, int64_t T, int64_t cb, int64_t ce, int D) {
+  c.kt += ATT_BLOCK_N;
+  if (c.kt < c.pc.k1) return;
+  c.p += c.pc.adv;
+  cursor_seek(c, a, pre, lens, T, cb, ce, D);
+}
+
+// 1/rms of a residual row from its per-group sums of squares; the same
+// summation order in every warp and CTA, so all users agree bit for bit.
+__device__ __forceinline__ float inv_rms(const float* part, int Hkv, int d, float eps, int lane) {
+  float t = 0.f;
+  for (int i = lane; i < Hkv; i += 32) t += __ldcg(part + i);
+  t = warp_sum(t);
+  t = __shfl_sync(0xffffffffu, t, 0);
+  return 1.0f / sqrtf(t / (float)d + eps);
+}
+
+// x_0[s] = E[y_{t-1}] into residual buffer 0 with its per-group sums of
+// squares, then ready[0] += Hkv.
+template <int D>
+__device__ bool embed_sequence(const StepAttArgs& a, const Scratch& sc, int s, uint32_t bar, uint32_t& ph, int ctid,
+                               int warp, int lane) {
+  const int d = a.Hq * D, GD = a.G * D, b = s / a.n1;
+  const int t = *a.step;
+  int tok = a.bos;
+  if (t > 0 && t <= a.max_steps) tok = a.history[(int64_t)b * a.max_steps + t - 1];
+  if (tok < 0 || tok >= a.V) {
+    if (ctid == 0) dev_flag(a.status, PCED_DEV_BAD_TOKEN);
+    tok = 0;
+  }
+  if (s == 0 && ctid == 0 && t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
+  const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(a.embed + (int64_t)tok * d);
+  float2* x = reinterpret_cast<float2*>(a.resid + (int64_t)s * d);
+  for (int h = warp; h < a.Hkv; h += ATT_CONSUMERS) {
+    float ss = 0.f;
+    for (int i = lane; i < GD / 2; i += 32) {
+      const float2 v = __bfloat1622float2(e[h * GD / 2 + i]);
+      x[h * GD / 2 + i] = v;
+      ss += v.x * v.x + v.y * v.y;
+    }
+    ss = warp_sum(ss);
+    if (lane == 0) a.part_ss[(int64_t)s * a.Hkv + h] = ss;
+  }
+  if (!warps_sync(bar, ph, a.status)) return false;
+  if (ctid == 0) red_release_gpu_add(&a.ready[0], a.Hkv);
+  return true;
+}
+
+// The row appended this step (u = bf16(x_l * inv), K head h and V head
+// Hkv + h of u viewed as [Hq][D]) into row r of the shared K/V tiles and into
+// the caches.  Called by the one warp that owns the row.
+template <int D>
+__device__ __forceinline__ void patch_row(const StepAttArgs& a, const float* xs, float inv, const Piece& pc,
+                                          int32_t row, int r, int l, uint32_t sk, uint32_t sv, int lane) {
+  using C = AttCfg<D>;
+  const float* xk = xs + (int64_t)pc.h * D;
+  const float* xv = xs + ((int64_t)a.Hkv + pc.h) * D;
+  const int64_t grow = (int64_t)l * a.layer_elems + a.kv_offset[pc.s] + ((int64_t)pc.h * a.cap[pc.s] + row) * D;
+  for (int e = 4 * lane; e < D; e += 128) {
+    const float4 kx = __ldcg(reinterpret_cast<const float4*>(xk + e));
+    const float4 vx = __ldcg(reinterpret_cast<const float4*>(xv + e));
+    const uint2 kb2 = make_uint2(pack_bf16(kx.x * inv, kx.y * inv), pack_bf16(kx.z * inv, kx.w * inv));
+    const uint2 vb2 = make_uint2(pack_bf16(vx.x * inv, vx.y * inv), pack_bf16(vx.z * inv, vx.w * inv));
+    const int c = e >> 3;  // 16-byte chunk of the row
+    const uint32_t off =
+        (c >> 3) * C::BOX_BYTES + r * 128 + ((((uint32_t)c & 7u) ^ ((uint32_t)r & 7u)) << 4) + (e & 7) * 2;
+    asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(sk + off), "r"(kb2.x), "r"(kb2.y) : "memory");
+    asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(sv + off), "r"(vb2.x), "r"(vb2.y) : "memory");
+    *reinterpret_cast<uint2*>(a.k_cache + grow + e) = kb2;
+    *reinterpret_cast<uint2*>(a.v_cache + grow + e) = vb2;
+  }
+  fence_proxy_async_smem();
+  __syncwarp();
+}
+
+// Segment (h, s) of layer l is complete with normalised output o[k] for this
+// thread's outputs: x_{l+1} = x_l + o for head group h, its sum of squares,
+// then signal ready[l+1] (or, at the last layer, the per-sequence counter;
+// the last of the Hkv groups writes the final hidden state of s).
+template <int D>
+__device__ bool finish_segment(const StepAttArgs& a, const Scratch& sc, int l, int h, int s,
+                               const float (&xold)[AttCfg<D>::OPT], const float (&o)[AttCfg<D>::OPT], uint32_t bar,
+                               uint32_t& ph, int ctid, int warp, int lane) {
+  using C = AttCfg<D>;
+  const int S = a.S, Hkv = a.Hkv, GD = a.G * D, d = a.Hq * D, nx = (l + 1) & 1;
+  float* xn = a.resid + ((int64_t)nx * S + s) * d + (int64_t)h * GD;
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < C::OPT; ++k) {
+    const int idx = ctid + k * ATT_CT;
+    if (idx >= GD) continue;
+    const float x = xold[k] + o[k];
+    xn[idx] = x;
+    ss += x * x;
   }
   ss = warp_sum(ss);
-  if ((tid & 31) == 0) red[tid >> 5] = ss;
-  __syncthreads();
-  if (tid == 0) {
+  if (lane == 0) sc.red[warp] = ss;
+  if (!warps_sync(bar, ph, a.status)) return false;
+  const bool last_layer = l + 1 == a.L;
+  if (ctid == 0) {
     float t = 0.f;
-    for (int w = 0; w < CMB_THREADS / 32; ++w) t += red[w];
-    a.part_ss[(int64_t)s * Hkv + h] = t;
-    __threadfence();
-    const int prev = atomicAdd(&a.counters[s], 1);
-    last = prev == Hkv - 1;
-    if (last) a.counters[s] = 0;
-  }
-  __syncthreads();
-  if (!last) return;
-  // last CTA of sequence s: normalise the whole residual row (sums in head order)
-  __threadfence();
-  __shared__ float inv_sh;
-  if (tid == 0) {
-    float t = 0.f;
-    for (int hh = 0; hh < Hkv; ++hh) t += __ldcg(&a.part_ss[(int64_t)s * Hkv + hh]);
-    inv_sh = 1.0f / sqrtf(t / (float)d + a.rms_eps);
-  }
-  __syncthreads();
-  const float inv = inv_sh;
-  const int32_t pos = a.seq_len[s] - 1;
-  const int32_t capv = a.cap[s];
-  const bool can_append = a.append && pos >= 0 && pos < capv;
-  const float* xs = a.resid + (int64_t)s * d;
-  for (int idx = tid; idx < d; idx += CMB_THREADS) {
-    const __nv_bfloat16 u = __float2bfloat16_rn(__ldcg(xs + idx) * inv);
-    if (a.append) {
-      a.q_next[(int64_t)s * d + idx] = u;
-      if (can_append && idx < 2 * Hkv * D) {
-        const int hh = idx / D, dd = idx - hh * D;
-        const bool isv = hh >= Hkv;
-        const int hk = isv ? hh - Hkv : hh;
-        const int64_t e = a.next_layer_elem_base + a.kv_offset[s] + ((int64_t)hk * capv + pos) * D + dd;
-        (isv ? a.v_cache : a.k_cache)[e] = u;
-      }
+#pragma unroll
+    for (int w = 0; w < ATT_CONSUMERS; ++w) t += sc.red[w];
+    a.part_ss[((int64_t)nx * S + s) * Hkv + h] = t;
+    if (!last_layer) {
+      red_release_gpu_add(&a.ready[(int64_t)(l + 1) * ATT_FLAG_STRIDE], 1);
     } else {
-      a.hidden[(int64_t)s * d + idx] = u;
-      if (a.hidden_copy) a.hidden_copy[(int64_t)s * d + idx] = u;
+      const int prev = atom_acq_rel_gpu_add(&a.seq_cnt[s], 1);
+      sc.flag[2] = prev == Hkv - 1;
+      if (prev == Hkv - 1) a.seq_cnt[s] = 0;
     }
+  }
+  if (!last_layer) return true;
+  if (!warps_sync(bar, ph, a.status)) return false;
+  if (!sc.flag[2]) return true;
+  // final hidden state h[s] = bf16(x_L[s] * inv_rms(x_L[s]))
+  const float inv = inv_rms(a.part_ss + ((int64_t)nx * S + s) * Hkv, Hkv, d, a.rms_eps, lane);
+  const float2* xs = reinterpret_cast<const float2*>(a.resid + ((int64_t)nx * S + s) * d);
+  uint32_t* hs = reinterpret_cast<uint32_t*>(a.hidden + (int64_t)s * d);
+  uint32_t* hc = a.hidden_copy ? reinterpret_cast<uint32_t*>(a.hidden_copy + (int64_t)s * d) : nullptr;
+  for (int i = ctid; i < d / 2; i += ATT_CT) {
+    const float2 x = __ldcg(xs + i);
+    const uint32_t u = pack_bf16(x.x * inv, x.y * inv);
+    hs[i] = u;
+    if (hc) hc[i] = u;
+  }
+  return true;
+}
+
+template <int D>
+__global__ void __launch_bounds__(ATT_THREADS, 1)
+    att_step_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                    StepAttArgs a) {
+  using C = AttCfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t bar_full = base + C::STAGES * C::STAGE_BYTES;
+  const uint32_t bar_empty = bar_full + C::STAGES * 8;
+  const uint32_t bar_c = bar_empty + C::STAGES * 8;
+  const Scratch sc = carve_scratch<D>(gbase + C::STAGES * C::STAGE_BYTES + C::BARS);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int32_t S = a.S, G = a.G, Hkv = a.Hkv, GD = G * D, d = a.Hq * D;
+
+  if (tid == 0) {
+    for (int i = 0; i < C::STAGES; ++i) {
+      mbar_init(bar_full + 8 * i, 1);
+      mbar_init(bar_empty + 8 * i, 4);
+    }
+    mbar_init(bar_c, ATT_CONSUMERS);
+    mbar_fence_init();
+  }
+  if (warp == ATT_CONSUMERS && lane == 0) {
+    tma_prefetch_desc(&kmap);
+    tma_prefetch_desc(&vmap);
+  }
+  // the next grid (LM head) may be scheduled as SMs free up; it waits for
+  // this grid's completion before reading the hidden states
+  pdl_launch_dependents();
+  // lengths after this step's append (a full cache appends nothing)
+  for (int i = tid; i < S; i += ATT_THREADS) {
+    int32_t n = a.seq_len[i];
+    const int32_t c = a.cap[i];
+    if (n < 0 || n > c) {
+      dev_flag(a.status, PCED_DEV_BAD_LENGTH);
+      n = n < 0 ? 0 : c;
+    }
+    const bool ap = n < c;
+    if (!ap) dev_flag(a.status, PCED_DEV_CACHE_FULL);
+    int32_t len = ap ? n + 1 : n;
+    if (len < 1) {
+      dev_flag(a.status, PCED_DEV_BAD_LENGTH);
+      len = 1;
+    }
+    sc.lens[i] = len;
+    sc.apnd[i] = ap ? 1 : 0;
+  }
+  __syncthreads();
+  if (warp == 0) prefix_extents(sc.lens, S, a.seg_cost, sc.pre, lane);
+  __syncthreads();
+  const int64_t* pre = sc.pre;
+  const int32_t* lens = sc.lens;
+  const int64_t T = pre[S];
+  const int64_t total = (int64_t)Hkv * T;
+  const int64_t P = (total + gridDim.x - 1) / gridDim.x;
+  const int64_t cb = min(total, (int64_t)blockIdx.x * P), ce = min(total, cb + P);
+  const int target = S * Hkv;
+
+  if (warp == ATT_CONSUMERS) {
+    // ------------------------------------------------------------ producer
+    // K/V tiles of every layer in consumption order; the L2 prefetch cursor
+    // runs pf_tiles ahead so HBM keeps streaming while the ring is full
+    if (lane == 0) {
+      const uint64_t pol = policy_evict_first();
+      TileCursor ld, pf;
+      cursor_begin(ld, a, pre, lens, T, cb, ce, D);
+      cursor_begin(pf, a, pre, lens, T, cb, ce, D);
+      for (int i = 0; i < a.pf_tiles && pf.ok; ++i) {
+#pragma unroll
+        for (int b = 0; b < C::BOXES; ++b) {
+          tma_prefetch_l2_2d(&kmap, b * 64, (int32_t)(pf.row0 + pf.kt));
+          tma_prefetch_l2_2d(&vmap, b * 64, (int32_t)(pf.row0 + pf.kt));
+        }
+        cursor_next(pf, a, pre, lens, T, cb, ce, D);
+      }
+      uint32_t it = 0;
+      bool ok = true;
+      while (ld.ok) {
+        const uint32_t st = it % C::STAGES, ph = (it / C::STAGES) & 1u;
+        if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
+          ok = false;
+          break;
+        }
+        const uint32_t fb = bar_full + 8 * st;
+        const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
+        mbar_arrive_expect_tx(fb, C::STAGE_BYTES);
+        const int32_t row = (int32_t)(ld.row0 + ld.kt);
+#pragma unroll
+        for (int b = 0; b < C::BOXES; ++b) {
+          tma_load_2d(sk + b * C::BOX_BYTES, &kmap, fb, b * 64, row, pol);
+          tma_load_2d(sv + b * C::BOX_BYTES, &vmap, fb, b * 64, row, pol);
+        }
+        ++it;
+        cursor_next(ld, a, pre, lens, T, cb, ce, D);
+        if (pf.ok) {
+#pragma unroll
+          for (int b = 0; b < C::BOXES; ++b) {
+            tma_prefetch_l2_2d(&kmap, b * 64, (int32_t)(pf.row0 + pf.kt));
+            tma_prefetch_l2_2d(&vmap, b * 64, (int32_t)(pf.row0 + pf.kt));
+          }
+          cursor_next(pf, a, pre, lens, T, cb, ce, D);
+        }
+      }
+      if (!ok) {
+        for (uint32_t j = (it >= C::STAGES ? it - C::STAGES : 0); j < it; ++j)
+          mbar_wait(bar_full + 8 * (j % C::STAGES), (j / C::STAGES) & 1u, a.status);
+      }
+    }
+    return;
+  }
+
+  // -------------------------------------------------------------- consumers
+  const int ctid = tid, wg = warp >> 2, wl = warp & 3;
+  const int g = lane >> 2, tq = lane & 3;
+  const int kb = 16 * wl;
+  uint32_t it = 0, cph = 0;
+  bool ok = true;
+  for (int s = blockIdx.x; s < S && ok; s += gridDim.x) ok = embed_sequence<D>(a, sc, s, bar_c, cph, ctid, warp, lane);
+
+  for (int l = 0; l < a.L && ok; ++l) {
+    const int par = l & 1;
+    bool open = false;
+    for (int64_t p = cb; p < ce && ok;) {
+      const Piece pc = find_piece(pre, lens, S, T, p, ce);
+      p += pc.adv;
+      if (pc.k0 == pc.k1) continue;
+      if (!open) {
+        // every segment of layer l-1 merged (grid-wide layer dependency)
+        if (ctid == 0) sc.flag[1] = counter_wait(&a.ready[(int64_t)l * ATT_FLAG_STRIDE], target, a.status) ? 1 : 0;
+        if (!warps_sync(bar_c, cph, a.status) || !sc.flag[1]) {
+          ok = false;
+          break;
+        }
+        open = true;
+      }
+      // query bf16(x_l * inv_rms) of head group h, and the stream values of
+      // this thread's outputs (used if this CTA completes the segment)
+      const float* xs = a.resid + ((int64_t)par * S + pc.s) * d;
+      const bool hv = g < G;
+      const float* xq = xs + ((int64_t)pc.h * G + (hv ? g : 0)) * D;
+      float2 xl[C::KSTEPS], xh[C::KSTEPS];
+#pragma unroll
+      for (int j = 0; j < C::KSTEPS; ++j) {
+        xl[j] = __ldcg(reinterpret_cast<const float2*>(xq + 16 * j + 2 * tq));
+        xh[j] = __ldcg(reinterpret_cast<const float2*>(xq + 16 * j + 8 + 2 * tq));
+      }
+      float xold[C::OPT];
+#pragma unroll
+      for (int k = 0; k < C::OPT; ++k) {
+        const int idx = ctid + k * ATT_CT;
+        xold[k] = idx < GD ? __ldcg(xs + (int64_t)pc.h * GD + idx) : 0.f;
+      }
+      const float inv = inv_rms(a.part_ss + ((int64_t)par * S + pc.s) * Hkv, Hkv, d, a.rms_eps, lane);
+      uint32_t qf[C::KSTEPS][2];
+#pragma unroll
+      for (int j = 0; j < C::KSTEPS; ++j) {
+        qf[j][0] = hv ? pack_bf16(xl[j].x * inv, xl[j].y * inv) : 0u;
+        qf[j][1] = hv ? pack_bf16(xh[j].x * inv, xh[j].y * inv) : 0u;
+      }
+      const int32_t app_row = (sc.apnd[pc.s] && pc.k1 == lens[pc.s]) ? lens[pc.s] - 1 : -1;
+
+      WarpAcc<D> A;
+      acc_reset(A);
+      for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
+        if ((int)(it & 1u) != wg) continue;
+        const uint32_t use = it / C::STAGES, st = it % C::STAGES, ph = use & 1u;
+        if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status)) {
+          ok = false;
+          break;
+        }
+        if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
+          ok = false;
+          break;
+        }
+        const int nvalid = min(ATT_BLOCK_N, pc.k1 - kt);
+        const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
+        if (app_row >= kt && app_row < kt + ATT_BLOCK_N && ((app_row - kt) >> 4) == wl)
+          patch_row<D>(a, xs, inv, pc, app_row, app_row - kt, l, sk, sv, lane);
+        if (kb < nvalid) tile_math<D>(A, qf, sk, sv, kb, nvalid, a.scale_log2, lane);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_empty + 8 * st);
+      }
+      if (!ok) break;
+
+      float mx[C::OPT], ls[C::OPT], acc[C::OPT], o[C::OPT];
+      if (!cta_merge<D>(A, sc, G, warp, lane, ctid, bar_c, cph, a.status, mx, ls, acc)) {
+        ok = false;
+        break;
+      }
+      const int64_t seg = (int64_t)pc.h * S + pc.s;
+      const int64_t pa = (int64_t)pc.h * T + pre[pc.s];
+      const int64_t c0 = pa / P, c1 = (pa + lens[pc.s] - 1) / P;
+      if (c0 == c1) {
+        // the whole segment lies in this CTA
+#pragma unroll
+        for (int k = 0; k < C::OPT; ++k) o[k] = ls[k] > 0.f ? acc[k] / ls[k] : 0.f;
+        if (!finish_segment<D>(a, sc, l, pc.h, pc.s, xold, o, bar_c, cph, ctid, warp, lane)) {
+          ok = false;
+          break;
+        }
+        continue;
+      }
+      // publish this CTA's record; the last of the segment's CTAs merges
+      const int64_t slot = (int64_t)blockIdx.x + seg;
+#pragma unroll
+      for (int k = 0; k < C::OPT; ++k) {
+        const int idx = ctid + k * ATT_CT;
+        if (idx >= GD) continue;
+        a.rec_o[slot * GD + idx] = acc[k];
+        if (idx % D == 0) a.rec_ml[slot * G + idx / D] = make_float2(mx[k], ls[k]);
+      }
+      if (!warps_sync(bar_c, cph, a.status)) {
+        ok = false;
+        break;
+      }
+      if (ctid == 0) {
+        int* cnt = &a.seg_cnt[seg];
+        const int prev = atom_acq_rel_gpu_add(cnt, 1);
+        sc.flag[0] = prev == (int)(c1 - c0);
+        if (prev == (int)(c1 - c0)) *cnt = 0;
+      }
+      if (!warps_sync(bar_c, cph, a.status)) {
+        ok = false;
+        break;
+      }
+      if (!sc.flag[0]) continue;
+      // merge records c0..c1 in order (deterministic whichever CTA merges)
+#pragma unroll
+      for (int k = 0; k < C::OPT; ++k) {
+        const int idx = ctid + k * ATT_CT;
+        o[k] = 0.f;
+        if (idx >= GD) continue;
+        const int hh = idx / D;
+        float M = -INFINITY, Ls = 0.f, Ac = 0.f;
+        for (int64_t c = c0; c <= c1; c += 4) {
+          float2 ml[4];
+          float ov[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const bool in = c + u <= c1;
+            ml[u] = in ? __ldcg(a.rec_ml + (c + u + seg) * G + hh) : make_float2(-INFINITY, 0.f);
+            ov[u] = in ? __ldcg(a.rec_o + (c + u + seg) * GD + idx) : 0.f;
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if (ml[u].x == -INFINITY) continue;
+            const float Mn = fmaxf(M, ml[u].x);
+            const float f = M == -INFINITY ? 0.f : exp2f(M - Mn), e = exp2f(ml[u].x - Mn);
+            Ac = Ac * f + ov[u] * e;
+            Ls = Ls * f + ml[u].y * e;
+            M = Mn;
+          }
+        }
+        o[k] = Ls > 0.f ? Ac / Ls : 0.f;
+      }
+      if (!finish_segment<D>(a, sc, l, pc.h, pc.s, xold, o, bar_c, cph, ctid, warp, lane)) {
+        ok = false;
+        break;
+      }
+    }
+  }
+
+  // ---- the last CTA to finish zeroes the layer counters and advances seq_len
+  if (ctid == 0) {
+    const int prev = atom_acq_rel_gpu_add(a.done_cnt, 1);
+    sc.flag[3] = prev == (int)gridDim.x - 1;
+  }
+  if (warps_sync(bar_c, cph, a.status) && sc.flag[3]) {
+    for (int l = ctid; l < a.L; l += ATT_CT) a.ready[(int64_t)l * ATT_FLAG_STRIDE] = 0;
+    for (int i = ctid; i < S; i += ATT_CT)
+      if (sc.apnd[i]) a.seq_len[i] = lens[i];
+    if (ctid == 0) *a.done_cnt = 0;
   }
 }
 
@@ -497,16 +957,38 @@ int att_grid(int64_t total_cap_keys) {
   return (int)(g < 1 ? 1 : g);
 }
 
+int64_t att_step_slots(int32_t S, int32_t Hkv) { return ATT_MAX_CTAS + (int64_t)S * Hkv; }
+
+static int env_int(const char* name, int dflt, int lo, int hi) {
+  const char* e = getenv(name);
+  if (!e || !*e) return dflt;
+  const int v = atoi(e);
+  return v < lo ? lo : (v > hi ? hi : v);
+}
+int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", D == 128 ? 1024 : 2048, 0, 1 << 20); }
+int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 6, 0, 64); }
+
+// cudaFuncSetAttribute once per kernel and device
+template <typename K>
+static cudaError_t set_smem_once(K kernel, size_t bytes, bool* done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!done[dev]) {
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e != cudaSuccess) return e;
+    done[dev] = true;
+  }
+  return cudaSuccess;
+}
+
 template <int D>
 static cudaError_t launch_split(const CUtensorMap& kmap, const CUtensorMap& vmap, const AttArgs& a, int ctas,
                                 cudaStream_t stream) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(att_split_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)AttCfg<D>::SMEM);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static bool configured[64];
+  cudaError_t e = set_smem_once(att_split_kernel<D>, AttCfg<D>::SMEM, configured);
+  if (e != cudaSuccess) return e;
   att_split_kernel<D><<<ctas, ATT_THREADS, AttCfg<D>::SMEM, stream>>>(kmap, vmap, a);
   return cudaGetLastError();
 }
@@ -521,6 +1003,34 @@ cudaError_t att_split_launch(int D, const CUtensorMap& kmap, const CUtensorMap& 
 cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream) {
   att_combine_kernel<<<dim3(a.Hkv, a.S), CMB_THREADS, 0, stream>>>(a);
   return cudaGetLastError();
+}
+
+template <int D>
+static cudaError_t launch_step(const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
+                               cudaStream_t stream) {
+  static bool configured[64];
+  cudaError_t e = set_smem_once(att_step_kernel<D>, AttCfg<D>::SMEM, configured);
+  if (e != cudaSuccess) return e;
+  // every CTA waits for the others' layer results, so all must be resident at
+  // once: a cooperative launch guarantees it (or fails)
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(ctas);
+  cfg.blockDim = dim3(ATT_THREADS);
+  cfg.dynamicSmemBytes = AttCfg<D>::SMEM;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, att_step_kernel<D>, kmap, vmap, a);
+}
+
+cudaError_t att_step_launch(int D, const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
+                            cudaStream_t stream) {
+  if (D == 128) return launch_step<128>(kmap, vmap, a, ctas, stream);
+  if (D == 64) return launch_step<64>(kmap, vmap, a, ctas, stream);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace pced
@@ -588,7 +1098,6 @@ extern "C" pced_status pced_decode_attention(const void* q, const void* k_cache,
   if (e != cudaSuccess) return cuda_status(e, "attention split launch");
 
   CombineArgs c = {};
-  c.mode = 0;
   c.S = S;
   c.Hq = Hq;
   c.Hkv = Hkv;
@@ -598,7 +1107,6 @@ extern "C" pced_status pced_decode_attention(const void* q, const void* k_cache,
   c.rec_ml = a.rec_ml;
   c.plan_pre = a.plan_pre;
   c.plan_per = a.plan_per;
-  c.seq_len = seq_len;
   c.out = out;
   c.status = a.status;
   e = att_combine_launch(c, s);

@@ -1,5 +1,5 @@
 // attention.cuh -- split-KV decode attention over per-expert caches (declarations
-// shared by the attention translation unit and the step orchestration).
+// shared by the attention translation units and the step orchestration).
 #pragma once
 #include "common.cuh"
 
@@ -9,10 +9,13 @@ constexpr int ATT_BLOCK_N = 64;     // keys per pipeline stage
 constexpr int ATT_CONSUMERS = 8;    // two warpgroups of four warps; warpgroup g takes the CTA's tiles with
                                     // index = g (mod 2), warp w of a group owns keys [16w, 16w+16) of a tile
 constexpr int ATT_THREADS = (ATT_CONSUMERS + 1) * 32;
+constexpr int ATT_CT = ATT_CONSUMERS * 32;  // consumer threads
 constexpr int ATT_MAX_S = 1024;     // sequences per launch (prefix table lives in shared memory)
 constexpr int ATT_MAX_G = 8;        // query heads per kv-head (mma N = 8)
 constexpr int ATT_MAX_CTAS = 1024;  // upper bound of the grid (sizes the partial-record pool)
+constexpr int ATT_FLAG_STRIDE = 32; // ints between layer counters: each owns a 128-byte line
 
+// ---------------------------------------------------------------- one layer
 // Partition of all (kv-head, sequence, key) positions into equal contiguous
 // ranges, one per CTA.  Position of key k of kv-head h of sequence s:
 //   h * T + pre[s] + k,   pre[s] = sum_{s' < s} len[s'],  T = pre[S].
@@ -42,36 +45,75 @@ int att_grid(int64_t total_cap_keys);
 cudaError_t att_split_launch(int D, const CUtensorMap& kmap, const CUtensorMap& vmap, const AttArgs& a, int ctas,
                              cudaStream_t stream);
 
-// Combine the partial records of one layer; one CTA per (kv-head, sequence).
-//   mode 0: out[s][hq][dd] = o (fp32)
-//   mode 1: resid[s] += o for the CTA's heads; the last CTA of a sequence
-//           then forms u = bf16(rmsnorm(resid[s])) and either writes u to
-//           q_next and appends the next layer's K/V rows at seq_len[s]-1, or
-//           (last layer) writes u to hidden (and hidden_copy if non-null).
+// Combine the partial records of one layer; one CTA per (kv-head, sequence):
+// out[s][hq][dd] = o (fp32).
 struct CombineArgs {
-  int mode;
   int32_t S, Hq, Hkv, G, D;
   const float* rec_o;
   const float2* rec_ml;
   const int64_t* plan_pre;
   const int64_t* plan_per;
-  const int32_t* seq_len;
-  float* out;                 // mode 0
-  float* resid;               // mode 1 [S][d]
-  float* part_ss;             // mode 1 [S][Hkv] partial sums of squares
-  int32_t* counters;          // mode 1 [S] arrival counters (zero between launches)
-  float rms_eps;
-  __nv_bfloat16* q_next;      // mode 1, not last layer
-  __nv_bfloat16* hidden;      // mode 1, last layer
-  __nv_bfloat16* hidden_copy; // optional
-  __nv_bfloat16* k_cache;     // mode 1: caches and geometry for the append
-  __nv_bfloat16* v_cache;
-  const int64_t* kv_offset;
-  const int32_t* cap;
-  int64_t next_layer_elem_base;  // element offset of the next layer's region
-  int append;                 // 1: append into the next layer (not last layer)
+  float* out;
   int* status;
 };
 cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream);
+
+// ------------------------------------------------------- whole decode step
+// One cooperative launch runs the embedding and every layer of the step.
+//
+// Partition: head-major positions as above, but each segment (h, s) spans
+// len[s] + seg_cost positions; the last seg_cost hold no keys and stand for
+// the fixed cost of a piece (query formation, partial merge, record), so CTAs
+// that cover many short segments get fewer keys.  The partition is the same
+// at every layer, so the producer warp streams K/V tiles straight through all
+// layers (a shared-memory ring plus L2 prefetch ahead of it) while the
+// consumers wait for the layer dependency.
+//
+// Layer dependency: the CTA that completes segment (h, s) at layer l (last
+// of its record writers, or the only one) merges the records, adds the head
+// group's attention output to the residual stream, x_{l+1} = x_l + o (double
+// buffered by layer parity), stores the group's sum of squares and adds one
+// to the layer counter ready[l+1]; the embedding adds Hkv per sequence to
+// ready[0].  A CTA starts the compute of layer l once ready[l] = S*Hkv (all
+// of layer l-1 merged).  Every piece forms its query bf16(x_l * inv_rms(x_l))
+// itself; the warp that owns the row appended this step writes that row's
+// K/V (the same normalised stream) into the shared tile and the cache.  At the
+// last layer a per-sequence counter picks the CTA that writes the final
+// hidden state.  The last CTA to finish zeroes the counters and advances
+// seq_len.
+struct StepAttArgs {
+  int32_t S, Hq, Hkv, G, L, n1, V, bos, max_steps;
+  int64_t rows_per_layer;     // rows (of D elements) of one layer's region in the tensor maps
+  int64_t layer_elems;
+  float scale_log2, rms_eps;
+  int32_t seg_cost;           // partition weight of a piece, in keys
+  int32_t pf_tiles;           // tiles prefetched into L2 ahead of the shared-memory ring
+  const int64_t* kv_offset;   // [S]
+  const int32_t* cap;         // [S]
+  int32_t* seq_len;           // [S] +1 per launch for every sequence with room
+  const int32_t* step;        // [1] step counter t (token y_{t-1} = history[b][t-1])
+  const int32_t* history;     // [B][max_steps]
+  const __nv_bfloat16* embed; // [V][d]
+  __nv_bfloat16* k_cache;
+  __nv_bfloat16* v_cache;
+  float* resid;               // [2][S][d]
+  float* part_ss;             // [2][S][Hkv]
+  float* rec_o;               // [slots][G][D]
+  float2* rec_ml;             // [slots][G]
+  int32_t* seg_cnt;           // [Hkv*S] arrival counters (zero between launches)
+  int32_t* seq_cnt;           // [S] last-layer arrival counters (zero between launches)
+  int32_t* ready;             // [L * ATT_FLAG_STRIDE] layer counters (zero between launches)
+  int32_t* done_cnt;          // [1] (zero between launches)
+  __nv_bfloat16* hidden;      // [S][d] final hidden state
+  __nv_bfloat16* hidden_copy; // optional copy of `hidden`
+  int* status;
+};
+int64_t att_step_slots(int32_t S, int32_t Hkv);
+// tuning of the partition and the prefetch distance (PCED_ATT_SEGCOST /
+// PCED_ATT_PF in the environment override the defaults)
+int att_step_seg_cost(int D);
+int att_step_pf_tiles();
+cudaError_t att_step_launch(int D, const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
+                            cudaStream_t stream);
 
 }  // namespace pced

@@ -140,7 +140,6 @@ extern "C" pced_status pced_decode_attention_noalloc(const void* q, const void* 
   if (e != cudaSuccess) return cuda_status(e, "pced_decode_attention_noalloc: split launch");
 
   CombineArgs c = {};
-  c.mode = 0;
   c.S = S;
   c.Hq = Hq;
   c.Hkv = Hkv;
@@ -150,7 +149,6 @@ extern "C" pced_status pced_decode_attention_noalloc(const void* q, const void* 
   c.rec_ml = a.rec_ml;
   c.plan_pre = a.plan_pre;
   c.plan_per = a.plan_per;
-  c.seq_len = seq_len;
   c.out = out;
   c.status = a.status;
   e = att_combine_launch(c, s);

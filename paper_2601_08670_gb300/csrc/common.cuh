@@ -81,6 +81,60 @@ __device__ __forceinline__ bool bar_sync_bounded(uint32_t bar, uint32_t& phase, 
   return ok;
 }
 
+// Barrier among whole warps on an mbarrier initialised with the number of
+// participating warps: lane 0 of each warp arrives and waits (bounded), the
+// rest of the warp follows it.  Writes made by any lane before the call are
+// visible to every participant after it.
+__device__ __forceinline__ bool warps_sync(uint32_t bar, uint32_t& phase, int* status) {
+  __syncwarp();
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) {
+    mbar_arrive(bar);
+    ok = mbar_wait(bar, phase, status) ? 1 : 0;
+  }
+  phase ^= 1u;
+  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+// ------------------------------------------- signalling between CTAs (gpu scope)
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// Release: every write this thread has observed (its own, and other threads'
+// ordered before it by a CTA barrier) is visible before the add.
+__device__ __forceinline__ void red_release_gpu_add(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int atom_acq_rel_gpu_add(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
+}
+// Wait until *p >= target (acquire).  Bounded like mbar_wait.
+static __device__ __noinline__ bool counter_wait(const int* p, int target, int* status) {
+  for (int i = 0; i < 8; ++i)
+    if (ld_acquire_gpu(p) >= target) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    __nanosleep(64);
+    if (ld_acquire_gpu(p) >= target) return true;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      dev_flag(status, PCED_DEV_TIMEOUT);
+      return false;
+    }
+  }
+}
+// generic-proxy writes to shared memory, ordered before later TMA writes to it
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+// programmatic dependent launch: wait for the preceding grid's completion and
+// memory, and allow the next grid to be scheduled
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ------------------------------------------------------------------ TMA copies
 __device__ __forceinline__ uint64_t policy_evict_first() {
   uint64_t p;
@@ -104,6 +158,12 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, uint
       " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
       "l"(tmap), "r"(bar), "r"(x), "r"(y), "l"(policy)
       : "memory");
+}
+
+// L2 prefetch of one tensor-map box (no shared memory, no completion tracking)
+__device__ __forceinline__ void tma_prefetch_l2_2d(const void* tmap, int32_t x, int32_t y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(tmap), "r"(x), "r"(y)
+               : "memory");
 }
 
 // --------------------------------------------------------- ldmatrix / mma.sync

@@ -1,138 +1,55 @@
 // step.cu -- one greedy PCED decode step for all queries (paper Sec. 3: the
 // N+1 experts run as one batch; Eq. 2 + Eq. 3 pick the token, which joins
-// every expert's history).  Launch sequence on one stream, no host sync:
-//   embed      x_0 = E[y_{t-1}], u = bf16(rmsnorm(x_0)), append layer-0 K/V, seq_len += 1
-//   L times    split-KV attention, then combine: x += o, u = bf16(rmsnorm(x)),
-//              append the next layer's K/V (or write h after the last layer)
+// every expert's history).  Three launches on one stream, no host sync:
+//   attention  one cooperative kernel: x_0 = E[y_{t-1}], then for every layer
+//              u = bf16(rmsnorm(x)), append K/V row of u, x += attention(u);
+//              h = bf16(rmsnorm(x_L)); seq_len += 1
 //   lm head    tcgen05 GEMM with log-softmax statistics + contrastive tile maxima
 //   select     Eq. 2 + Eq. 3 per query, history[b][t] = y, t += 1
 // Every quantity that changes between steps (t, lengths, history) lives on
 // the device, so one captured call replays as the next step.
 #include <math.h>
+#include <stdlib.h>
 
 #include "attention.cuh"
 #include "lm_head.cuh"
 
 namespace pced {
 
-constexpr int EMB_THREADS = 256;
-constexpr int EMB_MAX_PER_THREAD = 32;  // d <= 8192
-
-struct EmbedArgs {
-  const __nv_bfloat16* embed;
-  int32_t S, n1, d, Hkv, D, V, max_steps, bos;
-  const int32_t* step;
-  const int32_t* history;
-  int32_t* seq_len;
-  const int32_t* cap;
-  const int64_t* kv_offset;
-  __nv_bfloat16* k_cache;
-  __nv_bfloat16* v_cache;
-  float* resid;
-  __nv_bfloat16* q;
-  float rms_eps;
-  int* status;
-};
-
-__global__ void __launch_bounds__(EMB_THREADS) step_embed_kernel(EmbedArgs a) {
-  const int s = blockIdx.x, tid = threadIdx.x, b = s / a.n1, d = a.d;
-  __shared__ int sh_tok, sh_pos;
-  __shared__ float red[EMB_THREADS / 32];
-  if (tid == 0) {
-    const int t = *a.step;
-    int tok = a.bos;
-    if (t > 0 && t <= a.max_steps) tok = a.history[(int64_t)b * a.max_steps + t - 1];
-    if (t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
-    if (tok < 0 || tok >= a.V) {
-      dev_flag(a.status, PCED_DEV_BAD_TOKEN);
-      tok = 0;
-    }
-    const int L = a.seq_len[s], c = a.cap[s];
-    int pos = -1;
-    if (L < 0 || L >= c) {
-      dev_flag(a.status, PCED_DEV_CACHE_FULL);
-    } else {
-      a.seq_len[s] = L + 1;
-      pos = L;
-    }
-    sh_tok = tok;
-    sh_pos = pos;
-  }
-  __syncthreads();
-  const __nv_bfloat16* e = a.embed + (int64_t)sh_tok * d;
-  float xv[EMB_MAX_PER_THREAD];
-  float ss = 0.f;
-#pragma unroll
-  for (int j = 0; j < EMB_MAX_PER_THREAD; ++j) {
-    const int i = tid + j * EMB_THREADS;
-    xv[j] = 0.f;
-    if (i < d) {
-      xv[j] = __bfloat162float(e[i]);
-      a.resid[(int64_t)s * d + i] = xv[j];
-      ss += xv[j] * xv[j];
-    }
-  }
-  ss = warp_sum(ss);
-  if ((tid & 31) == 0) red[tid >> 5] = ss;
-  __syncthreads();
-  if (tid < 32) {
-    float v = tid < EMB_THREADS / 32 ? red[tid] : 0.f;
-    v = warp_sum(v);
-    if (tid == 0) red[0] = v;
-  }
-  __syncthreads();
-  const float inv = 1.0f / sqrtf(red[0] / (float)d + a.rms_eps);
-  const int pos = sh_pos, capv = a.cap[s];
-#pragma unroll
-  for (int j = 0; j < EMB_MAX_PER_THREAD; ++j) {
-    const int i = tid + j * EMB_THREADS;
-    if (i >= d) continue;
-    const __nv_bfloat16 u = __float2bfloat16_rn(xv[j] * inv);
-    a.q[(int64_t)s * d + i] = u;
-    if (pos >= 0 && i < 2 * a.Hkv * a.D) {
-      const int hh = i / a.D, dd = i - hh * a.D;
-      const bool isv = hh >= a.Hkv;
-      const int hk = isv ? hh - a.Hkv : hh;
-      const int64_t el = a.kv_offset[s] + ((int64_t)hk * capv + pos) * a.D + dd;
-      (isv ? a.v_cache : a.k_cache)[el] = u;
-    }
-  }
-}
-
 struct StepLayout {
   int* status;
+  int32_t* done_counter;  // selection kernel: queries finished this step
+  int32_t* att_done;      // attention: CTAs finished
+  int32_t* seg_cnt;
+  int32_t* seq_cnt;
+  int32_t* ready;
+  float* part_ss;
   float* resid;
-  __nv_bfloat16* q;
   __nv_bfloat16* h;
   float* rec_o;
   float2* rec_ml;
-  int64_t* plan_pre;
-  int64_t* plan_per;
   float2* lm_stats;
   float2* lm_arg;
-  int32_t* done_counter;
-  float* part_ss;
-  int32_t* seq_counters;
   size_t bytes;
 };
 
 static StepLayout step_layout(const pced_dims* dm, void* ws) {
   const int32_t S = dm->B * (dm->N + 1), d = dm->Hq * dm->D, G = dm->Hq / dm->Hkv;
-  const int64_t slots = ATT_MAX_CTAS + (int64_t)S * dm->Hkv;
+  const int64_t slots = att_step_slots(S, dm->Hkv);
   const int64_t ntiles = (dm->V + LM_TILE_V - 1) / LM_TILE_V;
   StepLayout L;
   pced_host::Carver c(ws);
   L.status = c.take<int>(64);
   L.done_counter = c.take<int32_t>(1);
-  L.seq_counters = c.take<int32_t>((size_t)S);
-  L.part_ss = c.take<float>((size_t)S * dm->Hkv);
-  L.resid = c.take<float>((size_t)S * d);
-  L.q = c.take<__nv_bfloat16>((size_t)S * d);
+  L.att_done = c.take<int32_t>(1);
+  L.seg_cnt = c.take<int32_t>((size_t)S * dm->Hkv);
+  L.seq_cnt = c.take<int32_t>((size_t)S);
+  L.ready = c.take<int32_t>((size_t)(dm->L > 0 ? dm->L : 1) * ATT_FLAG_STRIDE);
+  L.part_ss = c.take<float>((size_t)2 * S * dm->Hkv);
+  L.resid = c.take<float>((size_t)2 * S * d);
   L.h = c.take<__nv_bfloat16>((size_t)S * d);
   L.rec_o = c.take<float>((size_t)(slots * G * dm->D));
   L.rec_ml = c.take<float2>((size_t)(slots * G));
-  L.plan_pre = c.take<int64_t>((size_t)S + 1);
-  L.plan_per = c.take<int64_t>(1);
   L.lm_stats = c.take<float2>((size_t)(S * ntiles));
   L.lm_arg = c.take<float2>((size_t)(S * ntiles));
   L.bytes = c.used();
@@ -150,13 +67,12 @@ extern "C" size_t pced_step_workspace_size(const pced_dims* dm) {
   return step_layout(dm, nullptr).bytes;
 }
 
-extern "C" int32_t pced_step_launch_count(const pced_dims* dm) { return dm ? 1 + 2 * dm->L + 2 : 0; }
+extern "C" int32_t pced_step_launch_count(const pced_dims* dm) { return dm ? 3 : 0; }
 
 extern "C" const char* pced_step_launch_kind(const pced_dims* dm, int32_t i) {
+  static const char* kinds[3] = {"attention", "lm_head", "select"};
   if (!dm || i < 0 || i >= pced_step_launch_count(dm)) return nullptr;
-  if (i == 0) return "embed";
-  if (i <= 2 * dm->L) return (i % 2 == 1) ? "attn_split" : "attn_combine";
-  return i == 2 * dm->L + 1 ? "lm_head" : "select";
+  return kinds[i];
 }
 
 extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
@@ -211,87 +127,44 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   cudaError_t e = mark();
   if (e != cudaSuccess) return cuda_status(e, "stage event");
 
-  EmbedArgs ea;
-  ea.embed = (const __nv_bfloat16*)p->embed;
-  ea.S = S;
-  ea.n1 = dm.N + 1;
-  ea.d = d;
-  ea.Hkv = dm.Hkv;
-  ea.D = dm.D;
-  ea.V = dm.V;
-  ea.max_steps = p->max_steps;
-  ea.bos = p->bos_token;
-  ea.step = p->step;
-  ea.history = p->history;
-  ea.seq_len = p->seq_len;
-  ea.cap = p->cap;
-  ea.kv_offset = p->kv_offset;
-  ea.k_cache = (__nv_bfloat16*)p->k_cache;
-  ea.v_cache = (__nv_bfloat16*)p->v_cache;
-  ea.resid = W.resid;
-  ea.q = W.q;
-  ea.rms_eps = p->rms_eps;
-  ea.status = W.status;
-  step_embed_kernel<<<S, EMB_THREADS, 0, s>>>(ea);
-  e = cudaGetLastError();
+  StepAttArgs at = {};
+  at.S = S;
+  at.Hq = dm.Hq;
+  at.Hkv = dm.Hkv;
+  at.G = G;
+  at.L = dm.L;
+  at.n1 = dm.N + 1;
+  at.V = dm.V;
+  at.bos = p->bos_token;
+  at.max_steps = p->max_steps;
+  at.rows_per_layer = p->layer_elems / dm.D;
+  at.layer_elems = p->layer_elems;
+  at.scale_log2 = p->attn_scale * 1.4426950408889634f;
+  at.rms_eps = p->rms_eps;
+  at.seg_cost = att_step_seg_cost(dm.D);
+  at.pf_tiles = att_step_pf_tiles();
+  at.kv_offset = p->kv_offset;
+  at.cap = p->cap;
+  at.seq_len = p->seq_len;
+  at.step = p->step;
+  at.history = p->history;
+  at.embed = (const __nv_bfloat16*)p->embed;
+  at.k_cache = (__nv_bfloat16*)p->k_cache;
+  at.v_cache = (__nv_bfloat16*)p->v_cache;
+  at.resid = W.resid;
+  at.part_ss = W.part_ss;
+  at.rec_o = W.rec_o;
+  at.rec_ml = W.rec_ml;
+  at.seg_cnt = W.seg_cnt;
+  at.seq_cnt = W.seq_cnt;
+  at.ready = W.ready;
+  at.done_cnt = W.att_done;
+  at.hidden = W.h;
+  at.hidden_copy = (__nv_bfloat16*)p->hidden_out;
+  at.status = W.status;
+  e = att_step_launch(dm.D, kmap, vmap, at, att_grid(p->total_cap * dm.Hkv), s);
   if (e == cudaSuccess) e = mark();
-  if (e != cudaSuccess) return cuda_status(e, "embed launch");
-
-  const int ctas = att_grid(p->total_cap * dm.Hkv);
-  for (int l = 0; l < dm.L; ++l) {
-    AttArgs a;
-    a.q = W.q;
-    a.kv_offset = p->kv_offset;
-    a.cap = p->cap;
-    a.seq_len = p->seq_len;
-    a.S = S;
-    a.Hq = dm.Hq;
-    a.Hkv = dm.Hkv;
-    a.G = G;
-    a.row_base = (int64_t)l * (p->layer_elems / dm.D);
-    a.scale_log2 = p->attn_scale * 1.4426950408889634f;
-    a.rec_o = W.rec_o;
-    a.rec_ml = W.rec_ml;
-    a.plan_pre = W.plan_pre;
-    a.plan_per = W.plan_per;
-    a.status = W.status;
-    e = att_split_launch(dm.D, kmap, vmap, a, ctas, s);
-    if (e == cudaSuccess) e = mark();
-    if (e != cudaSuccess) return cuda_status(e, "attention split launch");
-    CombineArgs c = {};
-    c.mode = 1;
-    c.S = S;
-    c.Hq = dm.Hq;
-    c.Hkv = dm.Hkv;
-    c.G = G;
-    c.D = dm.D;
-    c.rec_o = W.rec_o;
-    c.rec_ml = W.rec_ml;
-    c.plan_pre = W.plan_pre;
-    c.plan_per = W.plan_per;
-    c.seq_len = p->seq_len;
-    c.resid = W.resid;
-    c.part_ss = W.part_ss;
-    c.counters = W.seq_counters;
-    c.rms_eps = p->rms_eps;
-    c.k_cache = (__nv_bfloat16*)p->k_cache;
-    c.v_cache = (__nv_bfloat16*)p->v_cache;
-    c.kv_offset = p->kv_offset;
-    c.cap = p->cap;
-    c.status = W.status;
-    if (l + 1 < dm.L) {
-      c.append = 1;
-      c.q_next = W.q;
-      c.next_layer_elem_base = (int64_t)(l + 1) * p->layer_elems;
-    } else {
-      c.append = 0;
-      c.hidden = W.h;
-      c.hidden_copy = (__nv_bfloat16*)p->hidden_out;
-    }
-    e = att_combine_launch(c, s);
-    if (e == cudaSuccess) e = mark();
-    if (e != cudaSuccess) return cuda_status(e, "attention combine launch");
-  }
+  if (e != cudaSuccess) return cuda_status(e, "attention launch");
 
   LmArgs la = {};
   la.mode = 1;

@@ -107,7 +107,8 @@ def test_step_rejects_bad_arguments(L):
 def test_launch_count_and_workspace_sizes(L):
     import paper_2601_08670_gb300 as pced
     dm = pced.dims(1, 8, 32, 32, 8, 128, 128256)
-    assert pced.step_launch_count(dm) == 2 * 32 + 3
+    assert pced.step_launch_count(dm) == 3
+    assert pced.step_launch_kinds(dm) == ["attention", "lm_head", "select"]
     assert pced.step_workspace_size(dm) > 0
     assert pced.step_workspace_size(pced.dims(1, 8, 32, 30, 8, 128, 100)) == 0
     assert L.pced_decode_attention_workspace_size(9, 32, 8, 128) > 0
