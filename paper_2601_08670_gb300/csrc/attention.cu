@@ -149,8 +149,8 @@ __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D 
                                           int kb, int nvalid, float scale_log2, int lane) {
   using C = AttCfg<D>;
   const int g = lane >> 2, tq = lane & 3, mat = lane >> 3, mr = lane & 7;
-  // ---- scores S^T (16 keys x 8 heads), two independent accumulation chains
-  float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+  // ---- scores S^T (16 keys x 8 heads), four independent accumulation chains
+  float sc4[4][4] = {};
   {
     const int key = kb + (mat & 1) * 8 + mr;
     const uint32_t rowa = sk + key * 128;
@@ -161,35 +161,44 @@ __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D 
       const uint32_t addr = rowa + (chunk >> 3) * C::BOX_BYTES + (((chunk & 7) ^ sw) << 4);
       uint32_t a0, a1, a2, a3;
       ldsm_x4(addr, a0, a1, a2, a3);
-      mma_bf16((j & 1) ? sb : sa, a0, a1, a2, a3, qf[j][0], qf[j][1]);
+      mma_bf16(sc4[j & 3], a0, a1, a2, a3, qf[j][0], qf[j][1]);
     }
   }
   const bool v0 = kb + g < nvalid, v1 = kb + g + 8 < nvalid;
-  const float s0 = v0 ? (sa[0] + sb[0]) * scale_log2 : -INFINITY;
-  const float s1 = v0 ? (sa[1] + sb[1]) * scale_log2 : -INFINITY;
-  const float s2 = v1 ? (sa[2] + sb[2]) * scale_log2 : -INFINITY;
-  const float s3 = v1 ? (sa[3] + sb[3]) * scale_log2 : -INFINITY;
+  const float s0 = v0 ? ((sc4[0][0] + sc4[1][0]) + (sc4[2][0] + sc4[3][0])) * scale_log2 : -INFINITY;
+  const float s1 = v0 ? ((sc4[0][1] + sc4[1][1]) + (sc4[2][1] + sc4[3][1])) * scale_log2 : -INFINITY;
+  const float s2 = v1 ? ((sc4[0][2] + sc4[1][2]) + (sc4[2][2] + sc4[3][2])) * scale_log2 : -INFINITY;
+  const float s3 = v1 ? ((sc4[0][3] + sc4[1][3]) + (sc4[2][3] + sc4[3][3])) * scale_log2 : -INFINITY;
+  // The reference max only moves when a score exceeds it by more than
+  // ATT_RESCALE_SLACK (log2 units): exp2 of the others stays below
+  // 2^ATT_RESCALE_SLACK, and the rescale of o, l (and the max reduction across
+  // the warp) is skipped for most tiles.  Any reference gives the same o / l.
   float x0 = fmaxf(s0, s2), x1 = fmaxf(s1, s3);
+  if (__any_sync(0xffffffffu, x0 > A.m0 + ATT_RESCALE_SLACK || x1 > A.m1 + ATT_RESCALE_SLACK)) {
 #pragma unroll
-  for (int off = 4; off < 32; off <<= 1) {
-    x0 = fmaxf(x0, __shfl_xor_sync(0xffffffffu, x0, off));
-    x1 = fmaxf(x1, __shfl_xor_sync(0xffffffffu, x1, off));
+    for (int off = 4; off < 32; off <<= 1) {
+      x0 = fmaxf(x0, __shfl_xor_sync(0xffffffffu, x0, off));
+      x1 = fmaxf(x1, __shfl_xor_sync(0xffffffffu, x1, off));
+    }
+    const float n0 = fmaxf(A.m0, x0), n1 = fmaxf(A.m1, x1);
+    const float al0 = A.m0 == -INFINITY ? 0.f : exp2f(A.m0 - n0);
+    const float al1 = A.m1 == -INFINITY ? 0.f : exp2f(A.m1 - n1);
+    A.l0 *= al0;
+    A.l1 *= al1;
+#pragma unroll
+    for (int i = 0; i < C::MTILES; ++i) {
+      A.o[i][0] *= al0;
+      A.o[i][2] *= al0;
+      A.o[i][1] *= al1;
+      A.o[i][3] *= al1;
+    }
+    A.m0 = n0;
+    A.m1 = n1;
   }
-  const float n0 = fmaxf(A.m0, x0), n1 = fmaxf(A.m1, x1);
-  const float u0 = n0 == -INFINITY ? 0.f : n0, u1 = n1 == -INFINITY ? 0.f : n1;
-  const float al0 = exp2f(A.m0 - u0), al1 = exp2f(A.m1 - u1);
+  const float u0 = A.m0 == -INFINITY ? 0.f : A.m0, u1 = A.m1 == -INFINITY ? 0.f : A.m1;
   const float p0 = exp2f(s0 - u0), p1 = exp2f(s1 - u1), p2 = exp2f(s2 - u0), p3 = exp2f(s3 - u1);
-  A.l0 = A.l0 * al0 + p0 + p2;
-  A.l1 = A.l1 * al1 + p1 + p3;
-  A.m0 = n0;
-  A.m1 = n1;
-#pragma unroll
-  for (int i = 0; i < C::MTILES; ++i) {
-    A.o[i][0] *= al0;
-    A.o[i][2] *= al0;
-    A.o[i][1] *= al1;
-    A.o[i][3] *= al1;
-  }
+  A.l0 += p0 + p2;
+  A.l1 += p1 + p3;
   // ---- P^T as the B operand (keys x heads), split into bf16 hi + lo
   const uint32_t h01 = pack_bf16(p0, p1), h23 = pack_bf16(p2, p3);
   const uint32_t q01 = pack_bf16(p0 - bf16_lo(h01), p1 - bf16_hi(h01));
@@ -224,8 +233,7 @@ __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D 
 // Merge the eight consumer warps' accumulators of a piece through shared
 // memory.  Afterwards this thread holds, for outputs idx = ctid + k*ATT_CT
 // (idx = hh*D + dd < G*D), the piece's running max mx[k] (log2 units), sum
-// ls[k] and unnormalised output acc[k].  The caller must pass another
-// consumer barrier before the next call (the scratch is reused).
+// ls[k] and unnormalised output acc[k].
 template <int D>
 __device__ __forceinline__ bool cta_merge(const WarpAcc<D>& A, const Scratch& sc, int G, int warp, int lane, int ctid,
                                           uint32_t bar, uint32_t& ph, int* status, float (&mx)[AttCfg<D>::OPT],
@@ -238,6 +246,8 @@ __device__ __forceinline__ bool cta_merge(const WarpAcc<D>& A, const Scratch& sc
     l0 += __shfl_xor_sync(0xffffffffu, l0, off);
     l1 += __shfl_xor_sync(0xffffffffu, l1, off);
   }
+  // every consumer is done with the previous piece's scratch
+  if (!warps_sync(bar, ph, status)) return false;
   if (g == 0) {
     sc.ms[warp * ATT_MAX_G + 2 * tq] = A.m0;
     sc.ms[warp * ATT_MAX_G + 2 * tq + 1] = A.m1;
@@ -495,6 +505,39 @@ __global__ void __launch_bounds__(CMB_THREADS) att_combine_kernel(CombineArgs a)
 }
 
 // ============================================================ whole step
+// Values exchanged between CTAs inside the step kernel are 64-bit words
+// (fp32 value, 32-bit tag) written and read with single relaxed gpu-scope
+// accesses, so a reader that sees the expected tag also sees the value: no
+// fences or arrival counters are needed, and a wait is a poll on the data
+// itself.  tag(l) = (epoch << 10) | (l + 1) names the launch and the layer
+// whose input the word belongs to (never 0, so zeroed memory never matches).
+__device__ __forceinline__ uint32_t step_tag(int32_t epoch, int l) {
+  return ((uint32_t)epoch << 10) | (uint32_t)(l + 1);
+}
+__device__ __forceinline__ void st_tagged(uint64_t* p, float v, uint32_t tag) {
+  const uint64_t w = ((uint64_t)tag << 32) | (uint64_t)__float_as_uint(v);
+  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(w) : "memory");
+}
+__device__ __forceinline__ uint64_t ld_tagged(const uint64_t* p) {
+  uint64_t w;
+  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(w) : "l"(p) : "memory");
+  return w;
+}
+__device__ __forceinline__ float tv_value(uint64_t w) { return __uint_as_float((uint32_t)w); }
+__device__ __forceinline__ bool tv_ok(uint64_t w, uint32_t tag) { return (uint32_t)(w >> 32) == tag; }
+
+// Bounded poll used by the tagged waits: false once the time limit is spent.
+__device__ __forceinline__ bool poll_again(uint64_t& t0, int* status) {
+  const uint64_t now = globaltimer_ns();
+  if (t0 == 0) t0 = now;
+  if (now - t0 > kWaitLimitNs) {
+    dev_flag(status, PCED_DEV_TIMEOUT);
+    return false;
+  }
+  __nanosleep(32);
+  return true;
+}
+
 // Tile cursor over a CTA's range through all layers (the producer's order).
 struct TileCursor {
   int32_t l, kt;
@@ -537,21 +580,35 @@ __device__ __forceinline__ void cursor_next(TileCursor& c, const StepAttArgs& a,
   cursor_seek(c, a, pre, lens, T, cb, ce, D);
 }
 
-// 1/rms of a residual row from its per-group sums of squares; the same
-// summation order in every warp and CTA, so all users agree bit for bit.
-__device__ __forceinline__ float inv_rms(const float* part, int Hkv, int d, float eps, int lane) {
-  float t = 0.f;
-  for (int i = lane; i < Hkv; i += 32) t += __ldcg(part + i);
-  t = warp_sum(t);
-  t = __shfl_sync(0xffffffffu, t, 0);
-  return 1.0f / sqrtf(t / (float)d + eps);
+// Sum of the Hkv * ATT_CONSUMERS partial sums of squares of x_l[s] (waits
+// for all of them): the same order in every warp and CTA, so every user gets
+// the same 1/rms bit for bit.  Whole warp.
+__device__ __forceinline__ bool wait_inv_rms(const uint64_t* part, int n, uint32_t tag, int d, float eps, int lane,
+                                             int* status, float& inv) {
+  uint64_t t0 = 0;
+  while (true) {
+    float t = 0.f;
+    bool ok = true;
+    for (int i = lane; i < n; i += 32) {
+      const uint64_t w = ld_tagged(part + i);
+      ok &= tv_ok(w, tag);
+      t += tv_value(w);
+    }
+    if (__all_sync(0xffffffffu, ok)) {
+      t = warp_sum(t);
+      t = __shfl_sync(0xffffffffu, t, 0);
+      inv = 1.0f / sqrtf(t / (float)d + eps);
+      return true;
+    }
+    if (!poll_again(t0, status)) return false;
+  }
 }
 
-// x_0[s] = E[y_{t-1}] into residual buffer 0 with its per-group sums of
-// squares, then ready[0] += Hkv.
+// x_0[s] = E[y_{t-1}] (tagged, residual buffer 0) and its partial sums of
+// squares: warp w handles head groups w, w + 8, ... and stores the group's
+// sum in partial slot 0 (slots 1..7 hold 0).
 template <int D>
-__device__ bool embed_sequence(const StepAttArgs& a, const Scratch& sc, int s, uint32_t bar, uint32_t& ph, int ctid,
-                               int warp, int lane) {
+__device__ void embed_sequence(const StepAttArgs& a, int s, uint32_t tag, int ctid, int warp, int lane) {
   const int d = a.Hq * D, GD = a.G * D, b = s / a.n1;
   const int t = *a.step;
   int tok = a.bos;
@@ -562,37 +619,49 @@ __device__ bool embed_sequence(const StepAttArgs& a, const Scratch& sc, int s, u
   }
   if (s == 0 && ctid == 0 && t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
   const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(a.embed + (int64_t)tok * d);
-  float2* x = reinterpret_cast<float2*>(a.resid + (int64_t)s * d);
+  uint64_t* x = a.resid + (int64_t)s * d;
+  uint64_t* ps = a.part_ss + (int64_t)s * a.Hkv * ATT_CONSUMERS;
   for (int h = warp; h < a.Hkv; h += ATT_CONSUMERS) {
     float ss = 0.f;
     for (int i = lane; i < GD / 2; i += 32) {
       const float2 v = __bfloat1622float2(e[h * GD / 2 + i]);
-      x[h * GD / 2 + i] = v;
+      st_tagged(x + h * GD + 2 * i, v.x, tag);
+      st_tagged(x + h * GD + 2 * i + 1, v.y, tag);
       ss += v.x * v.x + v.y * v.y;
     }
     ss = warp_sum(ss);
-    if (lane == 0) a.part_ss[(int64_t)s * a.Hkv + h] = ss;
+    if (lane < ATT_CONSUMERS) st_tagged(ps + h * ATT_CONSUMERS + lane, lane == 0 ? ss : 0.f, tag);
   }
-  if (!warps_sync(bar, ph, a.status)) return false;
-  if (ctid == 0) red_release_gpu_add(&a.ready[0], a.Hkv);
-  return true;
 }
 
 // The row appended this step (u = bf16(x_l * inv), K head h and V head
 // Hkv + h of u viewed as [Hq][D]) into row r of the shared K/V tiles and into
 // the caches.  Called by the one warp that owns the row.
 template <int D>
-__device__ __forceinline__ void patch_row(const StepAttArgs& a, const float* xs, float inv, const Piece& pc,
-                                          int32_t row, int r, int l, uint32_t sk, uint32_t sv, int lane) {
+__device__ __forceinline__ bool patch_row(const StepAttArgs& a, const uint64_t* xs, uint32_t tag, float inv,
+                                          const Piece& pc, int32_t row, int r, int l, uint32_t sk, uint32_t sv,
+                                          int lane) {
   using C = AttCfg<D>;
-  const float* xk = xs + (int64_t)pc.h * D;
-  const float* xv = xs + ((int64_t)a.Hkv + pc.h) * D;
+  const uint64_t* xk = xs + (int64_t)pc.h * D;
+  const uint64_t* xv = xs + ((int64_t)a.Hkv + pc.h) * D;
   const int64_t grow = (int64_t)l * a.layer_elems + a.kv_offset[pc.s] + ((int64_t)pc.h * a.cap[pc.s] + row) * D;
   for (int e = 4 * lane; e < D; e += 128) {
-    const float4 kx = __ldcg(reinterpret_cast<const float4*>(xk + e));
-    const float4 vx = __ldcg(reinterpret_cast<const float4*>(xv + e));
-    const uint2 kb2 = make_uint2(pack_bf16(kx.x * inv, kx.y * inv), pack_bf16(kx.z * inv, kx.w * inv));
-    const uint2 vb2 = make_uint2(pack_bf16(vx.x * inv, vx.y * inv), pack_bf16(vx.z * inv, vx.w * inv));
+    float kx[4], vx[4];
+    uint64_t t0 = 0;
+    while (true) {
+      bool ok = true;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint64_t wk = ld_tagged(xk + e + i), wv = ld_tagged(xv + e + i);
+        ok &= tv_ok(wk, tag) && tv_ok(wv, tag);
+        kx[i] = tv_value(wk);
+        vx[i] = tv_value(wv);
+      }
+      if (ok) break;
+      if (!poll_again(t0, a.status)) return false;
+    }
+    const uint2 kb2 = make_uint2(pack_bf16(kx[0] * inv, kx[1] * inv), pack_bf16(kx[2] * inv, kx[3] * inv));
+    const uint2 vb2 = make_uint2(pack_bf16(vx[0] * inv, vx[1] * inv), pack_bf16(vx[2] * inv, vx[3] * inv));
     const int c = e >> 3;  // 16-byte chunk of the row
     const uint32_t off =
         (c >> 3) * C::BOX_BYTES + r * 128 + ((((uint32_t)c & 7u) ^ ((uint32_t)r & 7u)) << 4) + (e & 7) * 2;
@@ -603,58 +672,46 @@ __device__ __forceinline__ void patch_row(const StepAttArgs& a, const float* xs,
   }
   fence_proxy_async_smem();
   __syncwarp();
+  return true;
 }
 
-// Segment (h, s) of layer l is complete with normalised output o[k] for this
-// thread's outputs: x_{l+1} = x_l + o for head group h, its sum of squares,
-// then signal ready[l+1] (or, at the last layer, the per-sequence counter;
-// the last of the Hkv groups writes the final hidden state of s).
+// Segment (h, s) of layer l is complete, with normalised output o[k] for this
+// thread's outputs: x_{l+1} = x_l + o for head group h and the warp's partial
+// sum of squares, tagged for layer l+1.  After the last layer the CTA also
+// writes its head group of the final hidden state bf16(x_L * inv_rms(x_L)).
 template <int D>
-__device__ bool finish_segment(const StepAttArgs& a, const Scratch& sc, int l, int h, int s,
-                               const float (&xold)[AttCfg<D>::OPT], const float (&o)[AttCfg<D>::OPT], uint32_t bar,
-                               uint32_t& ph, int ctid, int warp, int lane) {
+__device__ bool finish_segment(const StepAttArgs& a, int l, int h, int s, int32_t epoch,
+                               const float (&xold)[AttCfg<D>::OPT], const float (&o)[AttCfg<D>::OPT], int ctid,
+                               int warp, int lane) {
   using C = AttCfg<D>;
   const int S = a.S, Hkv = a.Hkv, GD = a.G * D, d = a.Hq * D, nx = (l + 1) & 1;
-  float* xn = a.resid + ((int64_t)nx * S + s) * d + (int64_t)h * GD;
+  const uint32_t tag = step_tag(epoch, l + 1);
+  uint64_t* xn = a.resid + ((int64_t)nx * S + s) * d + (int64_t)h * GD;
+  uint64_t* ps = a.part_ss + ((int64_t)nx * S + s) * Hkv * ATT_CONSUMERS;
+  float xv[C::OPT];
   float ss = 0.f;
 #pragma unroll
   for (int k = 0; k < C::OPT; ++k) {
     const int idx = ctid + k * ATT_CT;
+    xv[k] = xold[k] + o[k];
     if (idx >= GD) continue;
-    const float x = xold[k] + o[k];
-    xn[idx] = x;
-    ss += x * x;
+    st_tagged(xn + idx, xv[k], tag);
+    ss += xv[k] * xv[k];
   }
   ss = warp_sum(ss);
-  if (lane == 0) sc.red[warp] = ss;
-  if (!warps_sync(bar, ph, a.status)) return false;
-  const bool last_layer = l + 1 == a.L;
-  if (ctid == 0) {
-    float t = 0.f;
+  if (lane == 0) st_tagged(ps + h * ATT_CONSUMERS + warp, ss, tag);
+  if (l + 1 < a.L) return true;
+  float inv;
+  if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, tag, d, a.rms_eps, lane, a.status, inv)) return false;
+  __nv_bfloat16* hs = a.hidden + (int64_t)s * d + (int64_t)h * GD;
+  __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)s * d + (int64_t)h * GD : nullptr;
 #pragma unroll
-    for (int w = 0; w < ATT_CONSUMERS; ++w) t += sc.red[w];
-    a.part_ss[((int64_t)nx * S + s) * Hkv + h] = t;
-    if (!last_layer) {
-      red_release_gpu_add(&a.ready[(int64_t)(l + 1) * ATT_FLAG_STRIDE], 1);
-    } else {
-      const int prev = atom_acq_rel_gpu_add(&a.seq_cnt[s], 1);
-      sc.flag[2] = prev == Hkv - 1;
-      if (prev == Hkv - 1) a.seq_cnt[s] = 0;
-    }
-  }
-  if (!last_layer) return true;
-  if (!warps_sync(bar, ph, a.status)) return false;
-  if (!sc.flag[2]) return true;
-  // final hidden state h[s] = bf16(x_L[s] * inv_rms(x_L[s]))
-  const float inv = inv_rms(a.part_ss + ((int64_t)nx * S + s) * Hkv, Hkv, d, a.rms_eps, lane);
-  const float2* xs = reinterpret_cast<const float2*>(a.resid + ((int64_t)nx * S + s) * d);
-  uint32_t* hs = reinterpret_cast<uint32_t*>(a.hidden + (int64_t)s * d);
-  uint32_t* hc = a.hidden_copy ? reinterpret_cast<uint32_t*>(a.hidden_copy + (int64_t)s * d) : nullptr;
-  for (int i = ctid; i < d / 2; i += ATT_CT) {
-    const float2 x = __ldcg(xs + i);
-    const uint32_t u = pack_bf16(x.x * inv, x.y * inv);
-    hs[i] = u;
-    if (hc) hc[i] = u;
+  for (int k = 0; k < C::OPT; ++k) {
+    const int idx = ctid + k * ATT_CT;
+    if (idx >= GD) continue;
+    const __nv_bfloat16 u = __float2bfloat16_rn(xv[k] * inv);
+    hs[idx] = u;
+    if (hc) hc[idx] = u;
   }
   return true;
 }
@@ -675,6 +732,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int32_t S = a.S, G = a.G, Hkv = a.Hkv, GD = G * D, d = a.Hq * D;
+  const int32_t epoch = *a.epoch;
 
   if (tid == 0) {
     for (int i = 0; i < C::STAGES; ++i) {
@@ -718,7 +776,6 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   const int64_t total = (int64_t)Hkv * T;
   const int64_t P = (total + gridDim.x - 1) / gridDim.x;
   const int64_t cb = min(total, (int64_t)blockIdx.x * P), ce = min(total, cb + P);
-  const int target = S * Hkv;
 
   if (warp == ATT_CONSUMERS) {
     // ------------------------------------------------------------ producer
@@ -779,42 +836,58 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   const int kb = 16 * wl;
   uint32_t it = 0, cph = 0;
   bool ok = true;
-  for (int s = blockIdx.x; s < S && ok; s += gridDim.x) ok = embed_sequence<D>(a, sc, s, bar_c, cph, ctid, warp, lane);
+  for (int s = blockIdx.x; s < S; s += gridDim.x) embed_sequence<D>(a, s, step_tag(epoch, 0), ctid, warp, lane);
 
   for (int l = 0; l < a.L && ok; ++l) {
     const int par = l & 1;
-    bool open = false;
+    const uint32_t tag = step_tag(epoch, l);
     for (int64_t p = cb; p < ce && ok;) {
       const Piece pc = find_piece(pre, lens, S, T, p, ce);
       p += pc.adv;
       if (pc.k0 == pc.k1) continue;
-      if (!open) {
-        // every segment of layer l-1 merged (grid-wide layer dependency)
-        if (ctid == 0) sc.flag[1] = counter_wait(&a.ready[(int64_t)l * ATT_FLAG_STRIDE], target, a.status) ? 1 : 0;
-        if (!warps_sync(bar_c, cph, a.status) || !sc.flag[1]) {
-          ok = false;
-          break;
-        }
-        open = true;
-      }
-      // query bf16(x_l * inv_rms) of head group h, and the stream values of
-      // this thread's outputs (used if this CTA completes the segment)
-      const float* xs = a.resid + ((int64_t)par * S + pc.s) * d;
+      const int64_t pa = (int64_t)pc.h * T + pre[pc.s];
+      const int64_t c0 = pa / P, c1 = (pa + lens[pc.s] - 1) / P;
+      const bool merges = c0 == (int64_t)blockIdx.x;  // the segment's first CTA completes it
+      // wait for this piece's layer input (head group h of x_l[s] and the
+      // partial sums of squares of x_l[s]); form the query bf16(x_l * inv_rms)
+      const uint64_t* xs = a.resid + ((int64_t)par * S + pc.s) * d;
       const bool hv = g < G;
-      const float* xq = xs + ((int64_t)pc.h * G + (hv ? g : 0)) * D;
+      const uint64_t* xq = xs + ((int64_t)pc.h * G + (hv ? g : 0)) * D;
       float2 xl[C::KSTEPS], xh[C::KSTEPS];
-#pragma unroll
-      for (int j = 0; j < C::KSTEPS; ++j) {
-        xl[j] = __ldcg(reinterpret_cast<const float2*>(xq + 16 * j + 2 * tq));
-        xh[j] = __ldcg(reinterpret_cast<const float2*>(xq + 16 * j + 8 + 2 * tq));
-      }
       float xold[C::OPT];
+      {
+        uint64_t t0 = 0;
+        while (true) {
+          bool good = true;
 #pragma unroll
-      for (int k = 0; k < C::OPT; ++k) {
-        const int idx = ctid + k * ATT_CT;
-        xold[k] = idx < GD ? __ldcg(xs + (int64_t)pc.h * GD + idx) : 0.f;
+          for (int j = 0; j < C::KSTEPS; ++j) {
+            const uint64_t w0 = ld_tagged(xq + 16 * j + 2 * tq), w1 = ld_tagged(xq + 16 * j + 2 * tq + 1);
+            const uint64_t w2 = ld_tagged(xq + 16 * j + 8 + 2 * tq), w3 = ld_tagged(xq + 16 * j + 9 + 2 * tq);
+            good &= tv_ok(w0, tag) && tv_ok(w1, tag) && tv_ok(w2, tag) && tv_ok(w3, tag);
+            xl[j] = make_float2(tv_value(w0), tv_value(w1));
+            xh[j] = make_float2(tv_value(w2), tv_value(w3));
+          }
+#pragma unroll
+          for (int k = 0; k < C::OPT; ++k) {
+            const int idx = ctid + k * ATT_CT;
+            xold[k] = 0.f;
+            if (!merges || idx >= GD) continue;
+            const uint64_t w = ld_tagged(xs + (int64_t)pc.h * GD + idx);
+            good &= tv_ok(w, tag);
+            xold[k] = tv_value(w);
+          }
+          if (__all_sync(0xffffffffu, good)) break;
+          if (!poll_again(t0, a.status)) {
+            ok = false;
+            break;
+          }
+        }
       }
-      const float inv = inv_rms(a.part_ss + ((int64_t)par * S + pc.s) * Hkv, Hkv, d, a.rms_eps, lane);
+      float inv = 0.f;
+      if (ok && !wait_inv_rms(a.part_ss + ((int64_t)par * S + pc.s) * Hkv * ATT_CONSUMERS, Hkv * ATT_CONSUMERS, tag,
+                              d, a.rms_eps, lane, a.status, inv))
+        ok = false;
+      if (!ok) break;
       uint32_t qf[C::KSTEPS][2];
 #pragma unroll
       for (int j = 0; j < C::KSTEPS; ++j) {
@@ -838,8 +911,11 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         }
         const int nvalid = min(ATT_BLOCK_N, pc.k1 - kt);
         const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
-        if (app_row >= kt && app_row < kt + ATT_BLOCK_N && ((app_row - kt) >> 4) == wl)
-          patch_row<D>(a, xs, inv, pc, app_row, app_row - kt, l, sk, sv, lane);
+        if (app_row >= kt && app_row < kt + ATT_BLOCK_N && ((app_row - kt) >> 4) == wl &&
+            !patch_row<D>(a, xs, tag, inv, pc, app_row, app_row - kt, l, sk, sv, lane)) {
+          ok = false;
+          break;
+        }
         if (kb < nvalid) tile_math<D>(A, qf, sk, sv, kb, nvalid, a.scale_log2, lane);
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_empty + 8 * st);
@@ -852,88 +928,88 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         break;
       }
       const int64_t seg = (int64_t)pc.h * S + pc.s;
-      const int64_t pa = (int64_t)pc.h * T + pre[pc.s];
-      const int64_t c0 = pa / P, c1 = (pa + lens[pc.s] - 1) / P;
-      if (c0 == c1) {
-        // the whole segment lies in this CTA
+      if (!merges) {
+        // publish this CTA's record of the segment for its first CTA
+        const int64_t slot = (int64_t)blockIdx.x + seg;
 #pragma unroll
-        for (int k = 0; k < C::OPT; ++k) o[k] = ls[k] > 0.f ? acc[k] / ls[k] : 0.f;
-        if (!finish_segment<D>(a, sc, l, pc.h, pc.s, xold, o, bar_c, cph, ctid, warp, lane)) {
-          ok = false;
-          break;
+        for (int k = 0; k < C::OPT; ++k) {
+          const int idx = ctid + k * ATT_CT;
+          if (idx >= GD) continue;
+          st_tagged(a.rec_o + slot * GD + idx, acc[k], tag);
+          if (idx % D == 0) {
+            st_tagged(a.rec_ml + (slot * G + idx / D) * 2, mx[k], tag);
+            st_tagged(a.rec_ml + (slot * G + idx / D) * 2 + 1, ls[k], tag);
+          }
         }
         continue;
       }
-      // publish this CTA's record; the last of the segment's CTAs merges
-      const int64_t slot = (int64_t)blockIdx.x + seg;
-#pragma unroll
-      for (int k = 0; k < C::OPT; ++k) {
-        const int idx = ctid + k * ATT_CT;
-        if (idx >= GD) continue;
-        a.rec_o[slot * GD + idx] = acc[k];
-        if (idx % D == 0) a.rec_ml[slot * G + idx / D] = make_float2(mx[k], ls[k]);
-      }
-      if (!warps_sync(bar_c, cph, a.status)) {
-        ok = false;
-        break;
-      }
-      if (ctid == 0) {
-        int* cnt = &a.seg_cnt[seg];
-        const int prev = atom_acq_rel_gpu_add(cnt, 1);
-        sc.flag[0] = prev == (int)(c1 - c0);
-        if (prev == (int)(c1 - c0)) *cnt = 0;
-      }
-      if (!warps_sync(bar_c, cph, a.status)) {
-        ok = false;
-        break;
-      }
-      if (!sc.flag[0]) continue;
-      // merge records c0..c1 in order (deterministic whichever CTA merges)
+      // complete the segment: this CTA's part, then the records of CTAs
+      // c0+1..c1 in order (deterministic)
 #pragma unroll
       for (int k = 0; k < C::OPT; ++k) {
         const int idx = ctid + k * ATT_CT;
         o[k] = 0.f;
         if (idx >= GD) continue;
         const int hh = idx / D;
-        float M = -INFINITY, Ls = 0.f, Ac = 0.f;
-        for (int64_t c = c0; c <= c1; c += 4) {
-          float2 ml[4];
-          float ov[4];
+        float M = mx[k], Ls = ls[k], Ac = acc[k];
+        for (int64_t c = c0 + 1; c <= c1 && ok; c += 4) {
+          float mv[4], lv[4], ov[4];
+          uint64_t t0 = 0;
+          while (true) {
+            bool good = true;
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const bool in = c + u <= c1;
-            ml[u] = in ? __ldcg(a.rec_ml + (c + u + seg) * G + hh) : make_float2(-INFINITY, 0.f);
-            ov[u] = in ? __ldcg(a.rec_o + (c + u + seg) * GD + idx) : 0.f;
+            for (int u = 0; u < 4; ++u) {
+              mv[u] = -INFINITY;
+              lv[u] = 0.f;
+              ov[u] = 0.f;
+              if (c + u > c1) continue;
+              const int64_t sl = c + u + seg;
+              const uint64_t wm = ld_tagged(a.rec_ml + (sl * G + hh) * 2);
+              const uint64_t wl2 = ld_tagged(a.rec_ml + (sl * G + hh) * 2 + 1);
+              const uint64_t wo = ld_tagged(a.rec_o + sl * GD + idx);
+              good &= tv_ok(wm, tag) && tv_ok(wl2, tag) && tv_ok(wo, tag);
+              mv[u] = tv_value(wm);
+              lv[u] = tv_value(wl2);
+              ov[u] = tv_value(wo);
+            }
+            if (good) break;
+            if (!poll_again(t0, a.status)) {
+              ok = false;
+              break;
+            }
           }
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            if (ml[u].x == -INFINITY) continue;
-            const float Mn = fmaxf(M, ml[u].x);
-            const float f = M == -INFINITY ? 0.f : exp2f(M - Mn), e = exp2f(ml[u].x - Mn);
+            if (mv[u] == -INFINITY) continue;
+            const float Mn = fmaxf(M, mv[u]);
+            const float f = M == -INFINITY ? 0.f : exp2f(M - Mn), e = exp2f(mv[u] - Mn);
             Ac = Ac * f + ov[u] * e;
-            Ls = Ls * f + ml[u].y * e;
+            Ls = Ls * f + lv[u] * e;
             M = Mn;
           }
         }
         o[k] = Ls > 0.f ? Ac / Ls : 0.f;
       }
-      if (!finish_segment<D>(a, sc, l, pc.h, pc.s, xold, o, bar_c, cph, ctid, warp, lane)) {
+      if (!ok) break;
+      if (!finish_segment<D>(a, l, pc.h, pc.s, epoch, xold, o, ctid, warp, lane)) {
         ok = false;
         break;
       }
     }
   }
 
-  // ---- the last CTA to finish zeroes the layer counters and advances seq_len
+  // ---- the last CTA to finish advances seq_len and the epoch
   if (ctid == 0) {
     const int prev = atom_acq_rel_gpu_add(a.done_cnt, 1);
     sc.flag[3] = prev == (int)gridDim.x - 1;
   }
   if (warps_sync(bar_c, cph, a.status) && sc.flag[3]) {
-    for (int l = ctid; l < a.L; l += ATT_CT) a.ready[(int64_t)l * ATT_FLAG_STRIDE] = 0;
     for (int i = ctid; i < S; i += ATT_CT)
       if (sc.apnd[i]) a.seq_len[i] = lens[i];
-    if (ctid == 0) *a.done_cnt = 0;
+    if (ctid == 0) {
+      *a.done_cnt = 0;
+      *a.epoch = epoch + 1;
+    }
   }
 }
 

@@ -13,7 +13,7 @@ constexpr int ATT_CT = ATT_CONSUMERS * 32;  // consumer threads
 constexpr int ATT_MAX_S = 1024;     // sequences per launch (prefix table lives in shared memory)
 constexpr int ATT_MAX_G = 8;        // query heads per kv-head (mma N = 8)
 constexpr int ATT_MAX_CTAS = 1024;  // upper bound of the grid (sizes the partial-record pool)
-constexpr int ATT_FLAG_STRIDE = 32; // ints between layer counters: each owns a 128-byte line
+constexpr float ATT_RESCALE_SLACK = 8.f;  // log2 units the online-softmax reference may trail the max
 
 // ---------------------------------------------------------------- one layer
 // Partition of all (kv-head, sequence, key) positions into equal contiguous
@@ -69,18 +69,18 @@ cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream);
 // layers (a shared-memory ring plus L2 prefetch ahead of it) while the
 // consumers wait for the layer dependency.
 //
-// Layer dependency: the CTA that completes segment (h, s) at layer l (last
-// of its record writers, or the only one) merges the records, adds the head
-// group's attention output to the residual stream, x_{l+1} = x_l + o (double
-// buffered by layer parity), stores the group's sum of squares and adds one
-// to the layer counter ready[l+1]; the embedding adds Hkv per sequence to
-// ready[0].  A CTA starts the compute of layer l once ready[l] = S*Hkv (all
-// of layer l-1 merged).  Every piece forms its query bf16(x_l * inv_rms(x_l))
-// itself; the warp that owns the row appended this step writes that row's
-// K/V (the same normalised stream) into the shared tile and the cache.  At the
-// last layer a per-sequence counter picks the CTA that writes the final
-// hidden state.  The last CTA to finish zeroes the counters and advances
-// seq_len.
+// Layer dependency: a segment split over CTAs c0..c1 is completed by c0 (for
+// which it is the last piece of the layer); c0+1..c1 publish their records
+// for it.  The completing CTA adds the head group's attention output to the
+// residual stream, x_{l+1} = x_l + o (double buffered by layer parity), and
+// stores per-warp partial sums of squares.  A piece of layer l waits for its
+// head group of x_l[s] and all partial sums of x_l[s], forms its query
+// bf16(x_l * inv_rms(x_l)) itself, and the warp that owns the row appended
+// this step writes that row's K/V (the same normalised stream) into the
+// shared tile and the cache.  Everything exchanged between CTAs is a tagged
+// 64-bit word (see attention.cu).  After the last layer each completing CTA
+// writes its head group of the final hidden state; the last CTA to finish
+// advances seq_len and the epoch.
 struct StepAttArgs {
   int32_t S, Hq, Hkv, G, L, n1, V, bos, max_steps;
   int64_t rows_per_layer;     // rows (of D elements) of one layer's region in the tensor maps
@@ -96,18 +96,17 @@ struct StepAttArgs {
   const __nv_bfloat16* embed; // [V][d]
   __nv_bfloat16* k_cache;
   __nv_bfloat16* v_cache;
-  float* resid;               // [2][S][d]
-  float* part_ss;             // [2][S][Hkv]
-  float* rec_o;               // [slots][G][D]
-  float2* rec_ml;             // [slots][G]
-  int32_t* seg_cnt;           // [Hkv*S] arrival counters (zero between launches)
-  int32_t* seq_cnt;           // [S] last-layer arrival counters (zero between launches)
-  int32_t* ready;             // [L * ATT_FLAG_STRIDE] layer counters (zero between launches)
-  int32_t* done_cnt;          // [1] (zero between launches)
+  uint64_t* resid;            // [2][S][d] tagged residual stream x_l (buffer l % 2)
+  uint64_t* part_ss;          // [2][S][Hkv][8] tagged per-warp sums of squares of x_l
+  uint64_t* rec_o;            // [slots][G*D] tagged partial outputs
+  uint64_t* rec_ml;           // [slots][G][2] tagged (max, sum)
+  int32_t* epoch;             // [1] launches completed (tags name the launch)
+  int32_t* done_cnt;          // [1] CTAs finished (zero between launches)
   __nv_bfloat16* hidden;      // [S][d] final hidden state
   __nv_bfloat16* hidden_copy; // optional copy of `hidden`
   int* status;
 };
+constexpr int ATT_MAX_LAYERS = 1000;  // layer index fits the 10-bit field of the tags
 int64_t att_step_slots(int32_t S, int32_t Hkv);
 // tuning of the partition and the prefetch distance (PCED_ATT_SEGCOST /
 // PCED_ATT_PF in the environment override the defaults)

@@ -9,7 +9,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include "../../include/pced.h"
+#include "pced.h"
 
 namespace pced {
 

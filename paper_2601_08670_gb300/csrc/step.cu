@@ -20,14 +20,12 @@ struct StepLayout {
   int* status;
   int32_t* done_counter;  // selection kernel: queries finished this step
   int32_t* att_done;      // attention: CTAs finished
-  int32_t* seg_cnt;
-  int32_t* seq_cnt;
-  int32_t* ready;
-  float* part_ss;
-  float* resid;
+  int32_t* att_epoch;     // attention: launches completed
+  uint64_t* part_ss;
+  uint64_t* resid;
+  uint64_t* rec_o;
+  uint64_t* rec_ml;
   __nv_bfloat16* h;
-  float* rec_o;
-  float2* rec_ml;
   float2* lm_stats;
   float2* lm_arg;
   size_t bytes;
@@ -42,14 +40,12 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   L.status = c.take<int>(64);
   L.done_counter = c.take<int32_t>(1);
   L.att_done = c.take<int32_t>(1);
-  L.seg_cnt = c.take<int32_t>((size_t)S * dm->Hkv);
-  L.seq_cnt = c.take<int32_t>((size_t)S);
-  L.ready = c.take<int32_t>((size_t)(dm->L > 0 ? dm->L : 1) * ATT_FLAG_STRIDE);
-  L.part_ss = c.take<float>((size_t)2 * S * dm->Hkv);
-  L.resid = c.take<float>((size_t)2 * S * d);
+  L.att_epoch = c.take<int32_t>(1);
+  L.part_ss = c.take<uint64_t>((size_t)2 * S * dm->Hkv * ATT_CONSUMERS);
+  L.resid = c.take<uint64_t>((size_t)2 * S * d);
+  L.rec_o = c.take<uint64_t>((size_t)(slots * G * dm->D));
+  L.rec_ml = c.take<uint64_t>((size_t)(slots * G * 2));
   L.h = c.take<__nv_bfloat16>((size_t)S * d);
-  L.rec_o = c.take<float>((size_t)(slots * G * dm->D));
-  L.rec_ml = c.take<float2>((size_t)(slots * G));
   L.lm_stats = c.take<float2>((size_t)(S * ntiles));
   L.lm_arg = c.take<float2>((size_t)(S * ntiles));
   L.bytes = c.used();
@@ -82,7 +78,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
       !p->step || !p->history || !p->beta || !p->r || !p->workspace)
     return fail(PCED_ERR_INVALID_ARG, "pced_step: null pointer");
   if (dm.B < 1 || dm.N < 1 || dm.L < 1 || dm.Hq < 1 || dm.Hkv < 1 || dm.D < 1 || dm.V < 1 || dm.Hq % dm.Hkv != 0 ||
-      2 * dm.Hkv > dm.Hq || p->max_steps < 1 || p->layer_elems < dm.D || p->total_cap < 1)
+      2 * dm.Hkv > dm.Hq || dm.L > ATT_MAX_LAYERS || p->max_steps < 1 || p->layer_elems < dm.D || p->total_cap < 1)
     return fail(PCED_ERR_INVALID_ARG, "pced_step: bad dimensions");
   if (!isfinite(p->gamma) || !(p->attn_scale > 0.f) || !(p->rms_eps >= 0.f))
     return fail(PCED_ERR_INVALID_ARG, "pced_step: bad gamma / scale / eps");
@@ -155,9 +151,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   at.part_ss = W.part_ss;
   at.rec_o = W.rec_o;
   at.rec_ml = W.rec_ml;
-  at.seg_cnt = W.seg_cnt;
-  at.seq_cnt = W.seq_cnt;
-  at.ready = W.ready;
+  at.epoch = W.att_epoch;
   at.done_cnt = W.att_done;
   at.hidden = W.h;
   at.hidden_copy = (__nv_bfloat16*)p->hidden_out;
