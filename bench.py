@@ -160,14 +160,30 @@ KERNEL_SOURCES = {
 
 def ncu_traffic(kind: str, workload: str):
     """DRAM bytes per launch of `kind` from the committed ncu summary, or None
-    when missing or taken on a different version of the kernel source."""
+    when missing or taken on a different version of the kernel source.  A
+    capture of the same shapes with fewer layers is scaled by the layer count
+    (the attention launch streams every layer once)."""
+    import synth
     try:
         rec = json.load(open(os.path.join(ROOT, "profiles", "ncu_traffic.json")))[kind]
     except (OSError, ValueError, KeyError):
         return None
-    if rec.get("source_hash") != source_hash(KERNEL_SOURCES[kind]) or rec.get("workload") != workload:
+    if rec.get("source_hash") != source_hash(KERNEL_SOURCES[kind]):
         return None
-    return rec.get("dram_bytes_per_launch")
+    got = rec.get("dram_bytes_per_launch")
+    if rec.get("workload") == workload or got is None:
+        return got
+    wc, w = synth.get(rec["workload"]), synth.get(workload)
+    if kind == "attention" and replace_layers(wc, w.L) == replace_layers(w, w.L):
+        return got * w.L / wc.L
+    if kind == "lm_head" and (wc.S, wc.d, wc.V) == (w.S, w.d, w.V):
+        return got
+    return None
+
+
+def replace_layers(w, L):
+    from dataclasses import replace
+    return replace(w, L=L, name=None, steps=None, description=None) if w else w
 
 
 def step_bytes(w, lens_after) -> int:

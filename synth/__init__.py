@@ -87,6 +87,10 @@ WORKLOADS = {
         "llama8", B=1, N=8, L=32, Hq=32, Hkv=8, D=128, V=128256, steps=64,
         doc_len=("fixed", 2048),
         description="Llama-3-8B shapes, N=8 doc experts + amateur, doc KV 2048+32, vocab 128256, 64 steps"),
+    "llama8_l4": Workload(
+        "llama8_l4", B=1, N=8, L=4, Hq=32, Hkv=8, D=128, V=128256, steps=16,
+        doc_len=("fixed", 2048),
+        description="llama8 with 4 layers: the same per-layer work, small enough for multi-pass profiling"),
     "llama32": Workload(
         "llama32", B=1, N=32, L=32, Hq=32, Hkv=8, D=128, V=128256, steps=64,
         doc_len=("uniform", 512, 8192), r_recipe=("softmax_normal", 2.0),
