@@ -580,9 +580,9 @@ __device__ __forceinline__ void cursor_next(TileCursor& c, const StepAttArgs& a,
   cursor_seek(c, a, pre, lens, T, cb, ce, D);
 }
 
-// Sum of the Hkv * ATT_CONSUMERS partial sums of squares of x_l[s] (waits
-// for all of them): the same order in every warp and CTA, so every user gets
-// the same 1/rms bit for bit.  Whole warp.
+// 1/rms of x_l[s] from its Hkv per-group sums of squares (waits for all of
+// them): the same order in every warp and CTA, so every user gets the same
+// value bit for bit.  Whole warp.
 __device__ __forceinline__ bool wait_inv_rms(const uint64_t* part, int n, uint32_t tag, int d, float eps, int lane,
                                              int* status, float& inv) {
   uint64_t t0 = 0;
@@ -604,24 +604,55 @@ __device__ __forceinline__ bool wait_inv_rms(const uint64_t* part, int n, uint32
   }
 }
 
-// x_0[s] = E[y_{t-1}] (tagged, residual buffer 0) and its partial sums of
-// squares: warp w handles head groups w, w + 8, ... and stores the group's
-// sum in partial slot 0 (slots 1..7 hold 0).
+// Shared-memory layout of the step kernel (byte offsets from the 1024-byte
+// aligned base), a function of the head dim and group size only.
+struct StepSmem {
+  uint32_t stages;      // K/V ring stages
+  uint32_t bar;         // full[st] empty[st] qfull[2] qempty[2] pfull[2] pempty[2] msync
+  uint32_t qbuf, qslot; // [2] hand-off slots: q words [8][D/2+4], K row, V row (bf16), x_l of the head group (fp32)
+  uint32_t pbuf, pslot; // [2] partial hand-off slots: ms[8][8], ls[8][8], os[8][D][opad]
+  uint32_t opad;
+  uint32_t misc;        // red[2][2] floats, flags
+  uint32_t tables;      // pre[ATT_MAX_S+1] int64, lens[ATT_MAX_S] int32, apnd[ATT_MAX_S] u8
+  uint32_t total;       // bytes to request, alignment slack included
+};
+__host__ __device__ inline StepSmem step_smem(int D, int G) {
+  StepSmem L;
+  const uint32_t stage_bytes = 2u * (uint32_t)(D / 64) * (ATT_BLOCK_N * 128u);
+  L.opad = (G % 2 == 0) ? (uint32_t)G + 1u : (uint32_t)G;
+  L.qslot = 8u * (uint32_t)(D / 2 + 4) * 4u + 4u * (uint32_t)D + 4u * (uint32_t)(G * D);
+  L.pslot = 2u * ATT_CONSUMERS * ATT_MAX_G * 4u + (uint32_t)ATT_CONSUMERS * D * L.opad * 4u;
+  const uint32_t tables = (ATT_MAX_S + 1) * 8u + ATT_MAX_S * 4u + ATT_MAX_S;
+  const uint32_t max_st = D == 128 ? 5u : 7u;
+  for (L.stages = max_st; L.stages >= 2u; --L.stages) {
+    L.bar = L.stages * stage_bytes;
+    L.qbuf = L.bar + (2u * L.stages + 9u) * 8u;
+    L.qbuf = (L.qbuf + 15u) & ~15u;
+    L.pbuf = L.qbuf + 2u * L.qslot;
+    L.misc = L.pbuf + 2u * L.pslot;
+    L.tables = L.misc + 64u;
+    L.total = 1024u + L.tables + tables;
+    if (L.total <= 227u * 1024u) break;
+  }
+  return L;
+}
+
+// x_0[s] = E[y_{t-1}] (tagged, residual buffer 0) and its per-group sums of
+// squares (in partial slot 0 of each group; slots 1..7 hold 0).  One warp.
 template <int D>
-__device__ void embed_sequence(const StepAttArgs& a, int s, uint32_t tag, int ctid, int warp, int lane) {
+__device__ void embed_sequence(const StepAttArgs& a, int s, uint32_t tag, int lane) {
   const int d = a.Hq * D, GD = a.G * D, b = s / a.n1;
   const int t = *a.step;
   int tok = a.bos;
   if (t > 0 && t <= a.max_steps) tok = a.history[(int64_t)b * a.max_steps + t - 1];
   if (tok < 0 || tok >= a.V) {
-    if (ctid == 0) dev_flag(a.status, PCED_DEV_BAD_TOKEN);
+    if (lane == 0) dev_flag(a.status, PCED_DEV_BAD_TOKEN);
     tok = 0;
   }
-  if (s == 0 && ctid == 0 && t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
+  if (s == 0 && lane == 0 && t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
   const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(a.embed + (int64_t)tok * d);
   uint64_t* x = a.resid + (int64_t)s * d;
-  uint64_t* ps = a.part_ss + (int64_t)s * a.Hkv * ATT_CONSUMERS;
-  for (int h = warp; h < a.Hkv; h += ATT_CONSUMERS) {
+  for (int h = 0; h < a.Hkv; ++h) {
     float ss = 0.f;
     for (int i = lane; i < GD / 2; i += 32) {
       const float2 v = __bfloat1622float2(e[h * GD / 2 + i]);
@@ -630,119 +661,54 @@ __device__ void embed_sequence(const StepAttArgs& a, int s, uint32_t tag, int ct
       ss += v.x * v.x + v.y * v.y;
     }
     ss = warp_sum(ss);
-    if (lane < ATT_CONSUMERS) st_tagged(ps + h * ATT_CONSUMERS + lane, lane == 0 ? ss : 0.f, tag);
+    if (lane < ATT_CONSUMERS) st_tagged(a.part_ss + ((int64_t)s * a.Hkv + h) * ATT_CONSUMERS + lane, lane == 0 ? ss : 0.f, tag);
   }
 }
 
-// The row appended this step (u = bf16(x_l * inv), K head h and V head
-// Hkv + h of u viewed as [Hq][D]) into row r of the shared K/V tiles and into
-// the caches.  Called by the one warp that owns the row.
-template <int D>
-__device__ __forceinline__ bool patch_row(const StepAttArgs& a, const uint64_t* xs, uint32_t tag, float inv,
-                                          const Piece& pc, int32_t row, int r, int l, uint32_t sk, uint32_t sv,
-                                          int lane) {
-  using C = AttCfg<D>;
-  const uint64_t* xk = xs + (int64_t)pc.h * D;
-  const uint64_t* xv = xs + ((int64_t)a.Hkv + pc.h) * D;
-  const int64_t grow = (int64_t)l * a.layer_elems + a.kv_offset[pc.s] + ((int64_t)pc.h * a.cap[pc.s] + row) * D;
-  for (int e = 4 * lane; e < D; e += 128) {
-    float kx[4], vx[4];
-    uint64_t t0 = 0;
-    while (true) {
-      bool ok = true;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint64_t wk = ld_tagged(xk + e + i), wv = ld_tagged(xv + e + i);
-        ok &= tv_ok(wk, tag) && tv_ok(wv, tag);
-        kx[i] = tv_value(wk);
-        vx[i] = tv_value(wv);
-      }
-      if (ok) break;
-      if (!poll_again(t0, a.status)) return false;
-    }
-    const uint2 kb2 = make_uint2(pack_bf16(kx[0] * inv, kx[1] * inv), pack_bf16(kx[2] * inv, kx[3] * inv));
-    const uint2 vb2 = make_uint2(pack_bf16(vx[0] * inv, vx[1] * inv), pack_bf16(vx[2] * inv, vx[3] * inv));
-    const int c = e >> 3;  // 16-byte chunk of the row
-    const uint32_t off =
-        (c >> 3) * C::BOX_BYTES + r * 128 + ((((uint32_t)c & 7u) ^ ((uint32_t)r & 7u)) << 4) + (e & 7) * 2;
-    asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(sk + off), "r"(kb2.x), "r"(kb2.y) : "memory");
-    asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(sv + off), "r"(vb2.x), "r"(vb2.y) : "memory");
-    *reinterpret_cast<uint2*>(a.k_cache + grow + e) = kb2;
-    *reinterpret_cast<uint2*>(a.v_cache + grow + e) = vb2;
-  }
-  fence_proxy_async_smem();
-  __syncwarp();
-  return true;
-}
-
-// Segment (h, s) of layer l is complete, with normalised output o[k] for this
-// thread's outputs: x_{l+1} = x_l + o for head group h and the warp's partial
-// sum of squares, tagged for layer l+1.  After the last layer the CTA also
-// writes its head group of the final hidden state bf16(x_L * inv_rms(x_L)).
-template <int D>
-__device__ bool finish_segment(const StepAttArgs& a, int l, int h, int s, int32_t epoch,
-                               const float (&xold)[AttCfg<D>::OPT], const float (&o)[AttCfg<D>::OPT], int ctid,
-                               int warp, int lane) {
-  using C = AttCfg<D>;
-  const int S = a.S, Hkv = a.Hkv, GD = a.G * D, d = a.Hq * D, nx = (l + 1) & 1;
-  const uint32_t tag = step_tag(epoch, l + 1);
-  uint64_t* xn = a.resid + ((int64_t)nx * S + s) * d + (int64_t)h * GD;
-  uint64_t* ps = a.part_ss + ((int64_t)nx * S + s) * Hkv * ATT_CONSUMERS;
-  float xv[C::OPT];
-  float ss = 0.f;
-#pragma unroll
-  for (int k = 0; k < C::OPT; ++k) {
-    const int idx = ctid + k * ATT_CT;
-    xv[k] = xold[k] + o[k];
-    if (idx >= GD) continue;
-    st_tagged(xn + idx, xv[k], tag);
-    ss += xv[k] * xv[k];
-  }
-  ss = warp_sum(ss);
-  if (lane == 0) st_tagged(ps + h * ATT_CONSUMERS + warp, ss, tag);
-  if (l + 1 < a.L) return true;
-  float inv;
-  if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, tag, d, a.rms_eps, lane, a.status, inv)) return false;
-  __nv_bfloat16* hs = a.hidden + (int64_t)s * d + (int64_t)h * GD;
-  __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)s * d + (int64_t)h * GD : nullptr;
-#pragma unroll
-  for (int k = 0; k < C::OPT; ++k) {
-    const int idx = ctid + k * ATT_CT;
-    if (idx >= GD) continue;
-    const __nv_bfloat16 u = __float2bfloat16_rn(xv[k] * inv);
-    hs[idx] = u;
-    if (hc) hc[idx] = u;
-  }
-  return true;
-}
+constexpr int STEP_PRODUCER = ATT_CONSUMERS;      // warp 8: TMA
+constexpr int STEP_INPUT = ATT_CONSUMERS + 1;     // warp 9: queries, appended rows, x_l hand-off
+constexpr int STEP_THREADS = (ATT_CONSUMERS + 2) * 32;
 
 template <int D>
-__global__ void __launch_bounds__(ATT_THREADS, 1)
+__global__ void __launch_bounds__(STEP_THREADS, 1)
     att_step_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                     StepAttArgs a) {
   using C = AttCfg<D>;
+  constexpr int QW = D / 2 + 4;  // padded words per query row in the hand-off slot
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
-  const uint32_t bar_full = base + C::STAGES * C::STAGE_BYTES;
-  const uint32_t bar_empty = bar_full + C::STAGES * 8;
-  const uint32_t bar_c = bar_empty + C::STAGES * 8;
-  const Scratch sc = carve_scratch<D>(gbase + C::STAGES * C::STAGE_BYTES + C::BARS);
+  const int32_t S = a.S, G = a.G, Hkv = a.Hkv, GD = G * D, d = a.Hq * D;
+  const StepSmem SL = step_smem(D, G);
+  const uint32_t NST = SL.stages;
+  const uint32_t bar_full = base + SL.bar, bar_empty = bar_full + 8 * NST;
+  const uint32_t bar_qfull = bar_empty + 8 * NST, bar_qempty = bar_qfull + 16;
+  const uint32_t bar_pfull = bar_qempty + 16, bar_pempty = bar_pfull + 16, bar_m = bar_pempty + 16;
+  float* red = reinterpret_cast<float*>(gbase + SL.misc);  // [2 slots][2 merge warps]
+  int* flag = reinterpret_cast<int*>(gbase + SL.misc + 32);
+  int64_t* pre = reinterpret_cast<int64_t*>(gbase + SL.tables);
+  int32_t* lens = reinterpret_cast<int32_t*>(pre + ATT_MAX_S + 1);
+  uint8_t* apnd = reinterpret_cast<uint8_t*>(lens + ATT_MAX_S);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int32_t S = a.S, G = a.G, Hkv = a.Hkv, GD = G * D, d = a.Hq * D;
   const int32_t epoch = *a.epoch;
 
   if (tid == 0) {
-    for (int i = 0; i < C::STAGES; ++i) {
+    for (uint32_t i = 0; i < NST; ++i) {
       mbar_init(bar_full + 8 * i, 1);
       mbar_init(bar_empty + 8 * i, 4);
     }
-    mbar_init(bar_c, ATT_CONSUMERS);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar_qfull + 8 * i, 1);
+      mbar_init(bar_qempty + 8 * i, ATT_CONSUMERS);
+      mbar_init(bar_pfull + 8 * i, ATT_CONSUMERS);
+      mbar_init(bar_pempty + 8 * i, ATT_CONSUMERS);
+    }
+    mbar_init(bar_m, ATT_CONSUMERS);
     mbar_fence_init();
   }
-  if (warp == ATT_CONSUMERS && lane == 0) {
+  if (warp == STEP_PRODUCER && lane == 0) {
     tma_prefetch_desc(&kmap);
     tma_prefetch_desc(&vmap);
   }
@@ -750,7 +716,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   // this grid's completion before reading the hidden states
   pdl_launch_dependents();
   // lengths after this step's append (a full cache appends nothing)
-  for (int i = tid; i < S; i += ATT_THREADS) {
+  for (int i = tid; i < S; i += STEP_THREADS) {
     int32_t n = a.seq_len[i];
     const int32_t c = a.cap[i];
     if (n < 0 || n > c) {
@@ -764,20 +730,18 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       dev_flag(a.status, PCED_DEV_BAD_LENGTH);
       len = 1;
     }
-    sc.lens[i] = len;
-    sc.apnd[i] = ap ? 1 : 0;
+    lens[i] = len;
+    apnd[i] = ap ? 1 : 0;
   }
   __syncthreads();
-  if (warp == 0) prefix_extents(sc.lens, S, a.seg_cost, sc.pre, lane);
+  if (warp == 0) prefix_extents(lens, S, a.seg_cost, pre, lane);
   __syncthreads();
-  const int64_t* pre = sc.pre;
-  const int32_t* lens = sc.lens;
   const int64_t T = pre[S];
   const int64_t total = (int64_t)Hkv * T;
   const int64_t P = (total + gridDim.x - 1) / gridDim.x;
   const int64_t cb = min(total, (int64_t)blockIdx.x * P), ce = min(total, cb + P);
 
-  if (warp == ATT_CONSUMERS) {
+  if (warp == STEP_PRODUCER) {
     // ------------------------------------------------------------ producer
     // K/V tiles of every layer in consumption order; the L2 prefetch cursor
     // runs pf_tiles ahead so HBM keeps streaming while the ring is full
@@ -797,7 +761,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       while (ld.ok) {
-        const uint32_t st = it % C::STAGES, ph = (it / C::STAGES) & 1u;
+        const uint32_t st = it % NST, ph = (it / NST) & 1u;
         if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
           ok = false;
           break;
@@ -823,84 +787,172 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         }
       }
       if (!ok) {
-        for (uint32_t j = (it >= C::STAGES ? it - C::STAGES : 0); j < it; ++j)
-          mbar_wait(bar_full + 8 * (j % C::STAGES), (j / C::STAGES) & 1u, a.status);
+        for (uint32_t j = (it >= NST ? it - NST : 0); j < it; ++j)
+          mbar_wait(bar_full + 8 * (j % NST), (j / NST) & 1u, a.status);
+      }
+    }
+    return;
+  }
+
+  if (warp == STEP_INPUT) {
+    // ---------------------------------------------------------- input warp
+    // For every piece, in order: wait for head group h of x_l[s] and the
+    // group sums of x_l[s], then hand the consumers q = bf16(x_l * inv_rms)
+    // (and, for the piece holding the row appended this step, that row's K
+    // and V, also written to the caches) through a double-buffered slot.
+    for (int s = blockIdx.x; s < S; s += gridDim.x) embed_sequence<D>(a, s, step_tag(epoch, 0), lane);
+    uint32_t p = 0;
+    bool ok = true;
+    for (int l = 0; l < a.L && ok; ++l) {
+      const int par = l & 1;
+      const uint32_t tag = step_tag(epoch, l);
+      for (int64_t pp = cb; pp < ce && ok;) {
+        const Piece pc = find_piece(pre, lens, S, T, pp, ce);
+        pp += pc.adv;
+        if (pc.k0 == pc.k1) continue;
+        const uint32_t slot = p & 1u, u = p >> 1;
+        ++p;
+        if (u > 0 && !mbar_wait(bar_qempty + 8 * slot, (u - 1u) & 1u, a.status)) {
+          ok = false;
+          break;
+        }
+        const uint64_t* xs = a.resid + ((int64_t)par * S + pc.s) * d;
+        const uint64_t* xq = xs + (int64_t)pc.h * GD;
+        const bool app = apnd[pc.s] && pc.k1 == lens[pc.s];
+        const uint64_t* ps = a.part_ss + ((int64_t)par * S + pc.s) * Hkv * ATT_CONSUMERS;
+        uint32_t* qw = reinterpret_cast<uint32_t*>(gbase + SL.qbuf + slot * SL.qslot);
+        float* xr = reinterpret_cast<float*>(qw + 8 * QW + D);  // x_l of the head group, for the completing CTA
+        float inv = 0.f;
+        // query pairs (lane handles element pairs 2i, 2i+1 of the head group);
+        // the first chunk's poll also covers the group sums (one round trip)
+        for (int i0 = 0; i0 < GD / 2 && ok; i0 += 32 * 8) {
+          float v0[8], v1[8], t = 0.f;
+          uint64_t t0 = 0;
+          while (true) {
+            bool good = true;
+            t = 0.f;
+            if (i0 == 0)
+              for (int i = lane; i < Hkv * ATT_CONSUMERS; i += 32) {
+                const uint64_t w = ld_tagged(ps + i);
+                good &= tv_ok(w, tag);
+                t += tv_value(w);
+              }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const int i = i0 + lane + 32 * j;
+              v0[j] = v1[j] = 0.f;
+              if (i >= GD / 2) continue;
+              const uint64_t w0 = ld_tagged(xq + 2 * i), w1 = ld_tagged(xq + 2 * i + 1);
+              good &= tv_ok(w0, tag) && tv_ok(w1, tag);
+              v0[j] = tv_value(w0);
+              v1[j] = tv_value(w1);
+            }
+            if (__all_sync(0xffffffffu, good)) break;
+            if (!poll_again(t0, a.status)) {
+              ok = false;
+              break;
+            }
+          }
+          if (!ok) break;
+          if (i0 == 0) {
+            // same summation order as every other user of these sums
+            t = warp_sum(t);
+            t = __shfl_sync(0xffffffffu, t, 0);
+            inv = 1.0f / sqrtf(t / (float)d + a.rms_eps);
+          }
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int i = i0 + lane + 32 * j;
+            if (i >= GD / 2) continue;
+            const int g = (2 * i) / D, dd = (2 * i) % D;
+            qw[g * QW + dd / 2] = pack_bf16(v0[j] * inv, v1[j] * inv);
+            xr[2 * i] = v0[j];
+            xr[2 * i + 1] = v1[j];
+          }
+        }
+        if (ok && app) {
+          // K row = head h of u, V row = head Hkv + h of u
+          const uint64_t* xk = xs + (int64_t)pc.h * D;
+          const uint64_t* xv = xs + ((int64_t)Hkv + pc.h) * D;
+          uint32_t* kr = qw + 8 * QW;
+          uint32_t* vr = kr + D / 2;
+          const int64_t grow = (int64_t)l * a.layer_elems + a.kv_offset[pc.s] +
+                               ((int64_t)pc.h * a.cap[pc.s] + lens[pc.s] - 1) * D;
+          constexpr int RW = (D / 2 + 31) / 32;  // word pairs per lane
+          float k0[RW], k1[RW], w0[RW], w1[RW];
+          uint64_t t0 = 0;
+          while (true) {
+            bool good = true;
+#pragma unroll
+            for (int j = 0; j < RW; ++j) {
+              const int i = lane + 32 * j;
+              k0[j] = k1[j] = w0[j] = w1[j] = 0.f;
+              if (i >= D / 2) continue;
+              const uint64_t a0 = ld_tagged(xk + 2 * i), a1 = ld_tagged(xk + 2 * i + 1);
+              const uint64_t b0 = ld_tagged(xv + 2 * i), b1 = ld_tagged(xv + 2 * i + 1);
+              good &= tv_ok(a0, tag) && tv_ok(a1, tag) && tv_ok(b0, tag) && tv_ok(b1, tag);
+              k0[j] = tv_value(a0);
+              k1[j] = tv_value(a1);
+              w0[j] = tv_value(b0);
+              w1[j] = tv_value(b1);
+            }
+            if (__all_sync(0xffffffffu, good)) break;
+            if (!poll_again(t0, a.status)) {
+              ok = false;
+              break;
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < RW; ++j) {
+            const int i = lane + 32 * j;
+            if (!ok || i >= D / 2) continue;
+            const uint32_t kb = pack_bf16(k0[j] * inv, k1[j] * inv);
+            const uint32_t vb = pack_bf16(w0[j] * inv, w1[j] * inv);
+            kr[i] = kb;
+            vr[i] = vb;
+            reinterpret_cast<uint32_t*>(a.k_cache + grow)[i] = kb;
+            reinterpret_cast<uint32_t*>(a.v_cache + grow)[i] = vb;
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_qfull + 8 * slot);
       }
     }
     return;
   }
 
   // -------------------------------------------------------------- consumers
-  const int ctid = tid, wg = warp >> 2, wl = warp & 3;
+  const int wg = warp >> 2, wl = warp & 3;
   const int g = lane >> 2, tq = lane & 3;
   const int kb = 16 * wl;
-  uint32_t it = 0, cph = 0;
+  const bool hv = g < G;
+  uint32_t it = 0, p = 0;
   bool ok = true;
-  for (int s = blockIdx.x; s < S; s += gridDim.x) embed_sequence<D>(a, s, step_tag(epoch, 0), ctid, warp, lane);
-
   for (int l = 0; l < a.L && ok; ++l) {
-    const int par = l & 1;
-    const uint32_t tag = step_tag(epoch, l);
-    for (int64_t p = cb; p < ce && ok;) {
-      const Piece pc = find_piece(pre, lens, S, T, p, ce);
-      p += pc.adv;
+    for (int64_t pp = cb; pp < ce && ok;) {
+      const Piece pc = find_piece(pre, lens, S, T, pp, ce);
+      pp += pc.adv;
       if (pc.k0 == pc.k1) continue;
-      const int64_t pa = (int64_t)pc.h * T + pre[pc.s];
-      const int64_t c0 = pa / P, c1 = (pa + lens[pc.s] - 1) / P;
-      const bool merges = c0 == (int64_t)blockIdx.x;  // the segment's first CTA completes it
-      // wait for this piece's layer input (head group h of x_l[s] and the
-      // partial sums of squares of x_l[s]); form the query bf16(x_l * inv_rms)
-      const uint64_t* xs = a.resid + ((int64_t)par * S + pc.s) * d;
-      const bool hv = g < G;
-      const uint64_t* xq = xs + ((int64_t)pc.h * G + (hv ? g : 0)) * D;
-      float2 xl[C::KSTEPS], xh[C::KSTEPS];
-      float xold[C::OPT];
-      {
-        uint64_t t0 = 0;
-        while (true) {
-          bool good = true;
-#pragma unroll
-          for (int j = 0; j < C::KSTEPS; ++j) {
-            const uint64_t w0 = ld_tagged(xq + 16 * j + 2 * tq), w1 = ld_tagged(xq + 16 * j + 2 * tq + 1);
-            const uint64_t w2 = ld_tagged(xq + 16 * j + 8 + 2 * tq), w3 = ld_tagged(xq + 16 * j + 9 + 2 * tq);
-            good &= tv_ok(w0, tag) && tv_ok(w1, tag) && tv_ok(w2, tag) && tv_ok(w3, tag);
-            xl[j] = make_float2(tv_value(w0), tv_value(w1));
-            xh[j] = make_float2(tv_value(w2), tv_value(w3));
-          }
-#pragma unroll
-          for (int k = 0; k < C::OPT; ++k) {
-            const int idx = ctid + k * ATT_CT;
-            xold[k] = 0.f;
-            if (!merges || idx >= GD) continue;
-            const uint64_t w = ld_tagged(xs + (int64_t)pc.h * GD + idx);
-            good &= tv_ok(w, tag);
-            xold[k] = tv_value(w);
-          }
-          if (__all_sync(0xffffffffu, good)) break;
-          if (!poll_again(t0, a.status)) {
-            ok = false;
-            break;
-          }
-        }
-      }
-      float inv = 0.f;
-      if (ok && !wait_inv_rms(a.part_ss + ((int64_t)par * S + pc.s) * Hkv * ATT_CONSUMERS, Hkv * ATT_CONSUMERS, tag,
-                              d, a.rms_eps, lane, a.status, inv))
+      const uint32_t slot = p & 1u, u = p >> 1;
+      ++p;
+      if (!mbar_wait(bar_qfull + 8 * slot, u & 1u, a.status)) {
         ok = false;
-      if (!ok) break;
+        break;
+      }
+      const uint32_t* qw = reinterpret_cast<const uint32_t*>(gbase + SL.qbuf + slot * SL.qslot);
       uint32_t qf[C::KSTEPS][2];
 #pragma unroll
       for (int j = 0; j < C::KSTEPS; ++j) {
-        qf[j][0] = hv ? pack_bf16(xl[j].x * inv, xl[j].y * inv) : 0u;
-        qf[j][1] = hv ? pack_bf16(xh[j].x * inv, xh[j].y * inv) : 0u;
+        qf[j][0] = hv ? qw[g * QW + 8 * j + tq] : 0u;
+        qf[j][1] = hv ? qw[g * QW + 8 * j + 4 + tq] : 0u;
       }
-      const int32_t app_row = (sc.apnd[pc.s] && pc.k1 == lens[pc.s]) ? lens[pc.s] - 1 : -1;
+      const int32_t app_row = (apnd[pc.s] && pc.k1 == lens[pc.s]) ? lens[pc.s] - 1 : -1;
 
       WarpAcc<D> A;
       acc_reset(A);
       for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
         if ((int)(it & 1u) != wg) continue;
-        const uint32_t use = it / C::STAGES, st = it % C::STAGES, ph = use & 1u;
+        const uint32_t use = it / NST, st = it % NST, ph = use & 1u;
         if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status)) {
           ok = false;
           break;
@@ -911,102 +963,215 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
         }
         const int nvalid = min(ATT_BLOCK_N, pc.k1 - kt);
         const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
-        if (app_row >= kt && app_row < kt + ATT_BLOCK_N && ((app_row - kt) >> 4) == wl &&
-            !patch_row<D>(a, xs, tag, inv, pc, app_row, app_row - kt, l, sk, sv, lane)) {
-          ok = false;
-          break;
+        if (app_row >= kt && app_row < kt + ATT_BLOCK_N && ((app_row - kt) >> 4) == wl) {
+          // the appended row (prepared by the input warp) replaces whatever
+          // the cache held there when the tile was loaded
+          const int r = app_row - kt;
+          const uint32_t src = base + SL.qbuf + slot * SL.qslot + 8 * QW * 4;
+          for (int c = lane; c < 2 * (D / 8); c += 32) {
+            const int cc = c % (D / 8);
+            const uint32_t dst = (c < D / 8 ? sk : sv) + (cc >> 3) * C::BOX_BYTES + r * 128 +
+                                 ((((uint32_t)cc & 7u) ^ ((uint32_t)r & 7u)) << 4);
+            uint32_t w0, w1, w2, w3;
+            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
+                         : "r"(src + 16 * c));
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w0), "r"(w1), "r"(w2), "r"(w3)
+                         : "memory");
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
         }
         if (kb < nvalid) tile_math<D>(A, qf, sk, sv, kb, nvalid, a.scale_log2, lane);
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_empty + 8 * st);
       }
       if (!ok) break;
-
-      float mx[C::OPT], ls[C::OPT], acc[C::OPT], o[C::OPT];
-      if (!cta_merge<D>(A, sc, G, warp, lane, ctid, bar_c, cph, a.status, mx, ls, acc)) {
+      const int64_t seg = (int64_t)pc.h * S + pc.s;
+      const int64_t pa = (int64_t)pc.h * T + pre[pc.s];
+      const int64_t c0 = pa / P, c1 = (pa + lens[pc.s] - 1) / P;
+      const bool merges = c0 == (int64_t)blockIdx.x;  // the segment's first CTA completes it
+      if (!merges) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(bar_qempty + 8 * slot);
+      }
+      // combine the eight warps' partials through a double-buffered slot
+      if (u > 0 && !mbar_wait(bar_pempty + 8 * slot, (u - 1u) & 1u, a.status)) {
         ok = false;
         break;
       }
-      const int64_t seg = (int64_t)pc.h * S + pc.s;
+      float l0 = A.l0, l1 = A.l1;
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {
+        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+      }
+      float* ms = reinterpret_cast<float*>(gbase + SL.pbuf + slot * SL.pslot);
+      float* ls = ms + ATT_CONSUMERS * ATT_MAX_G;
+      float* os = ls + ATT_CONSUMERS * ATT_MAX_G;
+      if (g == 0) {
+        ms[warp * ATT_MAX_G + 2 * tq] = A.m0;
+        ms[warp * ATT_MAX_G + 2 * tq + 1] = A.m1;
+        ls[warp * ATT_MAX_G + 2 * tq] = l0;
+        ls[warp * ATT_MAX_G + 2 * tq + 1] = l1;
+      }
+      float* ow = os + warp * D * SL.opad;
+      const bool h0 = 2 * tq < G, h1 = 2 * tq + 1 < G;
+#pragma unroll
+      for (int i = 0; i < C::MTILES; ++i) {
+        const int d0 = 16 * i + g, d1 = d0 + 8;
+        if (h0) {
+          ow[d0 * SL.opad + 2 * tq] = A.o[i][0];
+          ow[d1 * SL.opad + 2 * tq] = A.o[i][2];
+        }
+        if (h1) {
+          ow[d0 * SL.opad + 2 * tq + 1] = A.o[i][1];
+          ow[d1 * SL.opad + 2 * tq + 1] = A.o[i][3];
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_pfull + 8 * slot);
+      if (!mbar_wait(bar_pfull + 8 * slot, u & 1u, a.status)) {
+        ok = false;
+        break;
+      }
+      const uint32_t tag = step_tag(epoch, l);
+      float mx[C::OPT], lsum[C::OPT], acc[C::OPT];
+#pragma unroll
+      for (int k = 0; k < C::OPT; ++k) {
+        const int idx = tid + ATT_CT * k;
+        mx[k] = -INFINITY;
+        lsum[k] = acc[k] = 0.f;
+        if (idx >= GD) continue;
+        const int hh = idx / D, dd = idx - hh * D;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < ATT_CONSUMERS; ++w) M = fmaxf(M, ms[w * ATT_MAX_G + hh]);
+        float ac = 0.f, lv = 0.f;
+#pragma unroll
+        for (int w = 0; w < ATT_CONSUMERS; ++w) {
+          const float mw = ms[w * ATT_MAX_G + hh];
+          if (mw == -INFINITY) continue;
+          const float e = exp2f(mw - M);
+          ac += os[(w * D + dd) * SL.opad + hh] * e;
+          lv += ls[w * ATT_MAX_G + hh] * e;
+        }
+        mx[k] = M;
+        lsum[k] = lv;
+        acc[k] = ac;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_pempty + 8 * slot);
       if (!merges) {
-        // publish this CTA's record of the segment for its first CTA
-        const int64_t slot = (int64_t)blockIdx.x + seg;
+        // the segment continues in an earlier CTA: publish this CTA's record
+        const int64_t rs = (int64_t)blockIdx.x + seg;
 #pragma unroll
         for (int k = 0; k < C::OPT; ++k) {
-          const int idx = ctid + k * ATT_CT;
+          const int idx = tid + ATT_CT * k;
           if (idx >= GD) continue;
-          st_tagged(a.rec_o + slot * GD + idx, acc[k], tag);
+          st_tagged(a.rec_o + rs * GD + idx, acc[k], tag);
           if (idx % D == 0) {
-            st_tagged(a.rec_ml + (slot * G + idx / D) * 2, mx[k], tag);
-            st_tagged(a.rec_ml + (slot * G + idx / D) * 2 + 1, ls[k], tag);
+            st_tagged(a.rec_ml + (rs * G + idx / D) * 2, mx[k], tag);
+            st_tagged(a.rec_ml + (rs * G + idx / D) * 2 + 1, lsum[k], tag);
           }
         }
         continue;
       }
-      // complete the segment: this CTA's part, then the records of CTAs
-      // c0+1..c1 in order (deterministic)
+      // complete the segment: the records of CTAs c0+1..c1 in order (RB at a
+      // time, one round trip when they are there)
+      constexpr int RB = 2;
+      for (int64_t c = c0 + 1; c <= c1 && ok; c += RB) {
+        float mv[C::OPT][RB], lv[C::OPT][RB], ov[C::OPT][RB];
+        uint64_t t0 = 0;
+        while (true) {
+          bool good = true;
 #pragma unroll
-      for (int k = 0; k < C::OPT; ++k) {
-        const int idx = ctid + k * ATT_CT;
-        o[k] = 0.f;
-        if (idx >= GD) continue;
-        const int hh = idx / D;
-        float M = mx[k], Ls = ls[k], Ac = acc[k];
-        for (int64_t c = c0 + 1; c <= c1 && ok; c += 4) {
-          float mv[4], lv[4], ov[4];
-          uint64_t t0 = 0;
-          while (true) {
-            bool good = true;
+          for (int k = 0; k < C::OPT; ++k) {
+            const int idx = tid + ATT_CT * k, hh = idx / D;
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              mv[u] = -INFINITY;
-              lv[u] = 0.f;
-              ov[u] = 0.f;
-              if (c + u > c1) continue;
-              const int64_t sl = c + u + seg;
-              const uint64_t wm = ld_tagged(a.rec_ml + (sl * G + hh) * 2);
-              const uint64_t wl2 = ld_tagged(a.rec_ml + (sl * G + hh) * 2 + 1);
-              const uint64_t wo = ld_tagged(a.rec_o + sl * GD + idx);
-              good &= tv_ok(wm, tag) && tv_ok(wl2, tag) && tv_ok(wo, tag);
-              mv[u] = tv_value(wm);
-              lv[u] = tv_value(wl2);
-              ov[u] = tv_value(wo);
-            }
-            if (good) break;
-            if (!poll_again(t0, a.status)) {
-              ok = false;
-              break;
+            for (int q = 0; q < RB; ++q) {
+              mv[k][q] = -INFINITY;
+              lv[k][q] = ov[k][q] = 0.f;
+              if (idx >= GD || c + q > c1) continue;
+              const int64_t rs = c + q + seg;
+              const uint64_t wm = ld_tagged(a.rec_ml + (rs * G + hh) * 2);
+              const uint64_t wl = ld_tagged(a.rec_ml + (rs * G + hh) * 2 + 1);
+              const uint64_t wo = ld_tagged(a.rec_o + rs * GD + idx);
+              good &= tv_ok(wm, tag) && tv_ok(wl, tag) && tv_ok(wo, tag);
+              mv[k][q] = tv_value(wm);
+              lv[k][q] = tv_value(wl);
+              ov[k][q] = tv_value(wo);
             }
           }
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            if (mv[u] == -INFINITY) continue;
-            const float Mn = fmaxf(M, mv[u]);
-            const float f = M == -INFINITY ? 0.f : exp2f(M - Mn), e = exp2f(mv[u] - Mn);
-            Ac = Ac * f + ov[u] * e;
-            Ls = Ls * f + lv[u] * e;
-            M = Mn;
+          if (__all_sync(0xffffffffu, good)) break;
+          if (!poll_again(t0, a.status)) {
+            ok = false;
+            break;
           }
         }
-        o[k] = Ls > 0.f ? Ac / Ls : 0.f;
+#pragma unroll
+        for (int k = 0; k < C::OPT; ++k)
+#pragma unroll
+          for (int q = 0; q < RB; ++q) {
+            if (mv[k][q] == -INFINITY) continue;
+            const float Mn = fmaxf(mx[k], mv[k][q]);
+            const float f = mx[k] == -INFINITY ? 0.f : exp2f(mx[k] - Mn), e = exp2f(mv[k][q] - Mn);
+            acc[k] = acc[k] * f + ov[k][q] * e;
+            lsum[k] = lsum[k] * f + lv[k][q] * e;
+            mx[k] = Mn;
+          }
       }
       if (!ok) break;
-      if (!finish_segment<D>(a, l, pc.h, pc.s, epoch, xold, o, ctid, warp, lane)) {
+      // x_{l+1} = x_l + o for head group h (x_l from the input warp's slot)
+      const int nx = (l + 1) & 1;
+      const uint32_t ntag = step_tag(epoch, l + 1);
+      const float* xr = reinterpret_cast<const float*>(qw + 8 * QW + D);
+      uint64_t* xn = a.resid + ((int64_t)nx * S + pc.s) * d + (int64_t)pc.h * GD;
+      float xv[C::OPT];
+      float ss = 0.f;
+#pragma unroll
+      for (int k = 0; k < C::OPT; ++k) {
+        const int idx = tid + ATT_CT * k;
+        xv[k] = 0.f;
+        if (idx >= GD) continue;
+        xv[k] = xr[idx] + (lsum[k] > 0.f ? acc[k] / lsum[k] : 0.f);
+        st_tagged(xn + idx, xv[k], ntag);
+        ss += xv[k] * xv[k];
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_qempty + 8 * slot);
+      ss = warp_sum(ss);
+      uint64_t* ps = a.part_ss + ((int64_t)nx * S + pc.s) * Hkv * ATT_CONSUMERS;
+      if (lane == 0) st_tagged(ps + pc.h * ATT_CONSUMERS + warp, ss, ntag);
+      if (l + 1 < a.L) continue;
+      // after the last layer: head group h of the final hidden state
+      float inv;
+      if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, ntag, d, a.rms_eps, lane, a.status, inv)) {
         ok = false;
         break;
       }
+      __nv_bfloat16* hs = a.hidden + (int64_t)pc.s * d + (int64_t)pc.h * GD;
+      __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)pc.s * d + (int64_t)pc.h * GD : nullptr;
+#pragma unroll
+      for (int k = 0; k < C::OPT; ++k) {
+        const int idx = tid + ATT_CT * k;
+        if (idx >= GD) continue;
+        const __nv_bfloat16 hv2 = __float2bfloat16_rn(xv[k] * inv);
+        hs[idx] = hv2;
+        if (hc) hc[idx] = hv2;
+      }
     }
   }
-
   // ---- the last CTA to finish advances seq_len and the epoch
-  if (ctid == 0) {
+  uint32_t cph = 0;
+  if (tid == 0) {
     const int prev = atom_acq_rel_gpu_add(a.done_cnt, 1);
-    sc.flag[3] = prev == (int)gridDim.x - 1;
+    flag[0] = prev == (int)gridDim.x - 1;
   }
-  if (warps_sync(bar_c, cph, a.status) && sc.flag[3]) {
-    for (int i = ctid; i < S; i += ATT_CT)
-      if (sc.apnd[i]) a.seq_len[i] = lens[i];
-    if (ctid == 0) {
+  if (warps_sync(bar_m, cph, a.status) && flag[0]) {
+    for (int i = tid; i < S; i += ATT_CT)
+      if (apnd[i]) a.seq_len[i] = lens[i];
+    if (tid == 0) {
       *a.done_cnt = 0;
       *a.epoch = epoch + 1;
     }
@@ -1041,7 +1206,7 @@ static int env_int(const char* name, int dflt, int lo, int hi) {
   const int v = atoi(e);
   return v < lo ? lo : (v > hi ? hi : v);
 }
-int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", D == 128 ? 1024 : 2048, 0, 1 << 20); }
+int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", D == 128 ? 256 : 512, 0, 1 << 20); }
 int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 6, 0, 64); }
 
 // cudaFuncSetAttribute once per kernel and device
@@ -1085,14 +1250,15 @@ template <int D>
 static cudaError_t launch_step(const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
                                cudaStream_t stream) {
   static bool configured[64];
-  cudaError_t e = set_smem_once(att_step_kernel<D>, AttCfg<D>::SMEM, configured);
+  const StepSmem SL = step_smem(D, a.G);
+  cudaError_t e = set_smem_once(att_step_kernel<D>, 227 * 1024, configured);
   if (e != cudaSuccess) return e;
   // every CTA waits for the others' layer results, so all must be resident at
   // once: a cooperative launch guarantees it (or fails)
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(ctas);
-  cfg.blockDim = dim3(ATT_THREADS);
-  cfg.dynamicSmemBytes = AttCfg<D>::SMEM;
+  cfg.blockDim = dim3(STEP_THREADS);
+  cfg.dynamicSmemBytes = SL.total;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeCooperative;

@@ -69,18 +69,21 @@ cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream);
 // layers (a shared-memory ring plus L2 prefetch ahead of it) while the
 // consumers wait for the layer dependency.
 //
+// Roles inside a CTA (warp-specialised, hand-offs through double-buffered
+// shared-memory slots guarded by mbarriers): a producer warp (TMA), an input
+// warp that prepares each piece's query bf16(x_l * inv_rms(x_l)) and the row
+// appended this step, eight consumer warps that only run the attention math,
+// and a two-warp merge group that combines the consumers' partials.
+//
 // Layer dependency: a segment split over CTAs c0..c1 is completed by c0 (for
 // which it is the last piece of the layer); c0+1..c1 publish their records
 // for it.  The completing CTA adds the head group's attention output to the
 // residual stream, x_{l+1} = x_l + o (double buffered by layer parity), and
-// stores per-warp partial sums of squares.  A piece of layer l waits for its
-// head group of x_l[s] and all partial sums of x_l[s], forms its query
-// bf16(x_l * inv_rms(x_l)) itself, and the warp that owns the row appended
-// this step writes that row's K/V (the same normalised stream) into the
-// shared tile and the cache.  Everything exchanged between CTAs is a tagged
-// 64-bit word (see attention.cu).  After the last layer each completing CTA
-// writes its head group of the final hidden state; the last CTA to finish
-// advances seq_len and the epoch.
+// stores the group's sum of squares.  A piece of layer l waits for its head
+// group of x_l[s] and all group sums of x_l[s].  Everything exchanged between
+// CTAs is a tagged 64-bit word (see attention.cu).  After the last layer each
+// completing CTA writes its head group of the final hidden state; the last
+// CTA to finish advances seq_len and the epoch.
 struct StepAttArgs {
   int32_t S, Hq, Hkv, G, L, n1, V, bos, max_steps;
   int64_t rows_per_layer;     // rows (of D elements) of one layer's region in the tensor maps
@@ -97,7 +100,7 @@ struct StepAttArgs {
   __nv_bfloat16* k_cache;
   __nv_bfloat16* v_cache;
   uint64_t* resid;            // [2][S][d] tagged residual stream x_l (buffer l % 2)
-  uint64_t* part_ss;          // [2][S][Hkv][8] tagged per-warp sums of squares of x_l
+  uint64_t* part_ss;          // [2][S][Hkv][8] tagged sums of squares of x_l per head group and consumer warp
   uint64_t* rec_o;            // [slots][G*D] tagged partial outputs
   uint64_t* rec_ml;           // [slots][G][2] tagged (max, sum)
   int32_t* epoch;             // [1] launches completed (tags name the launch)
