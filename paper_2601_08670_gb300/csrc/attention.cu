@@ -1207,7 +1207,7 @@ static int env_int(const char* name, int dflt, int lo, int hi) {
   return v < lo ? lo : (v > hi ? hi : v);
 }
 int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", D == 128 ? 256 : 512, 0, 1 << 20); }
-int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 6, 0, 64); }
+int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 12, 0, 64); }
 
 // cudaFuncSetAttribute once per kernel and device
 template <typename K>
