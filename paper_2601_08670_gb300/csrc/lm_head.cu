@@ -16,6 +16,7 @@
 // constant in v, Eq. 3 only needs these per-tile maxima and the log-sum-exps L:
 // the [S x V] logits never reach HBM on the fused path.
 #include <math.h>
+#include <stdlib.h>
 
 #include "lm_head.cuh"
 
@@ -44,8 +45,9 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
   const size_t slab = LM_A_BYTES + (size_t)g->S_pad * 128;
   const size_t fixed = 1024 + 64 * 8 + 16 + (size_t)2 * 4 * g->S_pad * sizeof(float2) +
                        (size_t)2 * g->S_pad * sizeof(float2) + (size_t)g->nbeta * 4 + 64;
-  // several consecutive K-slabs per stage so each row is fetched in longer runs;
-  // keep at least three stages in flight
+  // several consecutive K-slabs per stage so each row is fetched in longer
+  // runs and the tensor cores get longer bursts per stage; keep at least
+  // three stages in flight
   g->slabs = 1;
   for (int sl = 4; sl >= 2; sl >>= 1)
     if (g->nks % sl == 0 && fixed + 3 * sl * slab <= LM_SMEM_BUDGET) {
@@ -107,6 +109,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     tma_prefetch_desc(&wmap);
     tma_prefetch_desc(&hmap);
   }
+  if (a.pdl) pdl_launch_dependents();
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), a.tmem_cols);
     tmem_relinquish();
@@ -127,26 +130,45 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     // ---------------------------------------------------------------- TMA
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
+      // stage load i covers K-slabs (i % nst)*SL .. of tile blockIdx.x + (i / nst)*gridDim.x
+      const int my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+      const uint32_t nloads = (uint32_t)my_tiles * (uint32_t)nst;
+      auto load_w = [&](uint32_t i) {
+        const uint32_t st = i % stages;
+        const int tile = (int)blockIdx.x + (int)(i / nst) * (int)gridDim.x, ks = (int)(i % nst);
+        const uint32_t fb = bar_full + 8 * st, sa = base + st * st_bytes;
+        mbar_arrive_expect_tx(fb, st_bytes);
+        // consecutive K-slabs of the same 128 rows back to back: longer runs per row
+        for (int j = 0; j < SL; ++j)
+          tma_load_2d(sa + j * LM_A_BYTES, &wmap, fb, (ks * SL + j) * LM_TILE_K, tile * LM_TILE_V, pol_w);
+      };
+      auto load_h = [&](uint32_t i) {
+        const uint32_t st = i % stages;
+        const int ks = (int)(i % nst);
+        const uint32_t fb = bar_full + 8 * st, sb = base + st * st_bytes + SL * LM_A_BYTES;
+        for (int j = 0; j < SL; ++j)
+          for (int c = 0; c < a.nchunk; ++c)
+            tma_load_2d(sb + j * b_bytes + c * a.chunk_n * 128, &hmap, fb, (ks * SL + j) * LM_TILE_K,
+                        c * a.chunk_n, pol_h);
+      };
+      // With programmatic dependent launch the weights of the first stages
+      // stream while the previous kernel (which writes H) finishes.
       uint32_t it = 0;
+      if (a.pdl) {
+        const uint32_t npre = nloads < (uint32_t)stages ? nloads : (uint32_t)stages;
+        for (; it < npre; ++it) load_w(it);
+        pdl_wait();
+        for (uint32_t i = 0; i < npre; ++i) load_h(i);
+      }
       bool ok = true;
-      for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-        for (int ks = 0; ks < nst; ++ks, ++it) {
-          const uint32_t st = it % stages, ph = (it / stages) & 1u;
-          if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
-            ok = false;
-            break;
-          }
-          const uint32_t fb = bar_full + 8 * st;
-          const uint32_t sa = base + st * st_bytes, sb = sa + SL * LM_A_BYTES;
-          mbar_arrive_expect_tx(fb, st_bytes);
-          // consecutive K-slabs of the same 128 rows back to back: longer runs per row
-          for (int j = 0; j < SL; ++j)
-            tma_load_2d(sa + j * LM_A_BYTES, &wmap, fb, (ks * SL + j) * LM_TILE_K, tile * LM_TILE_V, pol_w);
-          for (int j = 0; j < SL; ++j)
-            for (int c = 0; c < a.nchunk; ++c)
-              tma_load_2d(sb + j * b_bytes + c * a.chunk_n * 128, &hmap, fb, (ks * SL + j) * LM_TILE_K,
-                          c * a.chunk_n, pol_h);
+      for (; it < nloads; ++it) {
+        const uint32_t st = it % stages, ph = (it / stages) & 1u;
+        if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
+          ok = false;
+          break;
         }
+        load_w(it);
+        load_h(it);
       }
       if (!ok) {
         for (uint32_t j = (it >= (uint32_t)stages ? it - stages : 0); j < it; ++j)
@@ -173,13 +195,26 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
           }
           tc_fence_after();
           const uint32_t sa = base + st * st_bytes, sb = sa + SL * LM_A_BYTES;
-          for (int j = 0; j < SL; ++j) {
+          // descriptors are built once per stage; a K-step moves the start
+          // address field (bytes >> 4) by 2, a slab by its size >> 4
+          const uint64_t ad0 = umma_desc_sw128(sa), bd0 = umma_desc_sw128(sb);
+          if (SL == 4 && a.nchunk == 1) {
+            const uint32_t bstep = b_bytes >> 4;
 #pragma unroll
-            for (int k = 0; k < LM_TILE_K / 16; ++k) {
-              const uint64_t ad = umma_desc_sw128(sa + j * LM_A_BYTES + 32 * k);
-              for (int c = 0; c < a.nchunk; ++c)
-                umma_bf16(dcol + c * a.chunk_n, ad, umma_desc_sw128(sb + j * b_bytes + c * a.chunk_n * 128 + 32 * k),
+            for (int j = 0; j < 4; ++j)
+#pragma unroll
+              for (int k = 0; k < LM_TILE_K / 16; ++k)
+                umma_bf16(dcol, ad0 + (uint64_t)(j * (LM_A_BYTES >> 4) + 2 * k), bd0 + (uint64_t)(j * bstep + 2 * k),
                           idesc, (ks | j | k) != 0);
+          } else {
+            for (int j = 0; j < SL; ++j) {
+#pragma unroll
+              for (int k = 0; k < LM_TILE_K / 16; ++k) {
+                const uint64_t ad = ad0 + (uint64_t)(j * (LM_A_BYTES >> 4) + 2 * k);
+                for (int c = 0; c < a.nchunk; ++c)
+                  umma_bf16(dcol + c * a.chunk_n, ad, bd0 + (uint64_t)((j * b_bytes + c * a.chunk_n * 128) >> 4) + 2 * k,
+                            idesc, (ks | j | k) != 0);
+              }
             }
           }
           umma_commit(bar_empty + 8 * st);
@@ -213,6 +248,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       for (int cb = 0; cb < S_pad / 16; ++cb) {
         float vals[16];
         tmem_ld16(trow + cb * 16, vals);
+
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int col = cb * 16 + i;
@@ -294,8 +330,17 @@ cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, con
     if (e != cudaSuccess) return e;
     configured = LM_SMEM_BUDGET;
   }
-  lm_head_kernel<<<g.grid, LM_THREADS, g.smem, stream>>>(wmap, hmap, a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(g.grid);
+  cfg.blockDim = dim3(LM_THREADS);
+  cfg.dynamicSmemBytes = g.smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = a.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, lm_head_kernel, wmap, hmap, a);
 }
 
 // ------------------------------------------------------------ mode-0 finish
@@ -341,6 +386,7 @@ cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float
 __global__ void __launch_bounds__(256) select_from_records_kernel(SelectArgs a) {
   const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int N = a.N, n1 = N + 1, s0 = b * n1, T = a.nrec;
+  if (a.pdl) pdl_wait();  // the LM head's records are complete and visible
   __shared__ float Ls[LM_MAX_N1];
   __shared__ float ksc[LM_MAX_N1];
   __shared__ int ktok[LM_MAX_N1];
@@ -429,8 +475,16 @@ __global__ void __launch_bounds__(256) select_from_records_kernel(SelectArgs a) 
 }
 
 cudaError_t select_from_records_launch(const SelectArgs& a, cudaStream_t stream) {
-  select_from_records_kernel<<<a.B, 256, 0, stream>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.B);
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = a.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, select_from_records_kernel, a);
 }
 
 }  // namespace pced

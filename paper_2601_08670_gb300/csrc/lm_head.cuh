@@ -27,6 +27,7 @@ struct LmArgs {
   float2* rec_stats;  // [S][grid] (max z, sum exp(z - max)) over each CTA's tiles
   float2* rec_arg;    // [S][grid] (max u, argmax v as int bits) for expert columns, mode 1
   const float* beta;  // [B][N]
+  int pdl;            // launched as a programmatic dependent of the kernel that writes H
   int* status;
 };
 
@@ -55,6 +56,7 @@ struct SelectArgs {
   float* score_trace;
   int32_t max_steps;
   int32_t* done_counter;
+  int pdl;            // launched as a programmatic dependent of the LM head
   int* status;
 };
 cudaError_t select_from_records_launch(const SelectArgs& a, cudaStream_t stream);

@@ -180,6 +180,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.rec_arg = W.lm_arg;
   la.beta = p->beta;
   la.status = W.status;
+  la.pdl = timed ? 0 : 1;  // stage events between the launches would break the overlap
   e = lm_head_launch(wmap, hmap, g, la, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "lm head launch");
@@ -201,6 +202,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.max_steps = p->max_steps;
   sa.done_counter = W.done_counter;
   sa.status = W.status;
+  sa.pdl = timed ? 0 : 1;
   e = select_from_records_launch(sa, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "select launch");
