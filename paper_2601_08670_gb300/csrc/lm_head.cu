@@ -9,9 +9,12 @@
 //   warp 0  TMA producer (W tile 128x64 + H slab S_pad x 64 per stage, 128B swizzle)
 //   warp 1  TMEM allocator and single-thread tcgen05.mma issuer (fp32 accumulators
 //           in TMEM, double-buffered when 2*S_pad <= 512 columns)
-//   warps 2-5 epilogue: tcgen05.ld of the 128 x S accumulator; per column the tile's
-//           (max, sum exp) for the log-softmax and, for each contextual expert k of
-//           query b, the tile's max and argmax of u_k(v) = (1+beta_k) z_k(v) - beta_k z_0(v).
+//   warps 2-9 epilogue: tcgen05.ld of the 128 x S accumulator (warp w reads TMEM lane
+//           quarter w % 4; warps 2-5 take the first half of the columns, 6-9 the rest);
+//           per column the tile's (max, sum exp) for the log-softmax and, for each
+//           contextual expert k of query b, the tile's max and argmax of
+//           u_k(v) = (1+beta_k) z_k(v) - beta_k z_0(v), reduced over the rows with
+//           transposed butterflies (one shuffle per column and reduction).
 // Because shat_k(v) = u_k(v) + c_k with c_k = -(1+beta_k) L_k + beta_k L_0 + gamma log r_k
 // constant in v, Eq. 3 only needs these per-tile maxima and the log-sum-exps L:
 // the [S x V] logits never reach HBM on the fused path.
@@ -44,7 +47,7 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
   g->nbeta = S;  // beta has B*N < S entries
   const size_t slab = LM_A_BYTES + (size_t)g->S_pad * 128;
   const size_t fixed = 1024 + 64 * 8 + 16 + (size_t)2 * 4 * g->S_pad * sizeof(float2) +
-                       (size_t)2 * g->S_pad * sizeof(float2) + (size_t)g->nbeta * 4 + 64;
+                       (size_t)2 * g->S_pad * sizeof(float2) + (size_t)(g->nbeta + 3) * 4 + 8 * 64 * 4 + 64;
   // several consecutive K-slabs per stage so each row is fetched in longer
   // runs and the tensor cores get longer bursts per stage; keep at least
   // three stages in flight
@@ -65,6 +68,118 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
   g->grid = g->ntiles < sms ? g->ntiles : sms;
   if (g->grid < 1) g->grid = 1;
   return true;
+}
+
+struct FMax {
+  __device__ __forceinline__ float operator()(float x, float y) const { return fmaxf(x, y); }
+};
+struct FAdd {
+  __device__ __forceinline__ float operator()(float x, float y) const { return x + y; }
+};
+
+// Reduce NB columns held one per register over the 32 lanes (vocabulary rows)
+// of a warp in transposed form: every exchange hands half of the columns still
+// held to the partner lane, so NB columns cost NB - 1 shuffles instead of
+// 5 NB.  The pairing (lane bit 4 first, bit 0 last) is that of a per-column
+// xor tree, so sums round identically.  NB = 32: lane l ends with column l;
+// NB = 16: after a full exchange across lane bit 4, lanes l and l ^ 16 both
+// end with column l & 15.
+template <int NB, class Op>
+__device__ __forceinline__ float bfly_reduce(float (&x)[NB], int lane, Op op) {
+  if (NB == 16) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) x[i] = op(x[i], __shfl_xor_sync(0xffffffffu, x[i], 16));
+  }
+#pragma unroll
+  for (int w = NB / 2; w >= 1; w >>= 1) {
+    const bool hi = (lane & w) != 0;
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      const float send = hi ? x[i] : x[i + w];
+      const float keep = hi ? x[i + w] : x[i];
+      x[i] = op(keep, __shfl_xor_sync(0xffffffffu, send, w));
+    }
+  }
+  return x[0];
+}
+
+// Epilogue of NB accumulator columns c0.. of one warp's 32 vocabulary rows:
+// mode 0 stores the logits; both modes record the per-column (max, sum of
+// exp) of the 32 rows; mode 1 also records per expert column the max of
+// u_k = (1 + beta) z_k - beta z_0 and its first (lowest) vocabulary index.
+// `bc` is this warp's 64-float broadcast buffer; z_am carries the row's
+// amateur logit from its query's first column to the expert columns.
+template <int NB>
+__device__ __forceinline__ void epi_block(const LmArgs& a, uint32_t taddr, int c0, int v, bool valid, int lane,
+                                          int q, float* bc, float2* wst, float2* wag, const float* sbeta,
+                                          float& z_am) {
+  const int S = a.S, S_pad = a.S_pad, n1 = a.N + 1;
+  float z[NB], t[NB];
+  tmem_ld16(taddr, z);
+  if (NB == 32) tmem_ld16(taddr + 16, z + 16);
+  if (a.mode == 0 && valid) {
+#pragma unroll
+    for (int i = 0; i < NB; ++i)
+      if (c0 + i < S) a.logits[(int64_t)(c0 + i) * a.V + v] = z[i];
+  }
+#pragma unroll
+  for (int i = 0; i < NB; ++i) t[i] = valid ? z[i] : -INFINITY;
+  const float m = bfly_reduce<NB>(t, lane, FMax());
+  const int li = lane & (NB - 1), mycol = c0 + li;
+  if (lane < NB) bc[lane] = m;
+  __syncwarp();
+#pragma unroll
+  for (int i = 0; i < NB; ++i) t[i] = valid ? __expf(z[i] - bc[i]) : 0.f;
+  const float sm = bfly_reduce<NB>(t, lane, FAdd());
+  if (lane < NB && mycol < S) wst[q * S_pad + mycol] = make_float2(m, sm);
+  if (a.mode == 1) {
+    float u[NB];
+#pragma unroll
+    for (int i = 0, j = c0 % n1, b = c0 / n1; i < NB; ++i) {
+      u[i] = -INFINITY;
+      if (c0 + i < S) {
+        if (j == 0) {
+          z_am = z[i];
+        } else {
+          const float bt = sbeta[b * a.N + j - 1];
+          if (valid) u[i] = (1.f + bt) * z[i] - bt * z_am;
+        }
+      }
+      t[i] = u[i];
+      if (++j == n1) {
+        j = 0;
+        ++b;
+      }
+    }
+    const float um = bfly_reduce<NB>(t, lane, FMax());
+    if (lane < NB) bc[32 + lane] = um;
+    __syncwarp();
+    unsigned mine = 0;
+#pragma unroll
+    for (int i = 0; i < NB; ++i) {
+      const unsigned hit = __ballot_sync(0xffffffffu, u[i] == bc[32 + i]);
+      if (li == i) mine = hit;
+    }
+    if (lane < NB && mycol < S && mycol % n1 != 0) {
+      const int r = mine ? __ffs(mine) - 1 : 0;
+      wag[q * S_pad + mycol] = make_float2(um, __int_as_float(v - lane + r));
+    }
+  }
+  __syncwarp();
+}
+
+// The MMAs of one stage of SL K-slabs (single N chunk), fully unrolled: the
+// start-address field of a K-major SW128 descriptor advances by 2 per 16-wide
+// K-step and by the slab size >> 4 per slab.
+template <int SL>
+__device__ __forceinline__ void umma_slabs(uint32_t dcol, uint64_t ad0, uint64_t bd0, uint32_t bstep, uint32_t idesc,
+                                           bool first) {
+#pragma unroll
+  for (int j = 0; j < SL; ++j)
+#pragma unroll
+    for (int k = 0; k < LM_TILE_K / 16; ++k)
+      umma_bf16(dcol, ad0 + (uint64_t)(j * (LM_A_BYTES >> 4) + 2 * k), bd0 + (uint64_t)(j * bstep + 2 * k), idesc,
+                !(first && j == 0 && k == 0));
 }
 
 __global__ void __launch_bounds__(LM_THREADS, 1)
@@ -90,6 +205,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
   float2* cst = wag + 4 * S_pad;   // [S_pad] running (max, sum) over this CTA's tiles
   float2* carg = cst + S_pad;      // [S_pad] running (max u, argmax)
   float* sbeta = reinterpret_cast<float*>(carg + S_pad);  // [nbeta]
+  float* bc = sbeta + ((a.nbeta + 3) & ~3);               // [8][64] per-warp column broadcast
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
@@ -99,9 +215,9 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_tfull + 8 * i, 1);
-      mbar_init(bar_tempty + 8 * i, 128);
+      mbar_init(bar_tempty + 8 * i, LM_EPI_THREADS);
     }
-    mbar_init(bar_epi, 128);
+    mbar_init(bar_epi, LM_EPI_THREADS);
     mbar_init(bar_drain, 1);
     mbar_fence_init();
   }
@@ -198,14 +314,15 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
           // descriptors are built once per stage; a K-step moves the start
           // address field (bytes >> 4) by 2, a slab by its size >> 4
           const uint64_t ad0 = umma_desc_sw128(sa), bd0 = umma_desc_sw128(sb);
-          if (SL == 4 && a.nchunk == 1) {
+          if (a.nchunk == 1 && (SL == 4 || SL == 2 || SL == 1)) {
             const uint32_t bstep = b_bytes >> 4;
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-#pragma unroll
-              for (int k = 0; k < LM_TILE_K / 16; ++k)
-                umma_bf16(dcol, ad0 + (uint64_t)(j * (LM_A_BYTES >> 4) + 2 * k), bd0 + (uint64_t)(j * bstep + 2 * k),
-                          idesc, (ks | j | k) != 0);
+            const bool first = ks == 0;
+            if (SL == 4)
+              umma_slabs<4>(dcol, ad0, bd0, bstep, idesc, first);
+            else if (SL == 2)
+              umma_slabs<2>(dcol, ad0, bd0, bstep, idesc, first);
+            else
+              umma_slabs<1>(dcol, ad0, bd0, bstep, idesc, first);
           } else {
             for (int j = 0; j < SL; ++j) {
 #pragma unroll
@@ -230,7 +347,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
   } else {
     // ----------------------------------------------------------- epilogue
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    const int etid = tid - 64;
+    const int etid = tid - 64, half = (warp - 2) >> 2;
     const int S = a.S, n1 = a.N + 1;
     uint32_t acc = 0, ephase = 0;
     bool ok = true;
@@ -244,35 +361,19 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       const int v = tile * LM_TILE_V + 32 * q + lane;
       const bool valid = v < a.V;
       const uint32_t trow = tmem_base + ((uint32_t)(32 * q) << 16) + buf * S_pad;
+      // column blocks of 32 (the last one may be 16 wide); the first half of
+      // the blocks goes to warps 2-5, the rest to warps 6-9
+      const int nb = (S + 31) / 32, kb0 = half ? (nb + 1) / 2 : 0, kb1 = half ? nb : (nb + 1) / 2;
       float z_am = 0.f;
-      for (int cb = 0; cb < S_pad / 16; ++cb) {
-        float vals[16];
-        tmem_ld16(trow + cb * 16, vals);
-
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const int col = cb * 16 + i;
-          if (col >= S) break;
-          const float z = valid ? vals[i] : -INFINITY;
-          if (a.mode == 0 && valid) a.logits[(int64_t)col * a.V + v] = z;
-          const float mw = warp_max(z);
-          const float e = valid ? __expf(z - mw) : 0.f;
-          const float sw = warp_sum(e);
-          if (lane == 0) wst[q * S_pad + col] = make_float2(mw, sw);
-          if (a.mode == 1) {
-            const int j = col % n1;
-            if (j == 0) {
-              z_am = vals[i];
-            } else {
-              const int b = col / n1;
-              const float bt = sbeta[b * a.N + j - 1];
-              float u = valid ? (1.f + bt) * vals[i] - bt * z_am : -INFINITY;
-              int vi = v;
-              warp_argmax(u, vi);
-              if (lane == 0) wag[q * S_pad + col] = make_float2(u, __int_as_float(vi));
-            }
-          }
-        }
+      if (a.mode == 1 && kb0 < kb1 && (32 * kb0) % n1 != 0)
+        z_am = tmem_ld1(trow + 32 * kb0 - (32 * kb0) % n1);  // the row's amateur logit of the open query
+      float* wbc = bc + 64 * (warp - 2);
+      for (int kb = kb0; kb < kb1; ++kb) {
+        const int c0 = 32 * kb;
+        if (c0 + 32 <= S_pad)
+          epi_block<32>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, sbeta, z_am);
+        else
+          epi_block<16>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, sbeta, z_am);
       }
       tc_fence_before();
       mbar_arrive(bar_tempty + 8 * buf);
@@ -281,7 +382,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
         break;
       }
       // fold the four warps' results into this CTA's running records
-      for (int col = etid; col < S; col += 128) {
+      for (int col = etid; col < S; col += LM_EPI_THREADS) {
         float2 c = cst[col];
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq) {
@@ -307,7 +408,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     }
     if (ok) {
       const int nrec = gridDim.x;
-      for (int col = etid; col < S; col += 128) {
+      for (int col = etid; col < S; col += LM_EPI_THREADS) {
         a.rec_stats[(int64_t)col * nrec + blockIdx.x] = cst[col];
         if (a.mode == 1 && col % n1 != 0) a.rec_arg[(int64_t)col * nrec + blockIdx.x] = carg[col];
       }

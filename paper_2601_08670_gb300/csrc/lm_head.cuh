@@ -5,7 +5,8 @@
 
 namespace pced {
 
-constexpr int LM_THREADS = 192;  // warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-5 epilogue
+constexpr int LM_EPI_THREADS = 256;  // eight epilogue warps: two per TMEM lane quarter, each half of the columns
+constexpr int LM_THREADS = 64 + LM_EPI_THREADS;  // warp 0 TMA, warp 1 MMA + TMEM owner, warps 2-9 epilogue
 constexpr int LM_TILE_V = 128;   // vocabulary rows per tile (UMMA M)
 constexpr int LM_TILE_K = 64;    // hidden elements per stage (one 128-byte swizzle row)
 constexpr int LM_MAX_S = 512;
