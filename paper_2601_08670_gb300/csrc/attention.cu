@@ -34,6 +34,7 @@ struct AttCfg {
   static constexpr int KSTEPS = D / 16;
   static constexpr int MTILES = D / 16;
   static constexpr int OPAD = 9;                        // padded head stride of the merge scratch
+  static constexpr int OROW = D + 4;                    // padded row (one head of one warp) of the step kernel's partials
   static constexpr int OPT = ATT_MAX_G * D / ATT_CT;   // outputs of a piece per consumer thread (G <= 8)
   static constexpr int MERGE_FLOATS = 2 * ATT_CONSUMERS * ATT_MAX_G + ATT_CONSUMERS * D * OPAD + ATT_CONSUMERS + 8;
   static constexpr size_t BARS = (2 * STAGES + 2) * 8;
@@ -365,11 +366,8 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
           const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
           mbar_arrive_expect_tx(fb, C::STAGE_BYTES);
           const int32_t row = (int32_t)(slab_row + kt);
-#pragma unroll
-          for (int b = 0; b < C::BOXES; ++b) {
-            tma_load_2d(sk + b * C::BOX_BYTES, &kmap, fb, b * 64, row, pol);
-            tma_load_2d(sv + b * C::BOX_BYTES, &vmap, fb, b * 64, row, pol);
-          }
+          tma_load_3d(sk, &kmap, fb, 0, row, 0, pol);
+          tma_load_3d(sv, &vmap, fb, 0, row, 0, pol);
         }
       }
       if (!ok) {
@@ -610,8 +608,7 @@ struct StepSmem {
   uint32_t stages;      // K/V ring stages
   uint32_t bar;         // full[st] empty[st] qfull[2] qempty[2] pfull[2] pempty[2] msync
   uint32_t qbuf, qslot; // [2] hand-off slots: q words [8][D/2+4], K row, V row (bf16), x_l of the head group (fp32)
-  uint32_t pbuf, pslot; // [2] partial hand-off slots: ms[8][8], ls[8][8], os[8][D][opad]
-  uint32_t opad;
+  uint32_t pbuf, pslot; // [2] partial hand-off slots: ms[8][8], ls[8][8], os[8][G][D + 4]
   uint32_t misc;        // red[2][2] floats, flags
   uint32_t tables;      // pre[ATT_MAX_S+1] int64, lens[ATT_MAX_S] int32, apnd[ATT_MAX_S] u8
   uint32_t total;       // bytes to request, alignment slack included
@@ -619,9 +616,8 @@ struct StepSmem {
 __host__ __device__ inline StepSmem step_smem(int D, int G) {
   StepSmem L;
   const uint32_t stage_bytes = 2u * (uint32_t)(D / 64) * (ATT_BLOCK_N * 128u);
-  L.opad = (G % 2 == 0) ? (uint32_t)G + 1u : (uint32_t)G;
   L.qslot = 8u * (uint32_t)(D / 2 + 4) * 4u + 4u * (uint32_t)D + 4u * (uint32_t)(G * D);
-  L.pslot = 2u * ATT_CONSUMERS * ATT_MAX_G * 4u + (uint32_t)ATT_CONSUMERS * D * L.opad * 4u;
+  L.pslot = 2u * ATT_CONSUMERS * ATT_MAX_G * 4u + (uint32_t)ATT_CONSUMERS * G * (D + 4) * 4u;
   const uint32_t tables = (ATT_MAX_S + 1) * 8u + ATT_MAX_S * 4u + ATT_MAX_S;
   const uint32_t max_st = D == 128 ? 5u : 7u;
   for (L.stages = max_st; L.stages >= 2u; --L.stages) {
@@ -751,17 +747,13 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
       cursor_begin(ld, a, pre, lens, T, cb, ce, D);
       cursor_begin(pf, a, pre, lens, T, cb, ce, D);
       for (int i = 0; i < a.pf_tiles && pf.ok; ++i) {
-#pragma unroll
-        for (int b = 0; b < C::BOXES; ++b) {
-          tma_prefetch_l2_2d(&kmap, b * 64, (int32_t)(pf.row0 + pf.kt));
-          tma_prefetch_l2_2d(&vmap, b * 64, (int32_t)(pf.row0 + pf.kt));
-        }
+        tma_prefetch_l2_3d(&kmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
+        tma_prefetch_l2_3d(&vmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
         cursor_next(pf, a, pre, lens, T, cb, ce, D);
       }
-      uint32_t it = 0;
+      uint32_t it = 0, st = 0, ph = 0;
       bool ok = true;
       while (ld.ok) {
-        const uint32_t st = it % NST, ph = (it / NST) & 1u;
         if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
           ok = false;
           break;
@@ -770,19 +762,17 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
         mbar_arrive_expect_tx(fb, C::STAGE_BYTES);
         const int32_t row = (int32_t)(ld.row0 + ld.kt);
-#pragma unroll
-        for (int b = 0; b < C::BOXES; ++b) {
-          tma_load_2d(sk + b * C::BOX_BYTES, &kmap, fb, b * 64, row, pol);
-          tma_load_2d(sv + b * C::BOX_BYTES, &vmap, fb, b * 64, row, pol);
-        }
+        tma_load_3d(sk, &kmap, fb, 0, row, 0, pol);
+        tma_load_3d(sv, &vmap, fb, 0, row, 0, pol);
         ++it;
+        if (++st == NST) {
+          st = 0;
+          ph ^= 1u;
+        }
         cursor_next(ld, a, pre, lens, T, cb, ce, D);
         if (pf.ok) {
-#pragma unroll
-          for (int b = 0; b < C::BOXES; ++b) {
-            tma_prefetch_l2_2d(&kmap, b * 64, (int32_t)(pf.row0 + pf.kt));
-            tma_prefetch_l2_2d(&vmap, b * 64, (int32_t)(pf.row0 + pf.kt));
-          }
+          tma_prefetch_l2_3d(&kmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
+          tma_prefetch_l2_3d(&vmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
           cursor_next(pf, a, pre, lens, T, cb, ce, D);
         }
       }
@@ -926,7 +916,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   const int g = lane >> 2, tq = lane & 3;
   const int kb = 16 * wl;
   const bool hv = g < G;
-  uint32_t it = 0, p = 0;
+  uint32_t it = 0, p = 0, cst = 0, cuse = 0;  // tile counter; its stage and use count (it % NST, it / NST)
   bool ok = true;
   for (int l = 0; l < a.L && ok; ++l) {
     for (int64_t pp = cb; pp < ce && ok;) {
@@ -950,9 +940,9 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
 
       WarpAcc<D> A;
       acc_reset(A);
-      for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
+      for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it, cst = cst + 1 == NST ? (++cuse, 0u) : cst + 1) {
         if ((int)(it & 1u) != wg) continue;
-        const uint32_t use = it / NST, st = it % NST, ph = use & 1u;
+        const uint32_t use = cuse, st = cst, ph = use & 1u;
         if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status)) {
           ok = false;
           break;
@@ -995,7 +985,8 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_qempty + 8 * slot);
       }
-      // combine the eight warps' partials through a double-buffered slot
+      // combine the eight warps' partials through a double-buffered slot;
+      // afterwards thread tid < G*D/4 owns outputs idx0..idx0+3 (head hh)
       if (u > 0 && !mbar_wait(bar_pempty + 8 * slot, (u - 1u) & 1u, a.status)) {
         ok = false;
         break;
@@ -1006,27 +997,29 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         l0 += __shfl_xor_sync(0xffffffffu, l0, off);
         l1 += __shfl_xor_sync(0xffffffffu, l1, off);
       }
-      float* ms = reinterpret_cast<float*>(gbase + SL.pbuf + slot * SL.pslot);
-      float* ls = ms + ATT_CONSUMERS * ATT_MAX_G;
-      float* os = ls + ATT_CONSUMERS * ATT_MAX_G;
+      float* ms = reinterpret_cast<float*>(gbase + SL.pbuf + slot * SL.pslot);  // [ATT_MAX_G][8 warps]
+      float* ls = ms + ATT_MAX_G * ATT_CONSUMERS;                                // [ATT_MAX_G][8 warps]
+      float* os = ls + ATT_MAX_G * ATT_CONSUMERS;                                // [8 warps][G][D + 4]
       if (g == 0) {
-        ms[warp * ATT_MAX_G + 2 * tq] = A.m0;
-        ms[warp * ATT_MAX_G + 2 * tq + 1] = A.m1;
-        ls[warp * ATT_MAX_G + 2 * tq] = l0;
-        ls[warp * ATT_MAX_G + 2 * tq + 1] = l1;
+        ms[(2 * tq) * ATT_CONSUMERS + warp] = A.m0;
+        ms[(2 * tq + 1) * ATT_CONSUMERS + warp] = A.m1;
+        ls[(2 * tq) * ATT_CONSUMERS + warp] = l0;
+        ls[(2 * tq + 1) * ATT_CONSUMERS + warp] = l1;
       }
-      float* ow = os + warp * D * SL.opad;
-      const bool h0 = 2 * tq < G, h1 = 2 * tq + 1 < G;
+      {
+        float* ow = os + warp * G * C::OROW;
+        const bool h0 = 2 * tq < G, h1 = 2 * tq + 1 < G;
 #pragma unroll
-      for (int i = 0; i < C::MTILES; ++i) {
-        const int d0 = 16 * i + g, d1 = d0 + 8;
-        if (h0) {
-          ow[d0 * SL.opad + 2 * tq] = A.o[i][0];
-          ow[d1 * SL.opad + 2 * tq] = A.o[i][2];
-        }
-        if (h1) {
-          ow[d0 * SL.opad + 2 * tq + 1] = A.o[i][1];
-          ow[d1 * SL.opad + 2 * tq + 1] = A.o[i][3];
+        for (int i = 0; i < C::MTILES; ++i) {
+          const int d0 = 16 * i + g, d1 = d0 + 8;
+          if (h0) {
+            ow[(2 * tq) * C::OROW + d0] = A.o[i][0];
+            ow[(2 * tq) * C::OROW + d1] = A.o[i][2];
+          }
+          if (h1) {
+            ow[(2 * tq + 1) * C::OROW + d0] = A.o[i][1];
+            ow[(2 * tq + 1) * C::OROW + d1] = A.o[i][3];
+          }
         }
       }
       __syncwarp();
@@ -1036,43 +1029,46 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         break;
       }
       const uint32_t tag = step_tag(epoch, l);
-      float mx[C::OPT], lsum[C::OPT], acc[C::OPT];
+      const bool own = tid < GD / 4;
+      const int hh = own ? tid / (D / 4) : 0, idx0 = own ? 4 * tid : 0;
+      float mx = -INFINITY, lsum = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
+      if (own) {
+        float mw[ATT_CONSUMERS], lw[ATT_CONSUMERS];
+        const float4* m4 = reinterpret_cast<const float4*>(ms + hh * ATT_CONSUMERS);
+        const float4* l4 = reinterpret_cast<const float4*>(ls + hh * ATT_CONSUMERS);
+        *reinterpret_cast<float4*>(mw) = m4[0];
+        *reinterpret_cast<float4*>(mw + 4) = m4[1];
+        *reinterpret_cast<float4*>(lw) = l4[0];
+        *reinterpret_cast<float4*>(lw + 4) = l4[1];
+        float M = mw[0];
 #pragma unroll
-      for (int k = 0; k < C::OPT; ++k) {
-        const int idx = tid + ATT_CT * k;
-        mx[k] = -INFINITY;
-        lsum[k] = acc[k] = 0.f;
-        if (idx >= GD) continue;
-        const int hh = idx / D, dd = idx - hh * D;
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < ATT_CONSUMERS; ++w) M = fmaxf(M, ms[w * ATT_MAX_G + hh]);
-        float ac = 0.f, lv = 0.f;
+        for (int w = 1; w < ATT_CONSUMERS; ++w) M = fmaxf(M, mw[w]);
+        const float* oc = os + hh * C::OROW + (idx0 - hh * D);
 #pragma unroll
         for (int w = 0; w < ATT_CONSUMERS; ++w) {
-          const float mw = ms[w * ATT_MAX_G + hh];
-          if (mw == -INFINITY) continue;
-          const float e = exp2f(mw - M);
-          ac += os[(w * D + dd) * SL.opad + hh] * e;
-          lv += ls[w * ATT_MAX_G + hh] * e;
+          if (mw[w] == -INFINITY) continue;  // a warp without live keys in this piece
+          const float e = exp2f(mw[w] - M);
+          const float4 o4 = *reinterpret_cast<const float4*>(oc + w * G * C::OROW);
+          acc[0] += o4.x * e;
+          acc[1] += o4.y * e;
+          acc[2] += o4.z * e;
+          acc[3] += o4.w * e;
+          lsum += lw[w] * e;
         }
-        mx[k] = M;
-        lsum[k] = lv;
-        acc[k] = ac;
+        mx = M;
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_pempty + 8 * slot);
       if (!merges) {
         // the segment continues in an earlier CTA: publish this CTA's record
         const int64_t rs = (int64_t)blockIdx.x + seg;
+        if (own) {
+          uint64_t* ro = a.rec_o + rs * GD + idx0;
 #pragma unroll
-        for (int k = 0; k < C::OPT; ++k) {
-          const int idx = tid + ATT_CT * k;
-          if (idx >= GD) continue;
-          st_tagged(a.rec_o + rs * GD + idx, acc[k], tag);
-          if (idx % D == 0) {
-            st_tagged(a.rec_ml + (rs * G + idx / D) * 2, mx[k], tag);
-            st_tagged(a.rec_ml + (rs * G + idx / D) * 2 + 1, lsum[k], tag);
+          for (int j = 0; j < 4; ++j) st_tagged(ro + j, acc[j], tag);
+          if (idx0 % D == 0) {
+            st_tagged(a.rec_ml + (rs * G + hh) * 2, mx, tag);
+            st_tagged(a.rec_ml + (rs * G + hh) * 2 + 1, lsum, tag);
           }
         }
         continue;
@@ -1081,27 +1077,31 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
       // time, one round trip when they are there)
       constexpr int RB = 2;
       for (int64_t c = c0 + 1; c <= c1 && ok; c += RB) {
-        float mv[C::OPT][RB], lv[C::OPT][RB], ov[C::OPT][RB];
+        float mv[RB], lv[RB], ov[RB][4];
         uint64_t t0 = 0;
         while (true) {
           bool good = true;
 #pragma unroll
-          for (int k = 0; k < C::OPT; ++k) {
-            const int idx = tid + ATT_CT * k, hh = idx / D;
+          for (int q = 0; q < RB; ++q) {
+            mv[q] = -INFINITY;
+            lv[q] = 0.f;
 #pragma unroll
-            for (int q = 0; q < RB; ++q) {
-              mv[k][q] = -INFINITY;
-              lv[k][q] = ov[k][q] = 0.f;
-              if (idx >= GD || c + q > c1) continue;
-              const int64_t rs = c + q + seg;
-              const uint64_t wm = ld_tagged(a.rec_ml + (rs * G + hh) * 2);
-              const uint64_t wl = ld_tagged(a.rec_ml + (rs * G + hh) * 2 + 1);
-              const uint64_t wo = ld_tagged(a.rec_o + rs * GD + idx);
-              good &= tv_ok(wm, tag) && tv_ok(wl, tag) && tv_ok(wo, tag);
-              mv[k][q] = tv_value(wm);
-              lv[k][q] = tv_value(wl);
-              ov[k][q] = tv_value(wo);
+            for (int j = 0; j < 4; ++j) ov[q][j] = 0.f;
+            if (!own || c + q > c1) continue;
+            const int64_t rs = c + q + seg;
+            const uint64_t wm = ld_tagged(a.rec_ml + (rs * G + hh) * 2);
+            const uint64_t wl = ld_tagged(a.rec_ml + (rs * G + hh) * 2 + 1);
+            uint64_t wo[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) wo[j] = ld_tagged(a.rec_o + rs * GD + idx0 + j);
+            good &= tv_ok(wm, tag) && tv_ok(wl, tag);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              good &= tv_ok(wo[j], tag);
+              ov[q][j] = tv_value(wo[j]);
             }
+            mv[q] = tv_value(wm);
+            lv[q] = tv_value(wl);
           }
           if (__all_sync(0xffffffffu, good)) break;
           if (!poll_again(t0, a.status)) {
@@ -1110,16 +1110,15 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           }
         }
 #pragma unroll
-        for (int k = 0; k < C::OPT; ++k)
+        for (int q = 0; q < RB; ++q) {
+          if (mv[q] == -INFINITY) continue;
+          const float Mn = fmaxf(mx, mv[q]);
+          const float f = mx == -INFINITY ? 0.f : exp2f(mx - Mn), e = exp2f(mv[q] - Mn);
 #pragma unroll
-          for (int q = 0; q < RB; ++q) {
-            if (mv[k][q] == -INFINITY) continue;
-            const float Mn = fmaxf(mx[k], mv[k][q]);
-            const float f = mx[k] == -INFINITY ? 0.f : exp2f(mx[k] - Mn), e = exp2f(mv[k][q] - Mn);
-            acc[k] = acc[k] * f + ov[k][q] * e;
-            lsum[k] = lsum[k] * f + lv[k][q] * e;
-            mx[k] = Mn;
-          }
+          for (int j = 0; j < 4; ++j) acc[j] = acc[j] * f + ov[q][j] * e;
+          lsum = lsum * f + lv[q] * e;
+          mx = Mn;
+        }
       }
       if (!ok) break;
       // x_{l+1} = x_l + o for head group h (x_l from the input warp's slot)
@@ -1127,16 +1126,17 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
       const uint32_t ntag = step_tag(epoch, l + 1);
       const float* xr = reinterpret_cast<const float*>(qw + 8 * QW + D);
       uint64_t* xn = a.resid + ((int64_t)nx * S + pc.s) * d + (int64_t)pc.h * GD;
-      float xv[C::OPT];
+      float xv[4] = {0.f, 0.f, 0.f, 0.f};
       float ss = 0.f;
+      if (own) {
+        const float4 x4 = *reinterpret_cast<const float4*>(xr + idx0);
+        const float xo[4] = {x4.x, x4.y, x4.z, x4.w};
 #pragma unroll
-      for (int k = 0; k < C::OPT; ++k) {
-        const int idx = tid + ATT_CT * k;
-        xv[k] = 0.f;
-        if (idx >= GD) continue;
-        xv[k] = xr[idx] + (lsum[k] > 0.f ? acc[k] / lsum[k] : 0.f);
-        st_tagged(xn + idx, xv[k], ntag);
-        ss += xv[k] * xv[k];
+        for (int j = 0; j < 4; ++j) {
+          xv[j] = xo[j] + (lsum > 0.f ? acc[j] / lsum : 0.f);
+          st_tagged(xn + idx0 + j, xv[j], ntag);
+          ss += xv[j] * xv[j];
+        }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_qempty + 8 * slot);
@@ -1150,15 +1150,15 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         ok = false;
         break;
       }
-      __nv_bfloat16* hs = a.hidden + (int64_t)pc.s * d + (int64_t)pc.h * GD;
-      __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)pc.s * d + (int64_t)pc.h * GD : nullptr;
+      if (own) {
+        __nv_bfloat16* hs = a.hidden + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0;
+        __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0 : nullptr;
 #pragma unroll
-      for (int k = 0; k < C::OPT; ++k) {
-        const int idx = tid + ATT_CT * k;
-        if (idx >= GD) continue;
-        const __nv_bfloat16 hv2 = __float2bfloat16_rn(xv[k] * inv);
-        hs[idx] = hv2;
-        if (hc) hc[idx] = hv2;
+        for (int j = 0; j < 4; ++j) {
+          const __nv_bfloat16 hv2 = __float2bfloat16_rn(xv[j] * inv);
+          hs[j] = hv2;
+          if (hc) hc[j] = hv2;
+        }
       }
     }
   }
@@ -1310,9 +1310,9 @@ extern "C" pced_status pced_decode_attention(const void* q, const void* k_cache,
 
   CUtensorMap kmap, vmap;
   const uint64_t rows = (uint64_t)(cache_elems / D);
-  pced_status st = make_tmap_2d(&kmap, k_cache, rows, (uint64_t)D, ATT_BLOCK_N, 64, true);
+  pced_status st = make_tmap_kv(&kmap, k_cache, rows, (uint32_t)D, ATT_BLOCK_N);
   if (st != PCED_OK) return st;
-  st = make_tmap_2d(&vmap, v_cache, rows, (uint64_t)D, ATT_BLOCK_N, 64, true);
+  st = make_tmap_kv(&vmap, v_cache, rows, (uint32_t)D, ATT_BLOCK_N);
   if (st != PCED_OK) return st;
 
   const int32_t G = Hq / Hkv;

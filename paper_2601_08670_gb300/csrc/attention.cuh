@@ -72,8 +72,10 @@ cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream);
 // Roles inside a CTA (warp-specialised, hand-offs through double-buffered
 // shared-memory slots guarded by mbarriers): a producer warp (TMA), an input
 // warp that prepares each piece's query bf16(x_l * inv_rms(x_l)) and the row
-// appended this step, eight consumer warps that only run the attention math,
-// and a two-warp merge group that combines the consumers' partials.
+// appended this step, and eight consumer warps that run the attention math and
+// then combine their partials through shared memory (each thread ends up
+// owning four consecutive outputs of one head).  K and V tiles arrive as one
+// 3-D tensor copy each.
 //
 // Layer dependency: a segment split over CTAs c0..c1 is completed by c0 (for
 // which it is the last piece of the layer); c0+1..c1 publish their records

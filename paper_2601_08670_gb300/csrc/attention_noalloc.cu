@@ -109,9 +109,9 @@ extern "C" pced_status pced_decode_attention_noalloc(const void* q, const void* 
 
   CUtensorMap kmap, vmap;
   const uint64_t rows = (uint64_t)(cache_elems / D);
-  st = make_tmap_2d(&kmap, k_cache, rows, (uint64_t)D, ATT_BLOCK_N, 64, true);
+  st = make_tmap_kv(&kmap, k_cache, rows, (uint32_t)D, ATT_BLOCK_N);
   if (st != PCED_OK) return st;
-  st = make_tmap_2d(&vmap, v_cache, rows, (uint64_t)D, ATT_BLOCK_N, 64, true);
+  st = make_tmap_kv(&vmap, v_cache, rows, (uint32_t)D, ATT_BLOCK_N);
   if (st != PCED_OK) return st;
 
   // Nothing here has to start at zero: every record and plan entry the combine

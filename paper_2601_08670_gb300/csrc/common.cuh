@@ -59,9 +59,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 // Wait for the phase with the given parity to complete; gives up after
-// kWaitLimitNs, flags PCED_DEV_TIMEOUT and returns false.
-static __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status) {
-  if (mbar_try_wait(bar, parity)) return true;
+// kWaitLimitNs, flags PCED_DEV_TIMEOUT and returns false.  The first test is
+// inlined: on the hot paths the phase has usually completed already.
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int* status) {
   const uint64_t t0 = globaltimer_ns();
   while (true) {
 #pragma unroll 1
@@ -72,6 +72,9 @@ static __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int
       return false;
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, status);
 }
 
 // Barrier among a subset of a CTA's threads built on an mbarrier initialised
@@ -161,6 +164,21 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, uint
       " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
       "l"(tmap), "r"(bar), "r"(x), "r"(y), "l"(policy)
       : "memory");
+}
+
+// 3-D tiled copy (the K/V tile maps: coordinates {0, row, 0})
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, uint32_t bar, int32_t x, int32_t y,
+                                            int32_t z, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(dst),
+      "l"(tmap), "r"(bar), "r"(x), "r"(y), "r"(z), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_l2_3d(const void* tmap, int32_t x, int32_t y, int32_t z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(tmap), "r"(x), "r"(y),
+               "r"(z)
+               : "memory");
 }
 
 // L2 prefetch of one tensor-map box (no shared memory, no completion tracking)
@@ -328,6 +346,7 @@ int num_sms();
 // 128-byte swizzle (box_cols * 2 must be 128).
 pced_status make_tmap_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
                          uint32_t box_cols, bool l2_promote_256);
+pced_status make_tmap_kv(CUtensorMap* map, const void* base, uint64_t rows, uint32_t D, uint32_t box_rows);
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 

@@ -88,6 +88,28 @@ pced_status make_tmap_2d(CUtensorMap* map, const void* base, uint64_t rows, uint
   return PCED_OK;
 }
 
+// Tensor map over a cache of `rows` rows of D bf16 (D = 64 or 128) whose box
+// is a whole 64-row K or V tile in one copy: dimension 0 is 64 elements
+// (128 bytes, the swizzle span), dimension 1 the rows, dimension 2 the D/64
+// column blocks of a row.  Shared memory receives [D/64][box_rows][128 B] with
+// the 128-byte swizzle, the layout of D/64 separate 64-column boxes.
+pced_status make_tmap_kv(CUtensorMap* map, const void* base, uint64_t rows, uint32_t D, uint32_t box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return fail(PCED_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  if ((D != 64 && D != 128) || box_rows < 1 || box_rows > 256 || rows < 1 || rows > (1ull << 32) ||
+      ((uintptr_t)base & 15u))
+    return fail(PCED_ERR_INVALID_ARG, "kv tensor map: unsupported geometry");
+  const cuuint64_t dims[3] = {64, rows, D / 64};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, 128};
+  const cuuint32_t box[3] = {64, box_rows, D / 64};
+  const cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(PCED_ERR_CUDA, "cuTensorMapEncodeTiled (kv tile) failed (%d)", (int)r);
+  return PCED_OK;
+}
+
 }  // namespace pced_host
 
 extern "C" const char* pced_status_string(int32_t status) {

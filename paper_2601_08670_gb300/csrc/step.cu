@@ -102,8 +102,8 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   const StepLayout W = step_layout(&dm, p->workspace);
   CUtensorMap kmap, vmap, wmap, hmap;
   const uint64_t rows = (uint64_t)dm.L * (uint64_t)(p->layer_elems / dm.D);
-  pced_status st = make_tmap_2d(&kmap, p->k_cache, rows, (uint64_t)dm.D, ATT_BLOCK_N, 64, true);
-  if (st == PCED_OK) st = make_tmap_2d(&vmap, p->v_cache, rows, (uint64_t)dm.D, ATT_BLOCK_N, 64, true);
+  pced_status st = make_tmap_kv(&kmap, p->k_cache, rows, (uint32_t)dm.D, ATT_BLOCK_N);
+  if (st == PCED_OK) st = make_tmap_kv(&vmap, p->v_cache, rows, (uint32_t)dm.D, ATT_BLOCK_N);
   if (st == PCED_OK) st = make_tmap_2d(&wmap, p->w_unembed, (uint64_t)dm.V, (uint64_t)d, LM_TILE_V, LM_TILE_K, true);
   if (st == PCED_OK) st = make_tmap_2d(&hmap, W.h, (uint64_t)S, (uint64_t)d, (uint32_t)g.chunk_n, LM_TILE_K, false);
   if (st != PCED_OK) return st;
