@@ -75,16 +75,17 @@ struct Piece {
   int64_t adv;           // positions the piece spans
 };
 
-// Piece that starts at global position p and ends at the next segment
-// boundary or at `end`.  Segment (h, s) spans positions
-// [h*T + pre[s], h*T + pre[s+1]); its first lens[s] positions are keys, the
+// Piece that starts at position p of the position space of sequences
+// [s_lo, s_hi) and ends at the next segment boundary or at `end`.  Segment
+// (h, s) spans positions [h*T + pre[s] - pre[s_lo], h*T + pre[s+1] - pre[s_lo])
+// with T = pre[s_hi] - pre[s_lo]; its first lens[s] positions are keys, the
 // rest (if any) only weight the partition.
-__device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* lens, int32_t S, int64_t T, int64_t p,
-                                            int64_t end) {
+__device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* lens, int32_t s_lo, int32_t s_hi,
+                                            int64_t T, int64_t p, int64_t end) {
   Piece pc;
   pc.h = (int32_t)(p / T);
-  const int64_t r = p - (int64_t)pc.h * T;
-  int32_t lo = 0, hi = S - 1;
+  const int64_t r = p - (int64_t)pc.h * T + pre[s_lo];
+  int32_t lo = s_lo, hi = s_hi - 1;
   while (lo < hi) {
     const int32_t mid = (lo + hi + 1) >> 1;
     if (pre[mid] <= r) lo = mid;
@@ -92,7 +93,7 @@ __device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* l
   }
   pc.s = lo;
   const int64_t off = r - pre[lo];
-  const int64_t seg_end = (int64_t)pc.h * T + pre[lo + 1];
+  const int64_t seg_end = (int64_t)pc.h * T + pre[lo + 1] - pre[s_lo];
   const int64_t e = seg_end < end ? seg_end : end;
   pc.adv = e - p;
   const int64_t len = lens[lo];
@@ -353,7 +354,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int64_t p = r_begin; p < r_end && ok;) {
-        const Piece pc = find_piece(pre, lens, S, T, p, r_end);
+        const Piece pc = find_piece(pre, lens, 0, S, T, p, r_end);
         p += pc.adv;
         const int64_t slab_row = a.row_base + (a.kv_offset[pc.s] + (int64_t)pc.h * a.cap[pc.s] * D) / D;
         for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it) {
@@ -386,7 +387,7 @@ __global__ void __launch_bounds__(ATT_THREADS, 1)
   uint32_t it = 0, cph = 0;
   bool ok = true;
   for (int64_t p = r_begin; p < r_end && ok;) {
-    const Piece pc = find_piece(pre, lens, S, T, p, r_end);
+    const Piece pc = find_piece(pre, lens, 0, S, T, p, r_end);
     p += pc.adv;
     uint32_t qf[C::KSTEPS][2];
     {
@@ -536,25 +537,67 @@ __device__ __forceinline__ bool poll_again(uint64_t& t0, int* status) {
   return true;
 }
 
-// Tile cursor over a CTA's range through all layers (the producer's order).
+// Sequence groups of the step kernel and this CTA's range in each (shared
+// memory, written once by thread 0).
+struct GroupPlan {
+  int32_t n;
+  int32_t s_lo[ATT_MAX_GROUPS + 1];  // group g holds sequences [s_lo[g], s_lo[g+1])
+  int64_t T[ATT_MAX_GROUPS];         // positions per kv-head
+  int64_t P[ATT_MAX_GROUPS];         // positions per CTA
+  int64_t cb[ATT_MAX_GROUPS], ce[ATT_MAX_GROUPS];
+};
+
+// Cut the sequences into min(want, S) contiguous groups of about equal weight
+// (pre: prefix of the extents) and partition each over the grid.
+__device__ __forceinline__ void plan_groups(GroupPlan& gp, const int64_t* pre, int32_t S, int32_t Hkv, int want,
+                                            int64_t grid, int64_t cta) {
+  int ng = want < 1 ? 1 : (want > ATT_MAX_GROUPS ? ATT_MAX_GROUPS : want);
+  if (ng > S) ng = S;
+  const int64_t T = pre[S];
+  gp.s_lo[0] = 0;
+  for (int g = 1; g < ng; ++g) {
+    const int64_t target = T * g / ng;
+    int32_t s = gp.s_lo[g - 1] + 1;
+    while (s < S - (ng - g) && pre[s] < target) ++s;
+    gp.s_lo[g] = s;
+  }
+  gp.s_lo[ng] = S;
+  for (int g = 0; g < ng; ++g) {
+    const int64_t Tg = pre[gp.s_lo[g + 1]] - pre[gp.s_lo[g]];
+    const int64_t tot = (int64_t)Hkv * Tg;
+    const int64_t Pg = (tot + grid - 1) / grid;
+    gp.T[g] = Tg;
+    gp.P[g] = Pg;
+    gp.cb[g] = min(tot, cta * Pg);
+    gp.ce[g] = min(tot, gp.cb[g] + Pg);
+  }
+  gp.n = ng;
+}
+
+// Tile cursor over a CTA's ranges through all layers and groups (the
+// producer's order: layer by layer, group by group).
 struct TileCursor {
-  int32_t l, kt;
+  int32_t l, g, kt;
   int64_t p, row0;  // row0: tensor-map row of key 0 of the current piece
   Piece pc;
   bool ok;
 };
 
 __device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
-                                            const int32_t* lens, int64_t T, int64_t cb, int64_t ce, int D) {
+                                            const int32_t* lens, const GroupPlan& gp, int D) {
   while (true) {
-    if (c.p >= ce) {
-      if (++c.l >= a.L) {
-        c.ok = false;
-        return;
+    if (c.p >= gp.ce[c.g]) {
+      if (++c.g >= gp.n) {
+        c.g = 0;
+        if (++c.l >= a.L) {
+          c.ok = false;
+          return;
+        }
       }
-      c.p = cb;
+      c.p = gp.cb[c.g];
+      continue;
     }
-    c.pc = find_piece(pre, lens, a.S, T, c.p, ce);
+    c.pc = find_piece(pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g]);
     if (c.pc.k0 < c.pc.k1) {
       c.kt = c.pc.k0;
       c.row0 = (int64_t)c.l * a.rows_per_layer + (a.kv_offset[c.pc.s] + (int64_t)c.pc.h * a.cap[c.pc.s] * D) / D;
@@ -564,18 +607,19 @@ __device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a,
   }
 }
 __device__ __forceinline__ void cursor_begin(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
-                                             const int32_t* lens, int64_t T, int64_t cb, int64_t ce, int D) {
+                                             const int32_t* lens, const GroupPlan& gp, int D) {
   c.l = 0;
-  c.p = cb;
-  c.ok = cb < ce && a.L > 0;
-  if (c.ok) cursor_seek(c, a, pre, lens, T, cb, ce, D);
+  c.g = 0;
+  c.p = gp.cb[0];
+  c.ok = a.L > 0;
+  if (c.ok) cursor_seek(c, a, pre, lens, gp, D);
 }
 __device__ __forceinline__ void cursor_next(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
-                                            const int32_t* lens, int64_t T, int64_t cb, int64_t ce, int D) {
+                                            const int32_t* lens, const GroupPlan& gp, int D) {
   c.kt += ATT_BLOCK_N;
   if (c.kt < c.pc.k1) return;
   c.p += c.pc.adv;
-  cursor_seek(c, a, pre, lens, T, cb, ce, D);
+  cursor_seek(c, a, pre, lens, gp, D);
 }
 
 // 1/rms of x_l[s] from its Hkv per-group sums of squares (waits for all of
@@ -610,7 +654,7 @@ struct StepSmem {
   uint32_t qbuf, qslot; // [2] hand-off slots: q words [8][D/2+4], K row, V row (bf16), x_l of the head group (fp32)
   uint32_t pbuf, pslot; // [2] partial hand-off slots: ms[8][8], ls[8][8], os[8][G][D + 4]
   uint32_t misc;        // red[2][2] floats, flags
-  uint32_t tables;      // pre[ATT_MAX_S+1] int64, lens[ATT_MAX_S] int32, apnd[ATT_MAX_S] u8
+  uint32_t tables;      // pre[ATT_MAX_S+1] int64, GroupPlan, lens[ATT_MAX_S] int32, apnd[ATT_MAX_S] u8
   uint32_t total;       // bytes to request, alignment slack included
 };
 __host__ __device__ inline StepSmem step_smem(int D, int G) {
@@ -618,7 +662,7 @@ __host__ __device__ inline StepSmem step_smem(int D, int G) {
   const uint32_t stage_bytes = 2u * (uint32_t)(D / 64) * (ATT_BLOCK_N * 128u);
   L.qslot = 8u * (uint32_t)(D / 2 + 4) * 4u + 4u * (uint32_t)D + 4u * (uint32_t)(G * D);
   L.pslot = 2u * ATT_CONSUMERS * ATT_MAX_G * 4u + (uint32_t)ATT_CONSUMERS * G * (D + 4) * 4u;
-  const uint32_t tables = (ATT_MAX_S + 1) * 8u + ATT_MAX_S * 4u + ATT_MAX_S;
+  const uint32_t tables = (ATT_MAX_S + 1) * 8u + (uint32_t)((sizeof(GroupPlan) + 7) & ~(size_t)7) + ATT_MAX_S * 4u + ATT_MAX_S;
   const uint32_t max_st = D == 128 ? 5u : 7u;
   for (L.stages = max_st; L.stages >= 2u; --L.stages) {
     L.bar = L.stages * stage_bytes;
@@ -684,7 +728,8 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   float* red = reinterpret_cast<float*>(gbase + SL.misc);  // [2 slots][2 merge warps]
   int* flag = reinterpret_cast<int*>(gbase + SL.misc + 32);
   int64_t* pre = reinterpret_cast<int64_t*>(gbase + SL.tables);
-  int32_t* lens = reinterpret_cast<int32_t*>(pre + ATT_MAX_S + 1);
+  GroupPlan& gp = *reinterpret_cast<GroupPlan*>(pre + ATT_MAX_S + 1);
+  int32_t* lens = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(&gp) + ((sizeof(GroupPlan) + 7) & ~(size_t)7));
   uint8_t* apnd = reinterpret_cast<uint8_t*>(lens + ATT_MAX_S);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -732,10 +777,8 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   __syncthreads();
   if (warp == 0) prefix_extents(lens, S, a.seg_cost, pre, lane);
   __syncthreads();
-  const int64_t T = pre[S];
-  const int64_t total = (int64_t)Hkv * T;
-  const int64_t P = (total + gridDim.x - 1) / gridDim.x;
-  const int64_t cb = min(total, (int64_t)blockIdx.x * P), ce = min(total, cb + P);
+  if (tid == 0) plan_groups(gp, pre, S, Hkv, a.groups, gridDim.x, blockIdx.x);
+  __syncthreads();
 
   if (warp == STEP_PRODUCER) {
     // ------------------------------------------------------------ producer
@@ -744,12 +787,12 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       TileCursor ld, pf;
-      cursor_begin(ld, a, pre, lens, T, cb, ce, D);
-      cursor_begin(pf, a, pre, lens, T, cb, ce, D);
+      cursor_begin(ld, a, pre, lens, gp, D);
+      cursor_begin(pf, a, pre, lens, gp, D);
       for (int i = 0; i < a.pf_tiles && pf.ok; ++i) {
         tma_prefetch_l2_3d(&kmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
         tma_prefetch_l2_3d(&vmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
-        cursor_next(pf, a, pre, lens, T, cb, ce, D);
+        cursor_next(pf, a, pre, lens, gp, D);
       }
       uint32_t it = 0, st = 0, ph = 0;
       bool ok = true;
@@ -769,11 +812,11 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           st = 0;
           ph ^= 1u;
         }
-        cursor_next(ld, a, pre, lens, T, cb, ce, D);
+        cursor_next(ld, a, pre, lens, gp, D);
         if (pf.ok) {
           tma_prefetch_l2_3d(&kmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
           tma_prefetch_l2_3d(&vmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
-          cursor_next(pf, a, pre, lens, T, cb, ce, D);
+          cursor_next(pf, a, pre, lens, gp, D);
         }
       }
       if (!ok) {
@@ -796,8 +839,9 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     for (int l = 0; l < a.L && ok; ++l) {
       const int par = l & 1;
       const uint32_t tag = step_tag(epoch, l);
-      for (int64_t pp = cb; pp < ce && ok;) {
-        const Piece pc = find_piece(pre, lens, S, T, pp, ce);
+      for (int gi = 0; gi < gp.n && ok; ++gi)
+      for (int64_t pp = gp.cb[gi]; pp < gp.ce[gi] && ok;) {
+        const Piece pc = find_piece(pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi]);
         pp += pc.adv;
         if (pc.k0 == pc.k1) continue;
         const uint32_t slot = p & 1u, u = p >> 1;
@@ -918,9 +962,13 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   const bool hv = g < G;
   uint32_t it = 0, p = 0, cst = 0, cuse = 0;  // tile counter; its stage and use count (it % NST, it / NST)
   bool ok = true;
-  for (int l = 0; l < a.L && ok; ++l) {
-    for (int64_t pp = cb; pp < ce && ok;) {
-      const Piece pc = find_piece(pre, lens, S, T, pp, ce);
+  for (int l = 0; l < a.L && ok; ++l)
+  for (int gi = 0; gi < gp.n && ok; ++gi) {
+    const int32_t g_lo = gp.s_lo[gi];
+    const int64_t gT = gp.T[gi], gP = gp.P[gi], gce = gp.ce[gi];
+    const int64_t rbase = (int64_t)gi * ((int64_t)gridDim.x + (int64_t)S * Hkv);  // this group's record slots
+    for (int64_t pp = gp.cb[gi]; pp < gce && ok;) {
+      const Piece pc = find_piece(pre, lens, g_lo, gp.s_lo[gi + 1], gT, pp, gce);
       pp += pc.adv;
       if (pc.k0 == pc.k1) continue;
       const uint32_t slot = p & 1u, u = p >> 1;
@@ -978,8 +1026,8 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
       }
       if (!ok) break;
       const int64_t seg = (int64_t)pc.h * S + pc.s;
-      const int64_t pa = (int64_t)pc.h * T + pre[pc.s];
-      const int64_t c0 = pa / P, c1 = (pa + lens[pc.s] - 1) / P;
+      const int64_t pa = (int64_t)pc.h * gT + pre[pc.s] - pre[g_lo];
+      const int64_t c0 = pa / gP, c1 = (pa + lens[pc.s] - 1) / gP;
       const bool merges = c0 == (int64_t)blockIdx.x;  // the segment's first CTA completes it
       if (!merges) {
         __syncwarp();
@@ -1061,7 +1109,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
       if (lane == 0) mbar_arrive(bar_pempty + 8 * slot);
       if (!merges) {
         // the segment continues in an earlier CTA: publish this CTA's record
-        const int64_t rs = (int64_t)blockIdx.x + seg;
+        const int64_t rs = rbase + (int64_t)blockIdx.x + seg;
         if (own) {
           uint64_t* ro = a.rec_o + rs * GD + idx0;
 #pragma unroll
@@ -1088,7 +1136,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
 #pragma unroll
             for (int j = 0; j < 4; ++j) ov[q][j] = 0.f;
             if (!own || c + q > c1) continue;
-            const int64_t rs = c + q + seg;
+            const int64_t rs = rbase + c + q + seg;
             const uint64_t wm = ld_tagged(a.rec_ml + (rs * G + hh) * 2);
             const uint64_t wl = ld_tagged(a.rec_ml + (rs * G + hh) * 2 + 1);
             uint64_t wo[4];
@@ -1198,7 +1246,7 @@ int att_grid(int64_t total_cap_keys) {
   return (int)(g < 1 ? 1 : g);
 }
 
-int64_t att_step_slots(int32_t S, int32_t Hkv) { return ATT_MAX_CTAS + (int64_t)S * Hkv; }
+int64_t att_step_slots(int32_t S, int32_t Hkv) { return ATT_MAX_GROUPS * (ATT_MAX_CTAS + (int64_t)S * Hkv); }
 
 static int env_int(const char* name, int dflt, int lo, int hi) {
   const char* e = getenv(name);
@@ -1206,8 +1254,9 @@ static int env_int(const char* name, int dflt, int lo, int hi) {
   const int v = atoi(e);
   return v < lo ? lo : (v > hi ? hi : v);
 }
-int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", D == 128 ? 256 : 512, 0, 1 << 20); }
+int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", 512, 0, 1 << 20); }
 int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 12, 0, 64); }
+int att_step_groups() { return env_int("PCED_ATT_GROUPS", 2, 1, ATT_MAX_GROUPS); }
 
 // cudaFuncSetAttribute once per kernel and device
 template <typename K>

@@ -14,6 +14,7 @@ constexpr int ATT_MAX_S = 1024;     // sequences per launch (prefix table lives 
 constexpr int ATT_MAX_G = 8;        // query heads per kv-head (mma N = 8)
 constexpr int ATT_MAX_CTAS = 1024;  // upper bound of the grid (sizes the partial-record pool)
 constexpr float ATT_RESCALE_SLACK = 8.f;  // log2 units the online-softmax reference may trail the max
+constexpr int ATT_MAX_GROUPS = 4;   // sequence groups of the step kernel
 
 // ---------------------------------------------------------------- one layer
 // Partition of all (kv-head, sequence, key) positions into equal contiguous
@@ -77,6 +78,13 @@ cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream);
 // owning four consecutive outputs of one head).  K and V tiles arrive as one
 // 3-D tensor copy each.
 //
+// Sequence groups: the sequences are cut into `groups` contiguous ranges of
+// about equal weight and every range is partitioned over all CTAs as above.
+// A CTA takes layer l of group 0, then of group 1, ..., then layer l+1 of
+// group 0: while one group's layer dependency resolves (merges, residual
+// update, next query), the CTAs stream the next group's keys.  Record slots of
+// group g start at g * (gridDim.x + S * Hkv).
+//
 // Layer dependency: a segment split over CTAs c0..c1 is completed by c0 (for
 // which it is the last piece of the layer); c0+1..c1 publish their records
 // for it.  The completing CTA adds the head group's attention output to the
@@ -93,6 +101,7 @@ struct StepAttArgs {
   float scale_log2, rms_eps;
   int32_t seg_cost;           // partition weight of a piece, in keys
   int32_t pf_tiles;           // tiles prefetched into L2 ahead of the shared-memory ring
+  int32_t groups;             // sequence groups (1..ATT_MAX_GROUPS), each partitioned over all CTAs
   const int64_t* kv_offset;   // [S]
   const int32_t* cap;         // [S]
   int32_t* seq_len;           // [S] +1 per launch for every sequence with room
@@ -117,6 +126,7 @@ int64_t att_step_slots(int32_t S, int32_t Hkv);
 // PCED_ATT_PF in the environment override the defaults)
 int att_step_seg_cost(int D);
 int att_step_pf_tiles();
+int att_step_groups();
 cudaError_t att_step_launch(int D, const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
                             cudaStream_t stream);
 

@@ -108,6 +108,14 @@ def test_llama8_graph_replay(cuda_ok):
     run_parity("llama8", 2, graph=True, min_ram_gb=8)
 
 
+@pytest.mark.parametrize("groups", [1, 3, 4])
+def test_llama8_sequence_groups(cuda_ok, monkeypatch, groups):
+    # the step kernel cuts the sequences into groups (default 2) that take
+    # turns per layer; every grouping must give the same results
+    monkeypatch.setenv("PCED_ATT_GROUPS", str(groups))
+    run_parity("llama8", 2, min_ram_gb=8)
+
+
 def test_qwen_flat_full_size(cuda_ok):
     run_parity("qwen_flat", 2, min_ram_gb=10)
 
