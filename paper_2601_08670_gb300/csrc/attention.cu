@@ -146,7 +146,13 @@ __device__ __forceinline__ void acc_reset(WarpAcc<D>& A) {
 // This warp's 16 keys [kb, kb+16) of the 64-key K/V tiles at sk / sv (TMA
 // 128-byte swizzle, D/64 boxes of 64 rows x 128 B); keys at or past nvalid
 // are masked.  qf: B operand of S^T = K Q^T (dims x heads).
-template <int D>
+//
+// P enters the P V product as bf16 hi + lo parts.  With PK (at most four
+// heads) both parts share one MMA: accumulator columns 0-3 take the hi parts
+// of heads 0-3 and columns 4-7 the lo parts of the same heads (the threads
+// owning columns 4-7, tq >= 2, mirror the scores of lane ^ 2), so o of head h
+// is column h plus column h + 4 (summed once per piece, see pack_fold).
+template <int D, bool PK = false>
 __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D / 16][2], uint32_t sk, uint32_t sv,
                                           int kb, int nvalid, float scale_log2, int lane) {
   using C = AttCfg<D>;
@@ -167,10 +173,20 @@ __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D 
     }
   }
   const bool v0 = kb + g < nvalid, v1 = kb + g + 8 < nvalid;
-  const float s0 = v0 ? ((sc4[0][0] + sc4[1][0]) + (sc4[2][0] + sc4[3][0])) * scale_log2 : -INFINITY;
-  const float s1 = v0 ? ((sc4[0][1] + sc4[1][1]) + (sc4[2][1] + sc4[3][1])) * scale_log2 : -INFINITY;
-  const float s2 = v1 ? ((sc4[0][2] + sc4[1][2]) + (sc4[2][2] + sc4[3][2])) * scale_log2 : -INFINITY;
-  const float s3 = v1 ? ((sc4[0][3] + sc4[1][3]) + (sc4[2][3] + sc4[3][3])) * scale_log2 : -INFINITY;
+  float s0 = v0 ? ((sc4[0][0] + sc4[1][0]) + (sc4[2][0] + sc4[3][0])) * scale_log2 : -INFINITY;
+  float s1 = v0 ? ((sc4[0][1] + sc4[1][1]) + (sc4[2][1] + sc4[3][1])) * scale_log2 : -INFINITY;
+  float s2 = v1 ? ((sc4[0][2] + sc4[1][2]) + (sc4[2][2] + sc4[3][2])) * scale_log2 : -INFINITY;
+  float s3 = v1 ? ((sc4[0][3] + sc4[1][3]) + (sc4[2][3] + sc4[3][3])) * scale_log2 : -INFINITY;
+  if (PK) {
+    const float r0 = __shfl_xor_sync(0xffffffffu, s0, 2), r1 = __shfl_xor_sync(0xffffffffu, s1, 2);
+    const float r2 = __shfl_xor_sync(0xffffffffu, s2, 2), r3 = __shfl_xor_sync(0xffffffffu, s3, 2);
+    if (tq >= 2) {
+      s0 = r0;
+      s1 = r1;
+      s2 = r2;
+      s3 = r3;
+    }
+  }
   // The reference max only moves when a score exceeds it by more than
   // ATT_RESCALE_SLACK (log2 units): exp2 of the others stays below
   // 2^ATT_RESCALE_SLACK, and the rescale of o, l (and the max reduction across
@@ -205,8 +221,9 @@ __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D 
   const uint32_t h01 = pack_bf16(p0, p1), h23 = pack_bf16(p2, p3);
   const uint32_t q01 = pack_bf16(p0 - bf16_lo(h01), p1 - bf16_hi(h01));
   const uint32_t q23 = pack_bf16(p2 - bf16_lo(h23), p3 - bf16_hi(h23));
-  const uint32_t bh0 = movmatrix_t(h01), bh1 = movmatrix_t(h23);
-  const uint32_t bl0 = movmatrix_t(q01), bl1 = movmatrix_t(q23);
+  const bool lo_cols = PK && tq >= 2;
+  const uint32_t bh0 = movmatrix_t(lo_cols ? q01 : h01), bh1 = movmatrix_t(lo_cols ? q23 : h23);
+  const uint32_t bl0 = PK ? 0u : movmatrix_t(q01), bl1 = PK ? 0u : movmatrix_t(q23);
   // ---- O^T += V^T P^T; rows of V past the live length are zeroed
   const bool partial = kb + 16 > nvalid;
   const int klo = kb + 2 * tq, khi = klo + 8;
@@ -228,8 +245,18 @@ __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D 
       a3 &= mhi;
     }
     mma_bf16(A.o[i], a0, a1, a2, a3, bh0, bh1);
-    mma_bf16(A.o[i], a0, a1, a2, a3, bl0, bl1);
+    if (!PK) mma_bf16(A.o[i], a0, a1, a2, a3, bl0, bl1);
   }
+}
+
+// After tile_math<D, true>: o of heads 2tq, 2tq+1 in the threads with tq < 2
+// (hi columns plus the lo columns held by lane ^ 2).
+template <int D>
+__device__ __forceinline__ void pack_fold(WarpAcc<D>& A) {
+#pragma unroll
+  for (int i = 0; i < D / 16; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) A.o[i][j] += __shfl_xor_sync(0xffffffffu, A.o[i][j], 2);
 }
 
 // Merge the eight consumer warps' accumulators of a piece through shared
@@ -709,7 +736,7 @@ constexpr int STEP_PRODUCER = ATT_CONSUMERS;      // warp 8: TMA
 constexpr int STEP_INPUT = ATT_CONSUMERS + 1;     // warp 9: queries, appended rows, x_l hand-off
 constexpr int STEP_THREADS = (ATT_CONSUMERS + 2) * 32;
 
-template <int D>
+template <int D, bool PK>
 __global__ void __launch_bounds__(STEP_THREADS, 1)
     att_step_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                     StepAttArgs a) {
@@ -1020,7 +1047,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           fence_proxy_async_smem();
           __syncwarp();
         }
-        if (kb < nvalid) tile_math<D>(A, qf, sk, sv, kb, nvalid, a.scale_log2, lane);
+        if (kb < nvalid) tile_math<D, PK>(A, qf, sk, sv, kb, nvalid, a.scale_log2, lane);
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_empty + 8 * st);
       }
@@ -1045,6 +1072,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         l0 += __shfl_xor_sync(0xffffffffu, l0, off);
         l1 += __shfl_xor_sync(0xffffffffu, l1, off);
       }
+      if (PK) pack_fold<D>(A);
       float* ms = reinterpret_cast<float*>(gbase + SL.pbuf + slot * SL.pslot);  // [ATT_MAX_G][8 warps]
       float* ls = ms + ATT_MAX_G * ATT_CONSUMERS;                                // [ATT_MAX_G][8 warps]
       float* os = ls + ATT_MAX_G * ATT_CONSUMERS;                                // [8 warps][G][D + 4]
@@ -1123,7 +1151,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
       }
       // complete the segment: the records of CTAs c0+1..c1 in order (RB at a
       // time, one round trip when they are there)
-      constexpr int RB = 2;
+      constexpr int RB = 4;
       for (int64_t c = c0 + 1; c <= c1 && ok; c += RB) {
         float mv[RB], lv[RB], ov[RB][4];
         uint64_t t0 = 0;
@@ -1255,7 +1283,7 @@ static int env_int(const char* name, int dflt, int lo, int hi) {
   return v < lo ? lo : (v > hi ? hi : v);
 }
 int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", 512, 0, 1 << 20); }
-int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 12, 0, 64); }
+int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 6, 0, 64); }
 int att_step_groups() { return env_int("PCED_ATT_GROUPS", 2, 1, ATT_MAX_GROUPS); }
 
 // cudaFuncSetAttribute once per kernel and device
@@ -1295,12 +1323,12 @@ cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-template <int D>
+template <int D, bool PK>
 static cudaError_t launch_step(const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
                                cudaStream_t stream) {
   static bool configured[64];
   const StepSmem SL = step_smem(D, a.G);
-  cudaError_t e = set_smem_once(att_step_kernel<D>, 227 * 1024, configured);
+  cudaError_t e = set_smem_once(att_step_kernel<D, PK>, 227 * 1024, configured);
   if (e != cudaSuccess) return e;
   // every CTA waits for the others' layer results, so all must be resident at
   // once: a cooperative launch guarantees it (or fails)
@@ -1314,13 +1342,16 @@ static cudaError_t launch_step(const CUtensorMap& kmap, const CUtensorMap& vmap,
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, att_step_kernel<D>, kmap, vmap, a);
+  return cudaLaunchKernelEx(&cfg, att_step_kernel<D, PK>, kmap, vmap, a);
 }
 
 cudaError_t att_step_launch(int D, const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
                             cudaStream_t stream) {
-  if (D == 128) return launch_step<128>(kmap, vmap, a, ctas, stream);
-  if (D == 64) return launch_step<64>(kmap, vmap, a, ctas, stream);
+  const bool pk = a.G <= 4;  // hi and lo parts of P share one MMA
+  if (D == 128) return pk ? launch_step<128, true>(kmap, vmap, a, ctas, stream)
+                          : launch_step<128, false>(kmap, vmap, a, ctas, stream);
+  if (D == 64) return pk ? launch_step<64, true>(kmap, vmap, a, ctas, stream)
+                         : launch_step<64, false>(kmap, vmap, a, ctas, stream);
   return cudaErrorInvalidValue;
 }
 
