@@ -70,6 +70,14 @@ __device__ __forceinline__ Scratch carve_scratch(uint8_t* p) {
   return sc;
 }
 
+// Non-negative 64-bit quotient through the 32-bit divider when both operands
+// fit (positions of any realistic step do); 64-bit division is a long
+// software sequence.
+__device__ __forceinline__ int64_t udiv_pos(int64_t a, int64_t b) {
+  if ((((uint64_t)a | (uint64_t)b) >> 32) == 0) return (int64_t)((uint32_t)a / (uint32_t)b);
+  return a / b;
+}
+
 struct Piece {
   int32_t s, h, k0, k1;  // real keys [k0, k1) of kv-head h of sequence s (k0 == k1: no keys)
   int64_t adv;           // positions the piece spans
@@ -83,7 +91,7 @@ struct Piece {
 __device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* lens, int32_t s_lo, int32_t s_hi,
                                             int64_t T, int64_t p, int64_t end) {
   Piece pc;
-  pc.h = (int32_t)(p / T);
+  pc.h = (int32_t)udiv_pos(p, T);
   const int64_t r = p - (int64_t)pc.h * T + pre[s_lo];
   int32_t lo = s_lo, hi = s_hi - 1;
   while (lo < hi) {
@@ -673,21 +681,35 @@ __device__ __forceinline__ bool wait_inv_rms(const uint64_t* part, int n, uint32
   }
 }
 
+// What the input warp tells the consumers about the piece in a hand-off slot
+// (the consumers take their pieces from the slots, in the input warp's order).
+struct PieceDesc {
+  int32_t s, h, k0, k1;  // keys [k0, k1) of kv-head h of sequence s
+  int32_t l, gi;         // layer, sequence group
+  int32_t c0, c1;        // CTAs holding the segment's keys (c0 completes it)
+  int32_t app_row;       // key appended this step if it falls in the piece, else -1
+  int32_t end;           // no more pieces
+  int32_t pad[2];
+};
+
 // Shared-memory layout of the step kernel (byte offsets from the 1024-byte
 // aligned base), a function of the head dim and group size only.
 struct StepSmem {
   uint32_t stages;      // K/V ring stages
   uint32_t bar;         // full[st] empty[st] qfull[2] qempty[2] pfull[2] pempty[2] msync
-  uint32_t qbuf, qslot; // [2] hand-off slots: q words [8][D/2+4], K row, V row (bf16), x_l of the head group (fp32)
+  uint32_t qbuf, qslot; // [2] hand-off slots: q words [8][D/2+4], K row, V row (bf16), x_l of the head group (fp32),
+                        // PieceDesc (at qdesc)
+  uint32_t qdesc;
   uint32_t pbuf, pslot; // [2] partial hand-off slots: ms[8][8], ls[8][8], os[8][G][D + 4]
-  uint32_t misc;        // red[2][2] floats, flags
+  uint32_t misc;        // flags
   uint32_t tables;      // pre[ATT_MAX_S+1] int64, GroupPlan, lens[ATT_MAX_S] int32, apnd[ATT_MAX_S] u8
   uint32_t total;       // bytes to request, alignment slack included
 };
 __host__ __device__ inline StepSmem step_smem(int D, int G) {
   StepSmem L;
   const uint32_t stage_bytes = 2u * (uint32_t)(D / 64) * (ATT_BLOCK_N * 128u);
-  L.qslot = 8u * (uint32_t)(D / 2 + 4) * 4u + 4u * (uint32_t)D + 4u * (uint32_t)(G * D);
+  L.qdesc = 8u * (uint32_t)(D / 2 + 4) * 4u + 4u * (uint32_t)D + 4u * (uint32_t)(G * D);
+  L.qslot = L.qdesc + (uint32_t)sizeof(PieceDesc);
   L.pslot = 2u * ATT_CONSUMERS * ATT_MAX_G * 4u + (uint32_t)ATT_CONSUMERS * G * (D + 4) * 4u;
   const uint32_t tables = (ATT_MAX_S + 1) * 8u + (uint32_t)((sizeof(GroupPlan) + 7) & ~(size_t)7) + ATT_MAX_S * 4u + ATT_MAX_S;
   const uint32_t max_st = D == 128 ? 5u : 7u;
@@ -752,7 +774,6 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   const uint32_t bar_full = base + SL.bar, bar_empty = bar_full + 8 * NST;
   const uint32_t bar_qfull = bar_empty + 8 * NST, bar_qempty = bar_qfull + 16;
   const uint32_t bar_pfull = bar_qempty + 16, bar_pempty = bar_pfull + 16, bar_m = bar_pempty + 16;
-  float* red = reinterpret_cast<float*>(gbase + SL.misc);  // [2 slots][2 merge warps]
   int* flag = reinterpret_cast<int*>(gbase + SL.misc + 32);
   int64_t* pre = reinterpret_cast<int64_t*>(gbase + SL.tables);
   GroupPlan& gp = *reinterpret_cast<GroupPlan*>(pre + ATT_MAX_S + 1);
@@ -975,8 +996,33 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
             reinterpret_cast<uint32_t*>(a.v_cache + grow)[i] = vb;
           }
         }
+        if (lane == 0) {
+          const int64_t pa = (int64_t)pc.h * gp.T[gi] + pre[pc.s] - pre[gp.s_lo[gi]];
+          PieceDesc* dsc = reinterpret_cast<PieceDesc*>(reinterpret_cast<uint8_t*>(qw) + SL.qdesc);
+          dsc->s = pc.s;
+          dsc->h = pc.h;
+          dsc->k0 = pc.k0;
+          dsc->k1 = pc.k1;
+          dsc->l = l;
+          dsc->gi = gi;
+          dsc->c0 = (int32_t)udiv_pos(pa, gp.P[gi]);
+          dsc->c1 = (int32_t)udiv_pos(pa + lens[pc.s] - 1, gp.P[gi]);
+          dsc->app_row = app ? lens[pc.s] - 1 : -1;
+          dsc->end = 0;
+        }
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_qfull + 8 * slot);
+      }
+    }
+    // end marker for the consumers
+    if (ok) {
+      const uint32_t slot = p & 1u, u = p >> 1;
+      if (u == 0 || mbar_wait(bar_qempty + 8 * slot, (u - 1u) & 1u, a.status)) {
+        if (lane == 0) {
+          PieceDesc* dsc = reinterpret_cast<PieceDesc*>(gbase + SL.qbuf + slot * SL.qslot + SL.qdesc);
+          dsc->end = 1;
+          mbar_arrive(bar_qfull + 8 * slot);
+        }
       }
     }
     return;
@@ -989,252 +1035,251 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   const bool hv = g < G;
   uint32_t it = 0, p = 0, cst = 0, cuse = 0;  // tile counter; its stage and use count (it % NST, it / NST)
   bool ok = true;
-  for (int l = 0; l < a.L && ok; ++l)
-  for (int gi = 0; gi < gp.n && ok; ++gi) {
-    const int32_t g_lo = gp.s_lo[gi];
-    const int64_t gT = gp.T[gi], gP = gp.P[gi], gce = gp.ce[gi];
-    const int64_t rbase = (int64_t)gi * ((int64_t)gridDim.x + (int64_t)S * Hkv);  // this group's record slots
-    for (int64_t pp = gp.cb[gi]; pp < gce && ok;) {
-      const Piece pc = find_piece(pre, lens, g_lo, gp.s_lo[gi + 1], gT, pp, gce);
-      pp += pc.adv;
-      if (pc.k0 == pc.k1) continue;
-      const uint32_t slot = p & 1u, u = p >> 1;
-      ++p;
-      if (!mbar_wait(bar_qfull + 8 * slot, u & 1u, a.status)) {
-        ok = false;
-        break;
-      }
-      const uint32_t* qw = reinterpret_cast<const uint32_t*>(gbase + SL.qbuf + slot * SL.qslot);
-      uint32_t qf[C::KSTEPS][2];
+  for (;;) {
+    const uint32_t slot = p & 1u, u = p >> 1;
+    ++p;
+    if (!mbar_wait(bar_qfull + 8 * slot, u & 1u, a.status)) {
+      ok = false;
+      break;
+    }
+    const uint32_t* qw = reinterpret_cast<const uint32_t*>(gbase + SL.qbuf + slot * SL.qslot);
+    const PieceDesc dsc = *reinterpret_cast<const PieceDesc*>(gbase + SL.qbuf + slot * SL.qslot + SL.qdesc);
+    if (dsc.end) break;
+    const int l = dsc.l;
+    const int64_t rbase = (int64_t)dsc.gi * ((int64_t)gridDim.x + (int64_t)S * Hkv);  // the group's record slots
+    Piece pc;
+    pc.s = dsc.s;
+    pc.h = dsc.h;
+    pc.k0 = dsc.k0;
+    pc.k1 = dsc.k1;
+    uint32_t qf[C::KSTEPS][2];
 #pragma unroll
-      for (int j = 0; j < C::KSTEPS; ++j) {
-        qf[j][0] = hv ? qw[g * QW + 8 * j + tq] : 0u;
-        qf[j][1] = hv ? qw[g * QW + 8 * j + 4 + tq] : 0u;
-      }
-      const int32_t app_row = (apnd[pc.s] && pc.k1 == lens[pc.s]) ? lens[pc.s] - 1 : -1;
+    for (int j = 0; j < C::KSTEPS; ++j) {
+      qf[j][0] = hv ? qw[g * QW + 8 * j + tq] : 0u;
+      qf[j][1] = hv ? qw[g * QW + 8 * j + 4 + tq] : 0u;
+    }
+    const int32_t app_row = dsc.app_row;
 
-      WarpAcc<D> A;
-      acc_reset(A);
-      for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it, cst = cst + 1 == NST ? (++cuse, 0u) : cst + 1) {
-        if ((int)(it & 1u) != wg) continue;
-        const uint32_t use = cuse, st = cst, ph = use & 1u;
-        if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status)) {
-          ok = false;
-          break;
-        }
-        if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
-          ok = false;
-          break;
-        }
-        const int nvalid = min(ATT_BLOCK_N, pc.k1 - kt);
-        const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
-        if (app_row >= kt && app_row < kt + ATT_BLOCK_N && ((app_row - kt) >> 4) == wl) {
-          // the appended row (prepared by the input warp) replaces whatever
-          // the cache held there when the tile was loaded
-          const int r = app_row - kt;
-          const uint32_t src = base + SL.qbuf + slot * SL.qslot + 8 * QW * 4;
-          for (int c = lane; c < 2 * (D / 8); c += 32) {
-            const int cc = c % (D / 8);
-            const uint32_t dst = (c < D / 8 ? sk : sv) + (cc >> 3) * C::BOX_BYTES + r * 128 +
-                                 ((((uint32_t)cc & 7u) ^ ((uint32_t)r & 7u)) << 4);
-            uint32_t w0, w1, w2, w3;
-            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                         : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
-                         : "r"(src + 16 * c));
-            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w0), "r"(w1), "r"(w2), "r"(w3)
-                         : "memory");
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-        }
-        if (kb < nvalid) tile_math<D, PK>(A, qf, sk, sv, kb, nvalid, a.scale_log2, lane);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar_empty + 8 * st);
-      }
-      if (!ok) break;
-      const int64_t seg = (int64_t)pc.h * S + pc.s;
-      const int64_t pa = (int64_t)pc.h * gT + pre[pc.s] - pre[g_lo];
-      const int64_t c0 = pa / gP, c1 = (pa + lens[pc.s] - 1) / gP;
-      const bool merges = c0 == (int64_t)blockIdx.x;  // the segment's first CTA completes it
-      if (!merges) {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bar_qempty + 8 * slot);
-      }
-      // combine the eight warps' partials through a double-buffered slot;
-      // afterwards thread tid < G*D/4 owns outputs idx0..idx0+3 (head hh)
-      if (u > 0 && !mbar_wait(bar_pempty + 8 * slot, (u - 1u) & 1u, a.status)) {
+    WarpAcc<D> A;
+    acc_reset(A);
+    for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it, cst = cst + 1 == NST ? (++cuse, 0u) : cst + 1) {
+      if ((int)(it & 1u) != wg) continue;
+      const uint32_t use = cuse, st = cst, ph = use & 1u;
+      if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status)) {
         ok = false;
         break;
       }
-      float l0 = A.l0, l1 = A.l1;
-#pragma unroll
-      for (int off = 4; off < 32; off <<= 1) {
-        l0 += __shfl_xor_sync(0xffffffffu, l0, off);
-        l1 += __shfl_xor_sync(0xffffffffu, l1, off);
-      }
-      if (PK) pack_fold<D>(A);
-      float* ms = reinterpret_cast<float*>(gbase + SL.pbuf + slot * SL.pslot);  // [ATT_MAX_G][8 warps]
-      float* ls = ms + ATT_MAX_G * ATT_CONSUMERS;                                // [ATT_MAX_G][8 warps]
-      float* os = ls + ATT_MAX_G * ATT_CONSUMERS;                                // [8 warps][G][D + 4]
-      if (g == 0) {
-        ms[(2 * tq) * ATT_CONSUMERS + warp] = A.m0;
-        ms[(2 * tq + 1) * ATT_CONSUMERS + warp] = A.m1;
-        ls[(2 * tq) * ATT_CONSUMERS + warp] = l0;
-        ls[(2 * tq + 1) * ATT_CONSUMERS + warp] = l1;
-      }
-      {
-        float* ow = os + warp * G * C::OROW;
-        const bool h0 = 2 * tq < G, h1 = 2 * tq + 1 < G;
-#pragma unroll
-        for (int i = 0; i < C::MTILES; ++i) {
-          const int d0 = 16 * i + g, d1 = d0 + 8;
-          if (h0) {
-            ow[(2 * tq) * C::OROW + d0] = A.o[i][0];
-            ow[(2 * tq) * C::OROW + d1] = A.o[i][2];
-          }
-          if (h1) {
-            ow[(2 * tq + 1) * C::OROW + d0] = A.o[i][1];
-            ow[(2 * tq + 1) * C::OROW + d1] = A.o[i][3];
-          }
-        }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar_pfull + 8 * slot);
-      if (!mbar_wait(bar_pfull + 8 * slot, u & 1u, a.status)) {
+      if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
         ok = false;
         break;
       }
-      const uint32_t tag = step_tag(epoch, l);
-      const bool own = tid < GD / 4;
-      const int hh = own ? tid / (D / 4) : 0, idx0 = own ? 4 * tid : 0;
-      float mx = -INFINITY, lsum = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
-      if (own) {
-        float mw[ATT_CONSUMERS], lw[ATT_CONSUMERS];
-        const float4* m4 = reinterpret_cast<const float4*>(ms + hh * ATT_CONSUMERS);
-        const float4* l4 = reinterpret_cast<const float4*>(ls + hh * ATT_CONSUMERS);
-        *reinterpret_cast<float4*>(mw) = m4[0];
-        *reinterpret_cast<float4*>(mw + 4) = m4[1];
-        *reinterpret_cast<float4*>(lw) = l4[0];
-        *reinterpret_cast<float4*>(lw + 4) = l4[1];
-        float M = mw[0];
-#pragma unroll
-        for (int w = 1; w < ATT_CONSUMERS; ++w) M = fmaxf(M, mw[w]);
-        const float* oc = os + hh * C::OROW + (idx0 - hh * D);
-#pragma unroll
-        for (int w = 0; w < ATT_CONSUMERS; ++w) {
-          if (mw[w] == -INFINITY) continue;  // a warp without live keys in this piece
-          const float e = exp2f(mw[w] - M);
-          const float4 o4 = *reinterpret_cast<const float4*>(oc + w * G * C::OROW);
-          acc[0] += o4.x * e;
-          acc[1] += o4.y * e;
-          acc[2] += o4.z * e;
-          acc[3] += o4.w * e;
-          lsum += lw[w] * e;
+      const int nvalid = min(ATT_BLOCK_N, pc.k1 - kt);
+      const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
+      if (app_row >= kt && app_row < kt + ATT_BLOCK_N && ((app_row - kt) >> 4) == wl) {
+        // the appended row (prepared by the input warp) replaces whatever
+        // the cache held there when the tile was loaded
+        const int r = app_row - kt;
+        const uint32_t src = base + SL.qbuf + slot * SL.qslot + 8 * QW * 4;
+        for (int c = lane; c < 2 * (D / 8); c += 32) {
+          const int cc = c % (D / 8);
+          const uint32_t dst = (c < D / 8 ? sk : sv) + (cc >> 3) * C::BOX_BYTES + r * 128 +
+                               ((((uint32_t)cc & 7u) ^ ((uint32_t)r & 7u)) << 4);
+          uint32_t w0, w1, w2, w3;
+          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                       : "=r"(w0), "=r"(w1), "=r"(w2), "=r"(w3)
+                       : "r"(src + 16 * c));
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w0), "r"(w1), "r"(w2), "r"(w3)
+                       : "memory");
         }
-        mx = M;
+        fence_proxy_async_smem();
+        __syncwarp();
       }
+      if (kb < nvalid) tile_math<D, PK>(A, qf, sk, sv, kb, nvalid, a.scale_log2, lane);
       __syncwarp();
-      if (lane == 0) mbar_arrive(bar_pempty + 8 * slot);
-      if (!merges) {
-        // the segment continues in an earlier CTA: publish this CTA's record
-        const int64_t rs = rbase + (int64_t)blockIdx.x + seg;
-        if (own) {
-          uint64_t* ro = a.rec_o + rs * GD + idx0;
-#pragma unroll
-          for (int j = 0; j < 4; ++j) st_tagged(ro + j, acc[j], tag);
-          if (idx0 % D == 0) {
-            st_tagged(a.rec_ml + (rs * G + hh) * 2, mx, tag);
-            st_tagged(a.rec_ml + (rs * G + hh) * 2 + 1, lsum, tag);
-          }
-        }
-        continue;
-      }
-      // complete the segment: the records of CTAs c0+1..c1 in order (RB at a
-      // time, one round trip when they are there)
-      constexpr int RB = 4;
-      for (int64_t c = c0 + 1; c <= c1 && ok; c += RB) {
-        float mv[RB], lv[RB], ov[RB][4];
-        uint64_t t0 = 0;
-        while (true) {
-          bool good = true;
-#pragma unroll
-          for (int q = 0; q < RB; ++q) {
-            mv[q] = -INFINITY;
-            lv[q] = 0.f;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) ov[q][j] = 0.f;
-            if (!own || c + q > c1) continue;
-            const int64_t rs = rbase + c + q + seg;
-            const uint64_t wm = ld_tagged(a.rec_ml + (rs * G + hh) * 2);
-            const uint64_t wl = ld_tagged(a.rec_ml + (rs * G + hh) * 2 + 1);
-            uint64_t wo[4];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) wo[j] = ld_tagged(a.rec_o + rs * GD + idx0 + j);
-            good &= tv_ok(wm, tag) && tv_ok(wl, tag);
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              good &= tv_ok(wo[j], tag);
-              ov[q][j] = tv_value(wo[j]);
-            }
-            mv[q] = tv_value(wm);
-            lv[q] = tv_value(wl);
-          }
-          if (__all_sync(0xffffffffu, good)) break;
-          if (!poll_again(t0, a.status)) {
-            ok = false;
-            break;
-          }
-        }
-#pragma unroll
-        for (int q = 0; q < RB; ++q) {
-          if (mv[q] == -INFINITY) continue;
-          const float Mn = fmaxf(mx, mv[q]);
-          const float f = mx == -INFINITY ? 0.f : exp2f(mx - Mn), e = exp2f(mv[q] - Mn);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) acc[j] = acc[j] * f + ov[q][j] * e;
-          lsum = lsum * f + lv[q] * e;
-          mx = Mn;
-        }
-      }
-      if (!ok) break;
-      // x_{l+1} = x_l + o for head group h (x_l from the input warp's slot)
-      const int nx = (l + 1) & 1;
-      const uint32_t ntag = step_tag(epoch, l + 1);
-      const float* xr = reinterpret_cast<const float*>(qw + 8 * QW + D);
-      uint64_t* xn = a.resid + ((int64_t)nx * S + pc.s) * d + (int64_t)pc.h * GD;
-      float xv[4] = {0.f, 0.f, 0.f, 0.f};
-      float ss = 0.f;
-      if (own) {
-        const float4 x4 = *reinterpret_cast<const float4*>(xr + idx0);
-        const float xo[4] = {x4.x, x4.y, x4.z, x4.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          xv[j] = xo[j] + (lsum > 0.f ? acc[j] / lsum : 0.f);
-          st_tagged(xn + idx0 + j, xv[j], ntag);
-          ss += xv[j] * xv[j];
-        }
-      }
+      if (lane == 0) mbar_arrive(bar_empty + 8 * st);
+    }
+    if (!ok) break;
+    const int64_t seg = (int64_t)pc.h * S + pc.s;
+    const int64_t c0 = dsc.c0, c1 = dsc.c1;
+    const bool merges = c0 == (int64_t)blockIdx.x;  // the segment's first CTA completes it
+    if (!merges) {
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_qempty + 8 * slot);
-      ss = warp_sum(ss);
-      uint64_t* ps = a.part_ss + ((int64_t)nx * S + pc.s) * Hkv * ATT_CONSUMERS;
-      if (lane == 0) st_tagged(ps + pc.h * ATT_CONSUMERS + warp, ss, ntag);
-      if (l + 1 < a.L) continue;
-      // after the last layer: head group h of the final hidden state
-      float inv;
-      if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, ntag, d, a.rms_eps, lane, a.status, inv)) {
-        ok = false;
-        break;
-      }
-      if (own) {
-        __nv_bfloat16* hs = a.hidden + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0;
-        __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0 : nullptr;
+    }
+    // combine the eight warps' partials through a double-buffered slot;
+    // afterwards thread tid < G*D/4 owns outputs idx0..idx0+3 (head hh)
+    if (u > 0 && !mbar_wait(bar_pempty + 8 * slot, (u - 1u) & 1u, a.status)) {
+      ok = false;
+      break;
+    }
+    float l0 = A.l0, l1 = A.l1;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const __nv_bfloat16 hv2 = __float2bfloat16_rn(xv[j] * inv);
-          hs[j] = hv2;
-          if (hc) hc[j] = hv2;
+    for (int off = 4; off < 32; off <<= 1) {
+      l0 += __shfl_xor_sync(0xffffffffu, l0, off);
+      l1 += __shfl_xor_sync(0xffffffffu, l1, off);
+    }
+    if (PK) pack_fold<D>(A);
+    float* ms = reinterpret_cast<float*>(gbase + SL.pbuf + slot * SL.pslot);  // [ATT_MAX_G][8 warps]
+    float* ls = ms + ATT_MAX_G * ATT_CONSUMERS;                                // [ATT_MAX_G][8 warps]
+    float* os = ls + ATT_MAX_G * ATT_CONSUMERS;                                // [8 warps][G][D + 4]
+    if (g == 0) {
+      ms[(2 * tq) * ATT_CONSUMERS + warp] = A.m0;
+      ms[(2 * tq + 1) * ATT_CONSUMERS + warp] = A.m1;
+      ls[(2 * tq) * ATT_CONSUMERS + warp] = l0;
+      ls[(2 * tq + 1) * ATT_CONSUMERS + warp] = l1;
+    }
+    {
+      float* ow = os + warp * G * C::OROW;
+      const bool h0 = 2 * tq < G, h1 = 2 * tq + 1 < G;
+#pragma unroll
+      for (int i = 0; i < C::MTILES; ++i) {
+        const int d0 = 16 * i + g, d1 = d0 + 8;
+        if (h0) {
+          ow[(2 * tq) * C::OROW + d0] = A.o[i][0];
+          ow[(2 * tq) * C::OROW + d1] = A.o[i][2];
         }
+        if (h1) {
+          ow[(2 * tq + 1) * C::OROW + d0] = A.o[i][1];
+          ow[(2 * tq + 1) * C::OROW + d1] = A.o[i][3];
+        }
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_pfull + 8 * slot);
+    if (!mbar_wait(bar_pfull + 8 * slot, u & 1u, a.status)) {
+      ok = false;
+      break;
+    }
+    const uint32_t tag = step_tag(epoch, l);
+    const bool own = tid < GD / 4;
+    const int hh = own ? tid / (D / 4) : 0, idx0 = own ? 4 * tid : 0;
+    float mx = -INFINITY, lsum = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
+    if (own) {
+      float mw[ATT_CONSUMERS], lw[ATT_CONSUMERS];
+      const float4* m4 = reinterpret_cast<const float4*>(ms + hh * ATT_CONSUMERS);
+      const float4* l4 = reinterpret_cast<const float4*>(ls + hh * ATT_CONSUMERS);
+      *reinterpret_cast<float4*>(mw) = m4[0];
+      *reinterpret_cast<float4*>(mw + 4) = m4[1];
+      *reinterpret_cast<float4*>(lw) = l4[0];
+      *reinterpret_cast<float4*>(lw + 4) = l4[1];
+      float M = mw[0];
+#pragma unroll
+      for (int w = 1; w < ATT_CONSUMERS; ++w) M = fmaxf(M, mw[w]);
+      const float* oc = os + hh * C::OROW + (idx0 - hh * D);
+#pragma unroll
+      for (int w = 0; w < ATT_CONSUMERS; ++w) {
+        if (mw[w] == -INFINITY) continue;  // a warp without live keys in this piece
+        const float e = exp2f(mw[w] - M);
+        const float4 o4 = *reinterpret_cast<const float4*>(oc + w * G * C::OROW);
+        acc[0] += o4.x * e;
+        acc[1] += o4.y * e;
+        acc[2] += o4.z * e;
+        acc[3] += o4.w * e;
+        lsum += lw[w] * e;
+      }
+      mx = M;
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_pempty + 8 * slot);
+    if (!merges) {
+      // the segment continues in an earlier CTA: publish this CTA's record
+      const int64_t rs = rbase + (int64_t)blockIdx.x + seg;
+      if (own) {
+        uint64_t* ro = a.rec_o + rs * GD + idx0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) st_tagged(ro + j, acc[j], tag);
+        if (idx0 % D == 0) {
+          st_tagged(a.rec_ml + (rs * G + hh) * 2, mx, tag);
+          st_tagged(a.rec_ml + (rs * G + hh) * 2 + 1, lsum, tag);
+        }
+      }
+      continue;
+    }
+    // complete the segment: the records of CTAs c0+1..c1 in order (RB at a
+    // time, one round trip when they are there)
+    constexpr int RB = 4;
+    for (int64_t c = c0 + 1; c <= c1 && ok; c += RB) {
+      float mv[RB], lv[RB], ov[RB][4];
+      uint64_t t0 = 0;
+      while (true) {
+        bool good = true;
+#pragma unroll
+        for (int q = 0; q < RB; ++q) {
+          mv[q] = -INFINITY;
+          lv[q] = 0.f;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) ov[q][j] = 0.f;
+          if (!own || c + q > c1) continue;
+          const int64_t rs = rbase + c + q + seg;
+          const uint64_t wm = ld_tagged(a.rec_ml + (rs * G + hh) * 2);
+          const uint64_t wl = ld_tagged(a.rec_ml + (rs * G + hh) * 2 + 1);
+          uint64_t wo[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) wo[j] = ld_tagged(a.rec_o + rs * GD + idx0 + j);
+          good &= tv_ok(wm, tag) && tv_ok(wl, tag);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            good &= tv_ok(wo[j], tag);
+            ov[q][j] = tv_value(wo[j]);
+          }
+          mv[q] = tv_value(wm);
+          lv[q] = tv_value(wl);
+        }
+        if (__all_sync(0xffffffffu, good)) break;
+        if (!poll_again(t0, a.status)) {
+          ok = false;
+          break;
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < RB; ++q) {
+        if (mv[q] == -INFINITY) continue;
+        const float Mn = fmaxf(mx, mv[q]);
+        const float f = mx == -INFINITY ? 0.f : exp2f(mx - Mn), e = exp2f(mv[q] - Mn);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[j] = acc[j] * f + ov[q][j] * e;
+        lsum = lsum * f + lv[q] * e;
+        mx = Mn;
+      }
+    }
+    if (!ok) break;
+    // x_{l+1} = x_l + o for head group h (x_l from the input warp's slot)
+    const int nx = (l + 1) & 1;
+    const uint32_t ntag = step_tag(epoch, l + 1);
+    const float* xr = reinterpret_cast<const float*>(qw + 8 * QW + D);
+    uint64_t* xn = a.resid + ((int64_t)nx * S + pc.s) * d + (int64_t)pc.h * GD;
+    float xv[4] = {0.f, 0.f, 0.f, 0.f};
+    float ss = 0.f;
+    if (own) {
+      const float4 x4 = *reinterpret_cast<const float4*>(xr + idx0);
+      const float xo[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        xv[j] = xo[j] + (lsum > 0.f ? acc[j] / lsum : 0.f);
+        st_tagged(xn + idx0 + j, xv[j], ntag);
+        ss += xv[j] * xv[j];
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_qempty + 8 * slot);
+    ss = warp_sum(ss);
+    uint64_t* ps = a.part_ss + ((int64_t)nx * S + pc.s) * Hkv * ATT_CONSUMERS;
+    if (lane == 0) st_tagged(ps + pc.h * ATT_CONSUMERS + warp, ss, ntag);
+    if (l + 1 < a.L) continue;
+    // after the last layer: head group h of the final hidden state
+    float inv;
+    if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, ntag, d, a.rms_eps, lane, a.status, inv)) {
+      ok = false;
+      break;
+    }
+    if (own) {
+      __nv_bfloat16* hs = a.hidden + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0;
+      __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0 : nullptr;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const __nv_bfloat16 hv2 = __float2bfloat16_rn(xv[j] * inv);
+        hs[j] = hv2;
+        if (hc) hc[j] = hv2;
       }
     }
   }
