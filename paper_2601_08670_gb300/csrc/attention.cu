@@ -86,10 +86,10 @@ struct Piece {
 // Piece that starts at position p of the position space of sequences
 // [s_lo, s_hi) and ends at the next segment boundary or at `end`.  Segment
 // (h, s) spans positions [h*T + pre[s] - pre[s_lo], h*T + pre[s+1] - pre[s_lo])
-// with T = pre[s_hi] - pre[s_lo]; its first lens[s] positions are keys, the
-// rest (if any) only weight the partition.
+// with T = pre[s_hi] - pre[s_lo]; positions lead .. lead + lens[s] - 1 of it
+// are its keys, the others (if any) only weight the partition.
 __device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* lens, int32_t s_lo, int32_t s_hi,
-                                            int64_t T, int64_t p, int64_t end) {
+                                            int64_t T, int64_t p, int64_t end, int32_t lead = 0) {
   Piece pc;
   pc.h = (int32_t)udiv_pos(p, T);
   const int64_t r = p - (int64_t)pc.h * T + pre[s_lo];
@@ -100,15 +100,15 @@ __device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* l
     else hi = mid - 1;
   }
   pc.s = lo;
-  const int64_t off = r - pre[lo];
+  const int64_t off = r - pre[lo] - lead;  // key index of position p (negative in the leading part)
   const int64_t seg_end = (int64_t)pc.h * T + pre[lo + 1] - pre[s_lo];
   const int64_t e = seg_end < end ? seg_end : end;
   pc.adv = e - p;
   const int64_t len = lens[lo];
-  if (off < len) {
-    const int64_t k1 = off + pc.adv;
-    pc.k0 = (int32_t)off;
-    pc.k1 = (int32_t)(k1 < len ? k1 : len);
+  const int64_t k0 = off < 0 ? 0 : off, k1 = off + pc.adv < len ? off + pc.adv : len;
+  if (k0 < k1) {
+    pc.k0 = (int32_t)k0;
+    pc.k1 = (int32_t)k1;
   } else {
     pc.k0 = pc.k1 = 0;
   }
@@ -157,9 +157,10 @@ __device__ __forceinline__ void acc_reset(WarpAcc<D>& A) {
 //
 // P enters the P V product as bf16 hi + lo parts.  With PK (at most four
 // heads) both parts share one MMA: accumulator columns 0-3 take the hi parts
-// of heads 0-3 and columns 4-7 the lo parts of the same heads (the threads
-// owning columns 4-7, tq >= 2, mirror the scores of lane ^ 2), so o of head h
-// is column h plus column h + 4 (summed once per piece, see pack_fold).
+// of heads 0-3 and columns 4-7 the lo parts of the same heads (qf repeats
+// heads 0-3 in columns 4-7, so the threads owning those columns, tq >= 2,
+// hold the same scores as lane ^ 2), and o of head h is column h plus column
+// h + 4 (summed once per piece, see pack_fold).
 template <int D, bool PK = false>
 __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D / 16][2], uint32_t sk, uint32_t sv,
                                           int kb, int nvalid, float scale_log2, int lane) {
@@ -181,20 +182,10 @@ __device__ __forceinline__ void tile_math(WarpAcc<D>& A, const uint32_t (&qf)[D 
     }
   }
   const bool v0 = kb + g < nvalid, v1 = kb + g + 8 < nvalid;
-  float s0 = v0 ? ((sc4[0][0] + sc4[1][0]) + (sc4[2][0] + sc4[3][0])) * scale_log2 : -INFINITY;
-  float s1 = v0 ? ((sc4[0][1] + sc4[1][1]) + (sc4[2][1] + sc4[3][1])) * scale_log2 : -INFINITY;
-  float s2 = v1 ? ((sc4[0][2] + sc4[1][2]) + (sc4[2][2] + sc4[3][2])) * scale_log2 : -INFINITY;
-  float s3 = v1 ? ((sc4[0][3] + sc4[1][3]) + (sc4[2][3] + sc4[3][3])) * scale_log2 : -INFINITY;
-  if (PK) {
-    const float r0 = __shfl_xor_sync(0xffffffffu, s0, 2), r1 = __shfl_xor_sync(0xffffffffu, s1, 2);
-    const float r2 = __shfl_xor_sync(0xffffffffu, s2, 2), r3 = __shfl_xor_sync(0xffffffffu, s3, 2);
-    if (tq >= 2) {
-      s0 = r0;
-      s1 = r1;
-      s2 = r2;
-      s3 = r3;
-    }
-  }
+  const float s0 = v0 ? ((sc4[0][0] + sc4[1][0]) + (sc4[2][0] + sc4[3][0])) * scale_log2 : -INFINITY;
+  const float s1 = v0 ? ((sc4[0][1] + sc4[1][1]) + (sc4[2][1] + sc4[3][1])) * scale_log2 : -INFINITY;
+  const float s2 = v1 ? ((sc4[0][2] + sc4[1][2]) + (sc4[2][2] + sc4[3][2])) * scale_log2 : -INFINITY;
+  const float s3 = v1 ? ((sc4[0][3] + sc4[1][3]) + (sc4[2][3] + sc4[3][3])) * scale_log2 : -INFINITY;
   // The reference max only moves when a score exceeds it by more than
   // ATT_RESCALE_SLACK (log2 units): exp2 of the others stays below
   // 2^ATT_RESCALE_SLACK, and the rescale of o, l (and the max reduction across
@@ -632,7 +623,7 @@ __device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a,
       c.p = gp.cb[c.g];
       continue;
     }
-    c.pc = find_piece(pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g]);
+    c.pc = find_piece(pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead);
     if (c.pc.k0 < c.pc.k1) {
       c.kt = c.pc.k0;
       c.row0 = (int64_t)c.l * a.rows_per_layer + (a.kv_offset[c.pc.s] + (int64_t)c.pc.h * a.cap[c.pc.s] * D) / D;
@@ -889,7 +880,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
       const uint32_t tag = step_tag(epoch, l);
       for (int gi = 0; gi < gp.n && ok; ++gi)
       for (int64_t pp = gp.cb[gi]; pp < gp.ce[gi] && ok;) {
-        const Piece pc = find_piece(pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi]);
+        const Piece pc = find_piece(pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead);
         pp += pc.adv;
         if (pc.k0 == pc.k1) continue;
         const uint32_t slot = p & 1u, u = p >> 1;
@@ -997,7 +988,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           }
         }
         if (lane == 0) {
-          const int64_t pa = (int64_t)pc.h * gp.T[gi] + pre[pc.s] - pre[gp.s_lo[gi]];
+          const int64_t pa = (int64_t)pc.h * gp.T[gi] + pre[pc.s] - pre[gp.s_lo[gi]] + a.seg_lead;  // first key
           PieceDesc* dsc = reinterpret_cast<PieceDesc*>(reinterpret_cast<uint8_t*>(qw) + SL.qdesc);
           dsc->s = pc.s;
           dsc->h = pc.h;
@@ -1032,7 +1023,10 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   const int wg = warp >> 2, wl = warp & 3;
   const int g = lane >> 2, tq = lane & 3;
   const int kb = 16 * wl;
-  const bool hv = g < G;
+  // B column g of S^T = K Q^T is head g; with PK columns 4-7 repeat heads 0-3,
+  // so the threads owning those columns compute the scores they mirror
+  const int qh = PK ? (g & 3) : g;
+  const bool hv = qh < G;
   uint32_t it = 0, p = 0, cst = 0, cuse = 0;  // tile counter; its stage and use count (it % NST, it / NST)
   bool ok = true;
   for (;;) {
@@ -1055,8 +1049,8 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     uint32_t qf[C::KSTEPS][2];
 #pragma unroll
     for (int j = 0; j < C::KSTEPS; ++j) {
-      qf[j][0] = hv ? qw[g * QW + 8 * j + tq] : 0u;
-      qf[j][1] = hv ? qw[g * QW + 8 * j + 4 + tq] : 0u;
+      qf[j][0] = hv ? qw[qh * QW + 8 * j + tq] : 0u;
+      qf[j][1] = hv ? qw[qh * QW + 8 * j + 4 + tq] : 0u;
     }
     const int32_t app_row = dsc.app_row;
 
@@ -1330,6 +1324,7 @@ static int env_int(const char* name, int dflt, int lo, int hi) {
 int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", 512, 0, 1 << 20); }
 int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 6, 0, 64); }
 int att_step_groups() { return env_int("PCED_ATT_GROUPS", 2, 1, ATT_MAX_GROUPS); }
+int att_step_seg_lead(int seg_cost) { return env_int("PCED_ATT_LEAD", 0, 0, seg_cost); }
 
 // cudaFuncSetAttribute once per kernel and device
 template <typename K>

@@ -100,6 +100,7 @@ struct StepAttArgs {
   int64_t layer_elems;
   float scale_log2, rms_eps;
   int32_t seg_cost;           // partition weight of a piece, in keys
+  int32_t seg_lead;           // how many of the seg_cost positions come before the keys (the rest after)
   int32_t pf_tiles;           // tiles prefetched into L2 ahead of the shared-memory ring
   int32_t groups;             // sequence groups (1..ATT_MAX_GROUPS), each partitioned over all CTAs
   const int64_t* kv_offset;   // [S]
@@ -127,6 +128,7 @@ int64_t att_step_slots(int32_t S, int32_t Hkv);
 int att_step_seg_cost(int D);
 int att_step_pf_tiles();
 int att_step_groups();
+int att_step_seg_lead(int seg_cost);
 cudaError_t att_step_launch(int D, const CUtensorMap& kmap, const CUtensorMap& vmap, const StepAttArgs& a, int ctas,
                             cudaStream_t stream);
 

@@ -140,6 +140,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   at.seg_cost = att_step_seg_cost(dm.D);
   at.pf_tiles = att_step_pf_tiles();
   at.groups = att_step_groups();
+  at.seg_lead = att_step_seg_lead(at.seg_cost);
   at.kv_offset = p->kv_offset;
   at.cap = p->cap;
   at.seq_len = p->seq_len;
