@@ -171,7 +171,9 @@ pced_status pced_contrastive_select(const float* logprobs, const float* beta, co
  * The step index t, lengths and history live on the device, so a captured
  * CUDA graph of one call can be replayed step after step.  Each call adds
  * one to *step and to every seq_len[s].  Requires 2*Hkv <= Hq plus the limits
- * of the three calls above.
+ * of the three calls above.  The workspace must be zero-filled before the
+ * first call: besides the status word it holds counters the kernels leave
+ * at zero when they finish.
  * ------------------------------------------------------------------------ */
 typedef struct pced_step_args {
   pced_dims dims;

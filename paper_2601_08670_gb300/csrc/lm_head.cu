@@ -47,7 +47,7 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
   g->nbeta = S;  // beta has B*N < S entries
   const size_t slab = LM_A_BYTES + (size_t)g->S_pad * 128;
   const size_t fixed = 1024 + 64 * 8 + 16 + (size_t)2 * 4 * g->S_pad * sizeof(float2) +
-                       (size_t)2 * g->S_pad * sizeof(float2) + (size_t)(g->nbeta + 3) * 4 + 8 * 64 * 4 + 64;
+                       (size_t)2 * g->S_pad * sizeof(float2) + (size_t)(g->nbeta + 3) * 4 + 8 * 64 * 4 + 64 + 128;
   // several consecutive K-slabs per stage so each row is fetched in longer
   // runs and the tensor cores get longer bursts per stage; keep at least
   // three stages in flight
@@ -192,19 +192,21 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
   const uint32_t b_bytes = (uint32_t)S_pad * 128u;
   const uint32_t st_bytes = (uint32_t)SL * (LM_A_BYTES + b_bytes);  // SL A slabs, then SL B slabs
   const int stages = a.stages;
-  // layout: stages | full | empty | tfull[2] | tempty[2] | epi | drain | tmem slot | scratch
+  // layout: stages | full | empty | tfull[2] | tempty[2] | tid[2] | epi | drain |
+  //         tmem slot, tile ring, accumulator tiles | scratch
   const uint32_t bar_full = base + stages * st_bytes;
   const uint32_t bar_empty = bar_full + 8 * stages;
   const uint32_t bar_tfull = bar_empty + 8 * stages;
   const uint32_t bar_tempty = bar_tfull + 16;
-  const uint32_t bar_epi = bar_tempty + 16;
+  const uint32_t bar_tid = bar_tempty + 16;
+  const uint32_t bar_epi = bar_tid + 16;
   const uint32_t bar_drain = bar_epi + 8;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + (bar_drain + 8 - base));
-  float2* wst = reinterpret_cast<float2*>(gbase + (bar_drain + 8 - base) + 16);  // [4][S_pad] per-warp stats
+  int32_t* tring = reinterpret_cast<int32_t*>(tmem_slot + 4);  // [LM_TRING] claimed tiles, producer -> MMA warp
+  int32_t* acc_tile = tring + LM_TRING;                        // [2] tile of each accumulator, MMA warp -> epilogue
+  float2* wst = reinterpret_cast<float2*>(gbase + (bar_drain + 8 - base) + 96);  // [4][S_pad] per-warp stats
   float2* wag = wst + 4 * S_pad;                                                  // [4][S_pad] per-warp argmax
-  float2* cst = wag + 4 * S_pad;   // [S_pad] running (max, sum) over this CTA's tiles
-  float2* carg = cst + S_pad;      // [S_pad] running (max u, argmax)
-  float* sbeta = reinterpret_cast<float*>(carg + S_pad);  // [nbeta]
+  float* sbeta = reinterpret_cast<float*>(wag + 6 * S_pad);  // [nbeta]
   float* bc = sbeta + ((a.nbeta + 3) & ~3);               // [8][64] per-warp column broadcast
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -216,6 +218,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_tfull + 8 * i, 1);
       mbar_init(bar_tempty + 8 * i, LM_EPI_THREADS);
+      mbar_init(bar_tid + 8 * i, 1);
     }
     mbar_init(bar_epi, LM_EPI_THREADS);
     mbar_init(bar_drain, 1);
@@ -230,10 +233,6 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     tmem_alloc(smem_u32(tmem_slot), a.tmem_cols);
     tmem_relinquish();
   }
-  for (int i = tid; i < S_pad; i += LM_THREADS) {
-    cst[i] = make_float2(-INFINITY, 0.f);
-    carg[i] = make_float2(-INFINITY, __int_as_float(0x7fffffff));
-  }
   if (a.mode == 1)
     for (int i = tid; i < a.nbeta; i += LM_THREADS) sbeta[i] = a.beta[i];
   tc_fence_before();
@@ -246,47 +245,64 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     // ---------------------------------------------------------------- TMA
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first(), pol_h = policy_evict_last();
-      // stage load i covers K-slabs (i % nst)*SL .. of tile blockIdx.x + (i / nst)*gridDim.x
-      const int my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
-      const uint32_t nloads = (uint32_t)my_tiles * (uint32_t)nst;
-      auto load_w = [&](uint32_t i) {
-        const uint32_t st = i % stages;
-        const int tile = (int)blockIdx.x + (int)(i / nst) * (int)gridDim.x, ks = (int)(i % nst);
+      // Tiles are claimed from a global counter, so CTAs that start early (as
+      // the previous kernel's CTAs leave their SMs) take more of them.  The
+      // claimed ids reach the MMA warp through tring (written before the
+      // arrive on the full barrier of the tile's first stage); -1 ends.
+      int tile = -1, ks = 0;
+      uint32_t tseq = 0;
+      auto claim = [&]() {
+        const int t = atomicAdd(a.tile_ctr, 1);
+        tile = t < ntiles ? t : -1;
+        tring[tseq % LM_TRING] = tile;
+        ++tseq;
+        ks = 0;
+      };
+      auto load_w = [&](uint32_t st) {
         const uint32_t fb = bar_full + 8 * st, sa = base + st * st_bytes;
         mbar_arrive_expect_tx(fb, st_bytes);
         // consecutive K-slabs of the same 128 rows back to back: longer runs per row
         for (int j = 0; j < SL; ++j)
           tma_load_2d(sa + j * LM_A_BYTES, &wmap, fb, (ks * SL + j) * LM_TILE_K, tile * LM_TILE_V, pol_w);
       };
-      auto load_h = [&](uint32_t i) {
-        const uint32_t st = i % stages;
-        const int ks = (int)(i % nst);
+      auto load_h = [&](uint32_t st, int kss) {
         const uint32_t fb = bar_full + 8 * st, sb = base + st * st_bytes + SL * LM_A_BYTES;
         for (int j = 0; j < SL; ++j)
           for (int c = 0; c < a.nchunk; ++c)
-            tma_load_2d(sb + j * b_bytes + c * a.chunk_n * 128, &hmap, fb, (ks * SL + j) * LM_TILE_K,
+            tma_load_2d(sb + j * b_bytes + c * a.chunk_n * 128, &hmap, fb, (kss * SL + j) * LM_TILE_K,
                         c * a.chunk_n, pol_h);
       };
+      claim();
+      uint32_t it = 0;
       // With programmatic dependent launch the weights of the first stages
       // stream while the previous kernel (which writes H) finishes.
-      uint32_t it = 0;
       if (a.pdl) {
-        const uint32_t npre = nloads < (uint32_t)stages ? nloads : (uint32_t)stages;
-        for (; it < npre; ++it) load_w(it);
+        int pre_ks[8];
+        while (tile >= 0 && it < (uint32_t)stages) {
+          load_w(it);
+          pre_ks[it++] = ks;
+          if (++ks == nst) claim();
+        }
         pdl_wait();
-        for (uint32_t i = 0; i < npre; ++i) load_h(i);
+        for (uint32_t i = 0; i < it; ++i) load_h(i, pre_ks[i]);
       }
       bool ok = true;
-      for (; it < nloads; ++it) {
+      while (tile >= 0) {
         const uint32_t st = it % stages, ph = (it / stages) & 1u;
         if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
           ok = false;
           break;
         }
-        load_w(it);
-        load_h(it);
+        load_w(st);
+        load_h(st, ks);
+        ++it;
+        if (++ks == nst) claim();
       }
-      if (!ok) {
+      if (ok) {
+        // end marker: a phase of the next stage's full barrier without data
+        const uint32_t st = it % stages, ph = (it / stages) & 1u;
+        if (mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) mbar_arrive(bar_full + 8 * st);
+      } else {
         for (uint32_t j = (it >= (uint32_t)stages ? it - stages : 0); j < it; ++j)
           mbar_wait(bar_full + 8 * (j % stages), (j / stages) & 1u, a.status);
       }
@@ -296,16 +312,32 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     // ---------------------------------------------------------------- MMA
     if (lane == 0) {
       const uint32_t idesc = umma_idesc_bf16(LM_TILE_V, a.chunk_n);
-      uint32_t it = 0, acc = 0;
+      uint32_t it = 0, acc = 0, tseq = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++acc) {
+      for (;; ++acc) {
         const uint32_t buf = acc % a.acc_bufs, aph = (acc / a.acc_bufs) & 1u;
-        if (!mbar_wait(bar_tempty + 8 * buf, aph ^ 1u, a.status)) break;
+        // the next tile's first stage (or the end marker) tells which tile it is
+        {
+          const uint32_t st = it % stages, ph = (it / stages) & 1u;
+          if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
+            ok = false;
+            break;
+          }
+        }
+        const int tile = tring[tseq % LM_TRING];
+        ++tseq;
+        if (!mbar_wait(bar_tempty + 8 * buf, aph ^ 1u, a.status)) {
+          ok = false;
+          break;
+        }
+        acc_tile[buf] = tile;
+        mbar_arrive(bar_tid + 8 * buf);
+        if (tile < 0) break;
         tc_fence_after();
         const uint32_t dcol = tmem_base + buf * S_pad;
         for (int ks = 0; ks < nst; ++ks, ++it) {
           const uint32_t st = it % stages, ph = (it / stages) & 1u;
-          if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
+          if (ks > 0 && !mbar_wait(bar_full + 8 * st, ph, a.status)) {
             ok = false;
             break;
           }
@@ -349,14 +381,13 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int etid = tid - 64, half = (warp - 2) >> 2;
     const int S = a.S, n1 = a.N + 1;
-    uint32_t acc = 0, ephase = 0;
-    bool ok = true;
-    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++acc) {
+    uint32_t ephase = 0;
+    for (uint32_t acc = 0;; ++acc) {
       const uint32_t buf = acc % a.acc_bufs, aph = (acc / a.acc_bufs) & 1u;
-      if (!mbar_wait(bar_tfull + 8 * buf, aph, a.status)) {
-        ok = false;
-        break;
-      }
+      if (!mbar_wait(bar_tid + 8 * buf, aph, a.status)) break;
+      const int tile = acc_tile[buf];
+      if (tile < 0) break;
+      if (!mbar_wait(bar_tfull + 8 * buf, aph, a.status)) break;
       tc_fence_after();
       const int v = tile * LM_TILE_V + 32 * q + lane;
       const bool valid = v < a.V;
@@ -377,41 +408,30 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       }
       tc_fence_before();
       mbar_arrive(bar_tempty + 8 * buf);
-      if (!bar_sync_bounded(bar_epi, ephase, a.status)) {
-        ok = false;
-        break;
-      }
-      // fold the four warps' results into this CTA's running records
+      if (!bar_sync_bounded(bar_epi, ephase, a.status)) break;
+      // this tile's records: the four lane quarters' results folded in a fixed
+      // order, stored per tile so the cross-tile merge order does not depend
+      // on which CTA took the tile
       for (int col = etid; col < S; col += LM_EPI_THREADS) {
-        float2 c = cst[col];
+        float cm = -INFINITY, cs = 0.f;
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq) {
           const float2 r = wst[qq * S_pad + col];
-          lse_merge(c.x, c.y, r.x, r.y);
+          lse_merge(cm, cs, r.x, r.y);
         }
-        cst[col] = c;
+        a.rec_stats[(int64_t)col * ntiles + tile] = make_float2(cm, cs);
         if (a.mode == 1 && col % n1 != 0) {
-          float bu = carg[col].x;
-          int bv = __float_as_int(carg[col].y);
+          float bu = -INFINITY;
+          int bv = 0x7fffffff;
 #pragma unroll
           for (int qq = 0; qq < 4; ++qq) {
             const float2 r = wag[qq * S_pad + col];
             argmax_merge(bu, bv, r.x, __float_as_int(r.y));
           }
-          carg[col] = make_float2(bu, __int_as_float(bv));
+          a.rec_arg[(int64_t)col * ntiles + tile] = make_float2(bu, __int_as_float(bv));
         }
       }
-      if (!bar_sync_bounded(bar_epi, ephase, a.status)) {
-        ok = false;
-        break;
-      }
-    }
-    if (ok) {
-      const int nrec = gridDim.x;
-      for (int col = etid; col < S; col += LM_EPI_THREADS) {
-        a.rec_stats[(int64_t)col * nrec + blockIdx.x] = cst[col];
-        if (a.mode == 1 && col % n1 != 0) a.rec_arg[(int64_t)col * nrec + blockIdx.x] = carg[col];
-      }
+      if (!bar_sync_bounded(bar_epi, ephase, a.status)) break;
     }
   }
   tc_fence_before();
@@ -481,95 +501,130 @@ cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float
 }
 
 // ------------------------------------------- Eq. 2 + Eq. 3 from tile records
-// Per query: L_j for its N+1 rows from the (max, sum) records; for each expert
-// k the best tile record of u_k; score_k = u_k* + c_k; the best (score desc,
-// token asc, expert asc) wins.
-__global__ void __launch_bounds__(256) select_from_records_kernel(SelectArgs a) {
-  const int b = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int N = a.N, n1 = N + 1, s0 = b * n1, T = a.nrec;
-  if (a.pdl) pdl_wait();  // the LM head's records are complete and visible
-  __shared__ float Ls[LM_MAX_N1];
-  __shared__ float ksc[LM_MAX_N1];
-  __shared__ int ktok[LM_MAX_N1];
-  __shared__ int t_step;
-  if (tid == 0) t_step = a.step ? *a.step : 0;
-  for (int j = warp; j < n1; j += 8) {
-    const int s = s0 + j;
-    float M = -INFINITY, sum = 0.f;
-    for (int t = lane; t < T; t += 32) {
-      const float2 r = a.rec_stats[(int64_t)s * T + t];
-      lse_merge(M, sum, r.x, r.y);
-    }
+// One CTA per row s = b*(N+1) + j: L_s from the row's tile records and, for an
+// expert row (j > 0), the best tile record of u_k; the last CTA of query b to
+// finish forms score_k = u_k* + c_k and picks the best (score desc, token
+// asc, expert asc).  Every reduction runs in a fixed order (thread t takes
+// records t, t + 256, ... in four interleaved chains, then a fixed tree), so
+// the result does not depend on timing.
+constexpr int SEL_R_THREADS = 256;
+
+__device__ __forceinline__ void lse_block(const float2* rec, int T, int tid, float2* red, float& L) {
+  float m[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY}, su[4] = {0.f, 0.f, 0.f, 0.f};
+  int t = tid;
+  for (; t + 3 * SEL_R_THREADS < T; t += 4 * SEL_R_THREADS) {
+    float2 r[4];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float m2 = __shfl_xor_sync(0xffffffffu, M, o), s2 = __shfl_xor_sync(0xffffffffu, sum, o);
-      lse_merge(M, sum, m2, s2);
-    }
-    if (lane == 0) {
-      Ls[j] = M + logf(sum);
-      if (a.lse_out) a.lse_out[s] = Ls[j];
-    }
+    for (int k = 0; k < 4; ++k) r[k] = rec[t + k * SEL_R_THREADS];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) lse_merge(m[k], su[k], r[k].x, r[k].y);
   }
+  for (; t < T; t += SEL_R_THREADS) {
+    const float2 r = rec[t];
+    lse_merge(m[0], su[0], r.x, r.y);
+  }
+#pragma unroll
+  for (int k = 1; k < 4; ++k) lse_merge(m[0], su[0], m[k], su[k]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m[0], o), s2 = __shfl_xor_sync(0xffffffffu, su[0], o);
+    lse_merge(m[0], su[0], m2, s2);
+  }
+  if ((tid & 31) == 0) red[tid >> 5] = make_float2(m[0], su[0]);
   __syncthreads();
-  for (int k = 1 + warp; k <= N; k += 8) {
-    const int s = s0 + k;
+  if (tid == 0) {
+    float M = -INFINITY, Sm = 0.f;
+    for (int w = 0; w < SEL_R_THREADS / 32; ++w) lse_merge(M, Sm, red[w].x, red[w].y);
+    L = M + logf(Sm);
+  }
+}
+
+__global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(SelectArgs a) {
+  const int j = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int N = a.N, n1 = N + 1, s = b * n1 + j, T = a.nrec;
+  if (a.pdl) pdl_wait();  // the LM head's records are complete and visible
+  if (j == 0 && b == 0 && tid == 0 && a.tile_ctr) *a.tile_ctr = 0;  // the next LM head claims its tiles from 0
+  __shared__ float2 red[SEL_R_THREADS / 32];
+  __shared__ float sv[SEL_R_THREADS / 32];
+  __shared__ int si[SEL_R_THREADS / 32];
+  __shared__ int last;
+  float L = 0.f;
+  lse_block(a.rec_stats + (int64_t)s * T, T, tid, red, L);
+  if (j > 0) {
+    const float2* rec = a.rec_arg + (int64_t)s * T;
     float bu = -INFINITY;
     int bv = 0x7fffffff;
-    for (int t = lane; t < T; t += 32) {
-      const float2 r = a.rec_arg[(int64_t)s * T + t];
+    for (int t = tid; t < T; t += SEL_R_THREADS) {
+      const float2 r = rec[t];
       argmax_merge(bu, bv, r.x, __float_as_int(r.y));
     }
     warp_argmax(bu, bv);
     if (lane == 0) {
-      const float bt = a.beta[b * N + k - 1];
-      const float rr = fminf(fmaxf(a.r[b * N + k - 1], 1e-8f), 1.0f);
-      const float c = -(1.f + bt) * Ls[k] + bt * Ls[0] + a.gamma * logf(rr);
-      ksc[k - 1] = bu + c;
-      ktok[k - 1] = bv;
+      sv[warp] = bu;
+      si[warp] = bv;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 1; w < SEL_R_THREADS / 32; ++w) argmax_merge(bu, bv, sv[w], si[w]);
+      a.sel_u[s] = bu;
+      a.sel_tok[s] = bv;
     }
   }
+  if (tid == 0) {
+    a.sel_L[s] = L;
+    if (a.lse_out) a.lse_out[s] = L;
+    __threadfence();
+    last = atomicAdd(a.qdone + b, 1) == n1 - 1;
+  }
   __syncthreads();
-  if (warp == 0) {
-    float bs = -INFINITY;
-    int bt = 0x7fffffff, bk = 0x7fffffff;
-    for (int k = lane; k < N; k += 32) {
-      const float sc = ksc[k];
-      const int tk = ktok[k];
-      if (sc > bs || (sc == bs && (tk < bt || (tk == bt && k < bk)))) {
-        bs = sc;
-        bt = tk;
-        bk = k;
-      }
+  if (!last) return;
+  __threadfence();  // the other rows' results of query b are visible
+  if (warp != 0) return;
+  const float L0 = __ldcg(a.sel_L + b * n1);
+  float bs = -INFINITY;
+  int bt = 0x7fffffff, bk = 0x7fffffff;
+  for (int k = lane; k < N; k += 32) {
+    const int sk = b * n1 + 1 + k;
+    const float btk = a.beta[b * N + k];
+    const float rr = fminf(fmaxf(a.r[b * N + k], 1e-8f), 1.0f);
+    const float c = -(1.f + btk) * __ldcg(a.sel_L + sk) + btk * L0 + a.gamma * logf(rr);
+    const float sc = __ldcg(a.sel_u + sk) + c;
+    const int tk = __ldcg(a.sel_tok + sk);
+    if (sc > bs || (sc == bs && (tk < bt || (tk == bt && k < bk)))) {
+      bs = sc;
+      bt = tk;
+      bk = k;
     }
+  }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float s2 = __shfl_xor_sync(0xffffffffu, bs, o);
-      const int t2 = __shfl_xor_sync(0xffffffffu, bt, o), k2 = __shfl_xor_sync(0xffffffffu, bk, o);
-      if (s2 > bs || (s2 == bs && (t2 < bt || (t2 == bt && k2 < bk)))) {
-        bs = s2;
-        bt = t2;
-        bk = k2;
-      }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float s2 = __shfl_xor_sync(0xffffffffu, bs, o);
+    const int t2 = __shfl_xor_sync(0xffffffffu, bt, o), k2 = __shfl_xor_sync(0xffffffffu, bk, o);
+    if (s2 > bs || (s2 == bs && (t2 < bt || (t2 == bt && k2 < bk)))) {
+      bs = s2;
+      bt = t2;
+      bk = k2;
     }
-    if (lane == 0) {
-      if (a.token) a.token[b] = bt;
-      if (a.expert) a.expert[b] = bk + 1;
-      if (a.score) a.score[b] = bs;
-      if (a.step) {
-        const int t = t_step;
-        if (t >= 0 && t < a.max_steps) {
-          a.history[(int64_t)b * a.max_steps + t] = bt;
-          if (a.expert_trace) a.expert_trace[(int64_t)b * a.max_steps + t] = bk + 1;
-          if (a.score_trace) a.score_trace[(int64_t)b * a.max_steps + t] = bs;
-        } else {
-          dev_flag(a.status, PCED_DEV_STEP_LIMIT);
-        }
+  }
+  if (lane == 0) {
+    a.qdone[b] = 0;
+    if (a.token) a.token[b] = bt;
+    if (a.expert) a.expert[b] = bk + 1;
+    if (a.score) a.score[b] = bs;
+    if (a.step) {
+      const int t = *a.step;
+      if (t >= 0 && t < a.max_steps) {
+        a.history[(int64_t)b * a.max_steps + t] = bt;
+        if (a.expert_trace) a.expert_trace[(int64_t)b * a.max_steps + t] = bk + 1;
+        if (a.score_trace) a.score_trace[(int64_t)b * a.max_steps + t] = bs;
+      } else {
+        dev_flag(a.status, PCED_DEV_STEP_LIMIT);
+      }
+      __threadfence();
+      if (atomicAdd(a.done_counter, 1) == a.B - 1) {
+        *a.step = t + 1;
+        *a.done_counter = 0;
         __threadfence();
-        if (atomicAdd(a.done_counter, 1) == a.B - 1) {
-          *a.step = t + 1;
-          *a.done_counter = 0;
-          __threadfence();
-        }
       }
     }
   }
@@ -577,8 +632,8 @@ __global__ void __launch_bounds__(256) select_from_records_kernel(SelectArgs a) 
 
 cudaError_t select_from_records_launch(const SelectArgs& a, cudaStream_t stream) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.B);
-  cfg.blockDim = dim3(256);
+  cfg.gridDim = dim3(a.N + 1, a.B);
+  cfg.blockDim = dim3(SEL_R_THREADS);
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -639,14 +694,17 @@ extern "C" pced_status pced_lm_head_logprobs(const void* hidden, const void* w_u
   a.chunk_n = g.chunk_n;
   a.tmem_cols = g.tmem_cols;
   a.logits = logprobs;
-  a.rec_stats = cv.take<float2>((size_t)S * g.grid);
+  a.rec_stats = cv.take<float2>((size_t)S * g.ntiles);
   a.rec_arg = nullptr;
   a.beta = nullptr;
   a.status = (int*)workspace;
+  a.tile_ctr = (int*)workspace + 1;  // tile counter, zeroed here
   cudaStream_t s = (cudaStream_t)stream;
-  cudaError_t e = lm_head_launch(wmap, hmap, g, a, s);
+  cudaError_t e = cudaMemsetAsync(a.tile_ctr, 0, sizeof(int), s);
+  if (e != cudaSuccess) return cuda_status(e, "lm head tile counter");
+  e = lm_head_launch(wmap, hmap, g, a, s);
   if (e != cudaSuccess) return cuda_status(e, "lm head launch");
-  e = lm_lse_finalize_launch(logprobs, a.rec_stats, lse, S, V, g.grid, s);
+  e = lm_lse_finalize_launch(logprobs, a.rec_stats, lse, S, V, g.ntiles, s);
   if (e != cudaSuccess) return cuda_status(e, "lse finalize launch");
   return PCED_OK;
 }

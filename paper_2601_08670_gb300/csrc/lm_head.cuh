@@ -11,6 +11,7 @@ constexpr int LM_TILE_V = 128;   // vocabulary rows per tile (UMMA M)
 constexpr int LM_TILE_K = 64;    // hidden elements per stage (one 128-byte swizzle row)
 constexpr int LM_MAX_S = 512;
 constexpr int LM_MAX_N1 = 256;   // experts + amateur per query in the selection kernels
+constexpr int LM_TRING = 16;     // claimed-tile ring between the TMA and MMA warps (> stages + 2 tiles in flight)
 
 struct LmGeom {
   int32_t S, S_pad, nchunk, chunk_n, d, V, ntiles, nks, slabs, nst, stages, acc_bufs, grid, nbeta;
@@ -25,8 +26,9 @@ struct LmArgs {
   int32_t S, N, V, ntiles, nks, slabs, nst, stages, acc_bufs, S_pad, nchunk, chunk_n, nbeta;
   uint32_t tmem_cols;
   float* logits;      // mode 0
-  float2* rec_stats;  // [S][grid] (max z, sum exp(z - max)) over each CTA's tiles
-  float2* rec_arg;    // [S][grid] (max u, argmax v as int bits) for expert columns, mode 1
+  float2* rec_stats;  // [S][ntiles] (max z, sum exp(z - max)) of each vocabulary tile
+  float2* rec_arg;    // [S][ntiles] (max u, argmax v as int bits) for expert columns, mode 1
+  int* tile_ctr;      // tiles claimed so far (zero at launch)
   const float* beta;  // [B][N]
   int pdl;            // launched as a programmatic dependent of the kernel that writes H
   int* status;
@@ -34,7 +36,7 @@ struct LmArgs {
 
 cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, const LmGeom& g, const LmArgs& a,
                            cudaStream_t stream);
-// mode-0 finish: lse[s] from the CTA records, logits -> log-probs in place
+// mode-0 finish: lse[s] from the tile records, logits -> log-probs in place
 cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float* lse, int32_t S, int32_t V,
                                    int32_t nrec, cudaStream_t stream);
 
@@ -42,7 +44,8 @@ cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float
 struct SelectArgs {
   const float2* rec_stats;
   const float2* rec_arg;
-  int32_t B, N, nrec;  // records per row (the LM-head grid size)
+  int32_t B, N, nrec;  // records per row (the LM head's vocabulary tiles)
+  int* tile_ctr;       // optional: the LM head's tile counter, reset here for its next launch
   const float* beta;
   const float* r;
   float gamma;
@@ -57,6 +60,12 @@ struct SelectArgs {
   float* score_trace;
   int32_t max_steps;
   int32_t* done_counter;
+  // per-row results and per-query counters (zero at the first launch; the
+  // last CTA of a query resets its counter)
+  float* sel_L;       // [S] log-sum-exp of each row
+  float* sel_u;       // [S] best u_k of each expert row
+  int32_t* sel_tok;   // [S] its token
+  int32_t* qdone;     // [B] rows of the query finished
   int pdl;            // launched as a programmatic dependent of the LM head
   int* status;
 };

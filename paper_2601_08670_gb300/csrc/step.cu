@@ -21,6 +21,11 @@ struct StepLayout {
   int32_t* done_counter;  // selection kernel: queries finished this step
   int32_t* att_done;      // attention: CTAs finished
   int32_t* att_epoch;     // attention: launches completed
+  int32_t* lm_tile_ctr;   // LM head: vocabulary tiles claimed (reset by the selection)
+  int32_t* sel_qdone;     // selection: rows finished per query
+  float* sel_L;
+  float* sel_u;
+  int32_t* sel_tok;
   uint64_t* part_ss;
   uint64_t* resid;
   uint64_t* rec_o;
@@ -48,6 +53,11 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   L.h = c.take<__nv_bfloat16>((size_t)S * d);
   L.lm_stats = c.take<float2>((size_t)(S * ntiles));
   L.lm_arg = c.take<float2>((size_t)(S * ntiles));
+  L.lm_tile_ctr = c.take<int32_t>(1);
+  L.sel_qdone = c.take<int32_t>((size_t)dm->B);
+  L.sel_L = c.take<float>((size_t)S);
+  L.sel_u = c.take<float>((size_t)S);
+  L.sel_tok = c.take<int32_t>((size_t)S);
   L.bytes = c.used();
   return L;
 }
@@ -180,6 +190,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.tmem_cols = g.tmem_cols;
   la.rec_stats = W.lm_stats;
   la.rec_arg = W.lm_arg;
+  la.tile_ctr = W.lm_tile_ctr;
   la.beta = p->beta;
   la.status = W.status;
   la.pdl = timed ? 0 : 1;  // stage events between the launches would break the overlap
@@ -192,7 +203,12 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.rec_arg = W.lm_arg;
   sa.B = dm.B;
   sa.N = dm.N;
-  sa.nrec = g.grid;
+  sa.nrec = g.ntiles;
+  sa.tile_ctr = W.lm_tile_ctr;
+  sa.sel_L = W.sel_L;
+  sa.sel_u = W.sel_u;
+  sa.sel_tok = W.sel_tok;
+  sa.qdone = W.sel_qdone;
   sa.beta = p->beta;
   sa.r = p->r;
   sa.gamma = p->gamma;
