@@ -355,9 +355,12 @@ struct Carver {
   char* base;
   size_t off = 0;
   explicit Carver(void* b) : base((char*)b) {}
+  // `align` applies to the address (the base itself is only 256-byte
+  // aligned): sizes computed without a base need up to align - 256 spare
+  // bytes per such take
   template <typename T>
-  T* take(size_t count) {
-    off = align_up(off, 256);
+  T* take(size_t count, size_t align = 256) {
+    off = align_up((size_t)(uintptr_t)base + off, align) - (size_t)(uintptr_t)base;
     T* p = base ? (T*)(base + off) : nullptr;
     off += count * sizeof(T);
     return p;
