@@ -65,6 +65,10 @@ def lib():
         L.oracle_decode_step.argtypes = [ctypes.POINTER(_Dims), P, P, I64, P, P, P, P, P, P, P, P, P, P, P, P,
                                          P, P, I32]
         L.oracle_decode_step.restype = I32
+        L.oracle_decode_step_ex.argtypes = list(L.oracle_decode_step.argtypes[:-1]) + [P, I32]
+        L.oracle_decode_step_ex.restype = I32
+        L.oracle_adacad_beta.argtypes = [P, I32, I32, I32, P]
+        L.oracle_adacad_beta.restype = I32
         _lib = L
     return _lib
 
@@ -149,8 +153,24 @@ def contrastive_select(lp, beta, r, gamma, B, N):
     return dict(token=tok, expert=exp_, score=sc, token_gap=tg, expert_gap=eg)
 
 
-def decode_step(dims: dict, kc, vc, layer_elems, kv_off, cap, lens, emb_rows, w_bits, beta, r):
-    """One full decode step; kc, vc and lens are updated in place."""
+def adacad_beta(lp, B, N):
+    """Dynamic contrast strength (Sec. 3 after Eq. 2, as in AdaCAD): per
+    expert, the Jensen-Shannon divergence in bits between its distribution
+    exp(lp_k) and the amateur's exp(lp_0).  lp: [B*(N+1), V]; returns [B, N]."""
+    lp = _c(lp, np.float64)
+    V = lp.shape[1]
+    out = np.empty((B, N), np.float64)
+    rc = lib().oracle_adacad_beta(_p(lp), B, N, V, _p(out))
+    if rc != 0:
+        raise ValueError(f"oracle_adacad_beta rc={rc}")
+    return out
+
+
+def decode_step(dims: dict, kc, vc, layer_elems, kv_off, cap, lens, emb_rows, w_bits, beta, r,
+                dynamic_beta: bool = False):
+    """One full decode step; kc, vc and lens are updated in place.  With
+    dynamic_beta the contrast strengths come from this step's distributions
+    (adacad_beta, rounded to fp32; returned as "beta")."""
     dm = _Dims(dims["B"], dims["N"], dims["L"], dims["Hq"], dims["Hkv"], dims["D"], dims["V"],
                float(dims["gamma"]), float(dims.get("rms_eps", RMS_EPS)),
                float(dims.get("attn_scale", 1.0 / math.sqrt(dims["D"]))))
@@ -165,10 +185,14 @@ def decode_step(dims: dict, kc, vc, layer_elems, kv_off, cap, lens, emb_rows, w_
     eg = np.empty(B, np.float64)
     h = np.empty((S, d), np.uint16)
     lse = np.empty(S, np.float64)
-    rc = lib().oracle_decode_step(ctypes.byref(dm), _p(kc), _p(vc), int(layer_elems), _p(_c(kv_off, np.int64)),
-                                  _p(_c(cap, np.int32)), _p(lens), _p(_c(emb_rows, np.uint16)),
-                                  _p(_c(w_bits, np.uint16)), _p(_c(beta, np.float32)), _p(_c(r, np.float32)),
-                                  _p(tok), _p(exp_), _p(sc), _p(tg), _p(eg), _p(h), _p(lse), threads())
+    bdyn = np.empty((B, N), np.float32) if dynamic_beta else None
+    rc = lib().oracle_decode_step_ex(ctypes.byref(dm), _p(kc), _p(vc), int(layer_elems), _p(_c(kv_off, np.int64)),
+                                     _p(_c(cap, np.int32)), _p(lens), _p(_c(emb_rows, np.uint16)),
+                                     _p(_c(w_bits, np.uint16)), _p(_c(beta, np.float32)), _p(_c(r, np.float32)),
+                                     _p(tok), _p(exp_), _p(sc), _p(tg), _p(eg), _p(h), _p(lse), _p(bdyn), threads())
     if rc != 0:
         raise ValueError(f"oracle_decode_step rc={rc}")
-    return dict(token=tok, expert=exp_, score=sc, token_gap=tg, expert_gap=eg, h=h, lse=lse)
+    out = dict(token=tok, expert=exp_, score=sc, token_gap=tg, expert_gap=eg, h=h, lse=lse)
+    if dynamic_beta:
+        out["beta"] = bdyn
+    return out

@@ -232,6 +232,29 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
   return 0;
 }
 
+/* ------------------------------------- dynamic contrast strength (AdaCAD) */
+
+int32_t oracle_adacad_beta(const double* lp, int32_t B, int32_t N, int32_t V, double* beta) {
+  if (!lp || !beta || B < 1 || N < 1 || V < 1) return -1;
+  for (int32_t b = 0; b < B; ++b) {
+    const double* lp0 = lp + (int64_t)b * (N + 1) * V; /* amateur row */
+    for (int32_t k = 1; k <= N; ++k) {
+      const double* lpk = lp + ((int64_t)b * (N + 1) + k) * V;
+      /* Jensen-Shannon divergence in bits: the mean of the two
+       * Kullback-Leibler divergences to the midpoint distribution */
+      double kl_k = 0.0, kl_0 = 0.0;
+      for (int32_t v = 0; v < V; ++v) {
+        double pk = exp(lpk[v]), p0 = exp(lp0[v]);
+        double m = 0.5 * (pk + p0);
+        if (pk > 0.0) kl_k += pk * log2(pk / m);
+        if (p0 > 0.0) kl_0 += p0 * log2(p0 / m);
+      }
+      beta[(int64_t)b * N + (k - 1)] = 0.5 * (kl_k + kl_0);
+    }
+  }
+  return 0;
+}
+
 /* ------------------------------------------------------------- full step */
 
 int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, int64_t layer_elems,
@@ -239,6 +262,15 @@ int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, in
                            const uint16_t* w, const float* beta, const float* r, int32_t* token, int32_t* expert,
                            double* score, double* token_gap, double* expert_gap, uint16_t* h_out, double* lse_out,
                            int32_t nthreads) {
+  return oracle_decode_step_ex(dm, kc, vc, layer_elems, kv_off, cap, len, emb_rows, w, beta, r, token, expert,
+                               score, token_gap, expert_gap, h_out, lse_out, NULL, nthreads);
+}
+
+int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, int64_t layer_elems,
+                              const int64_t* kv_off, const int32_t* cap, int32_t* len, const uint16_t* emb_rows,
+                              const uint16_t* w, const float* beta, const float* r, int32_t* token, int32_t* expert,
+                              double* score, double* token_gap, double* expert_gap, uint16_t* h_out,
+                              double* lse_out, float* beta_dyn, int32_t nthreads) {
   if (!dm || !kc || !vc || !kv_off || !cap || !len || !emb_rows || !w || !beta || !r || !token || !expert ||
       !score)
     return -1;
@@ -292,8 +324,23 @@ int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, in
 
   oracle_lm_head_logprobs(u, w, S, d, V, lp, lse, nthreads);
   if (lse_out) memcpy(lse_out, lse, sizeof(double) * (size_t)S);
-  oracle_contrastive_select(lp, beta, r, dm->gamma, B, N, V, token, expert, score, token_gap, expert_gap);
+  int32_t rc = 0;
+  if (beta_dyn) {
+    /* first generated token of a dynamic-beta run: beta from this step's
+     * distributions, rounded to the fp32 the selection takes */
+    double* bd = (double*)malloc(sizeof(double) * (size_t)B * N);
+    if (!bd) {
+      rc = -1;
+    } else {
+      oracle_adacad_beta(lp, B, N, V, bd);
+      for (int64_t i = 0; i < (int64_t)B * N; ++i) beta_dyn[i] = (float)bd[i];
+      free(bd);
+      beta = beta_dyn;
+    }
+  }
+  if (rc == 0)
+    oracle_contrastive_select(lp, beta, r, dm->gamma, B, N, V, token, expert, score, token_gap, expert_gap);
 
   free(x); free(xn); free(u); free(o); free(lp); free(lse);
-  return 0;
+  return rc;
 }

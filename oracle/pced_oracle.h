@@ -53,6 +53,15 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
                                   int32_t N, int32_t V, int32_t* token, int32_t* expert, double* score,
                                   double* token_gap, double* expert_gap);
 
+/* Dynamic contrast strength (Sec. 3 after Eq. 2: beta_0 is computed as in
+ * AdaCAD for the first generated token and kept fixed thereafter).  Reading
+ * used here: one beta per contextual expert, the Jensen-Shannon divergence in
+ * bits between the expert's next-token distribution and the amateur's,
+ *   beta[b][k-1] = 1/2 sum_v [ p_k(v) log2(p_k(v)/m(v)) + p_0(v) log2(p_0(v)/m(v)) ],
+ *   m = (p_k + p_0)/2,  p = exp(lp),  terms with p = 0 contribute 0,
+ * so 0 <= beta <= 1.  lp [S][V] as in oracle_contrastive_select. */
+int32_t oracle_adacad_beta(const double* lp, int32_t B, int32_t N, int32_t V, double* beta);
+
 typedef struct oracle_dims {
   int32_t B, N, L, Hq, Hkv, D, V; /* S = B*(N+1), d = Hq*D, requires 2*Hkv <= Hq */
   double gamma;                   /* retrieval-prior weight of Eq. 2 */
@@ -76,6 +85,15 @@ int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, in
                            const uint16_t* w, const float* beta, const float* r, int32_t* token, int32_t* expert,
                            double* score, double* token_gap, double* expert_gap, uint16_t* h_out, double* lse_out,
                            int32_t nthreads);
+/* The same step; when beta_dyn is not NULL the contrast strengths are not
+ * taken from `beta` but computed from this step's log-probabilities with
+ * oracle_adacad_beta, rounded to fp32, stored in beta_dyn [B][N] and used for
+ * the selection (the first generated token of a dynamic-beta run). */
+int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, int64_t layer_elems,
+                              const int64_t* kv_off, const int32_t* cap, int32_t* len, const uint16_t* emb_rows,
+                              const uint16_t* w, const float* beta, const float* r, int32_t* token, int32_t* expert,
+                              double* score, double* token_gap, double* expert_gap, uint16_t* h_out,
+                              double* lse_out, float* beta_dyn, int32_t nthreads);
 
 #ifdef __cplusplus
 }

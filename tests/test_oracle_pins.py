@@ -418,3 +418,78 @@ def test_kv_storage_example_from_paper():
     total = per_tok * g["passages"] * g["tokens_per_passage"]
     assert per_tok == 128 * 1024
     assert abs(total / 2 ** 30 - g["reported_gb"]) < 0.005
+
+
+# ------------------------------------------ dynamic contrast strength (AdaCAD)
+# beta_k = Jensen-Shannon divergence in bits between expert k's and the
+# amateur's next-token distributions (the reading of "computed as in AdaCAD").
+def _rows_from_probs(*rows):
+    """log-probability rows (-inf where p = 0) of the given probability rows"""
+    with np.errstate(divide="ignore"):
+        return np.log(np.array(rows, np.float64))
+
+
+def test_adacad_beta_identical_distributions_is_zero():
+    p = rng0.dirichlet(np.ones(40))
+    beta = oracle.adacad_beta(_rows_from_probs(p, p), 1, 1)
+    assert abs(beta[0, 0]) < 1e-15
+
+
+def test_adacad_beta_disjoint_supports_is_one_bit():
+    amateur = np.zeros(6)
+    amateur[1] = 1.0
+    expert = np.zeros(6)
+    expert[4] = 1.0
+    beta = oracle.adacad_beta(_rows_from_probs(amateur, expert), 1, 1)
+    assert beta[0, 0] == pytest.approx(1.0, abs=1e-15)
+
+
+def test_adacad_beta_two_point_closed_form():
+    # expert (1, 0) against amateur (1/2, 1/2): the midpoint is (3/4, 1/4), so
+    # JSD = H(3/4, 1/4) - (H(expert) + H(amateur)) / 2 = (2 - 3/4 log2 3) - 1/2
+    beta = oracle.adacad_beta(_rows_from_probs([0.5, 0.5], [1.0, 0.0]), 1, 1)
+    assert beta[0, 0] == pytest.approx(1.5 - 0.75 * math.log2(3.0), abs=1e-14)
+
+
+def test_adacad_beta_matches_entropy_form_is_symmetric_and_bounded():
+    def H(p):
+        p = p[p > 0]
+        return float(-(p * np.log2(p)).sum())
+    for trial in range(5):
+        V = int(rng0.integers(2, 300))
+        p = rng0.dirichlet(np.full(V, 0.3))
+        q = rng0.dirichlet(np.full(V, 0.3))
+        b_pq = oracle.adacad_beta(_rows_from_probs(q, p), 1, 1)[0, 0]
+        b_qp = oracle.adacad_beta(_rows_from_probs(p, q), 1, 1)[0, 0]
+        assert b_pq == pytest.approx(H(0.5 * (p + q)) - 0.5 * (H(p) + H(q)), abs=1e-12)
+        assert b_pq == pytest.approx(b_qp, abs=1e-14)
+        assert 0.0 <= b_pq <= 1.0
+
+
+def test_adacad_beta_row_layout_per_query_and_expert():
+    # query-major rows, the amateur first: beta[b][k-1] compares row b*(N+1)+k with row b*(N+1)
+    B, N, V = 2, 3, 17
+    probs = [rng0.dirichlet(np.ones(V)) for _ in range(B * (N + 1))]
+    beta = oracle.adacad_beta(_rows_from_probs(*probs), B, N)
+    for b in range(B):
+        for k in range(1, N + 1):
+            single = oracle.adacad_beta(_rows_from_probs(probs[b * (N + 1)], probs[b * (N + 1) + k]), 1, 1)
+            assert beta[b, k - 1] == single[0, 0]
+
+
+def test_step_with_dynamic_beta_uses_the_first_step_distributions():
+    # the step's beta is the divergence of this step's own distributions, and
+    # the selection of that step is Eq. 2 + Eq. 3 with it
+    from oracle.run import OracleRun
+    w = synth.get("tiny")
+    run = OracleRun(w, dynamic_beta=True)
+    out = run.step()
+    lp, _ = oracle.lm_head_logprobs(out["h"], run.w_bits)
+    want = oracle.adacad_beta(lp, w.B, w.N).astype(np.float32)
+    assert np.array_equal(out["beta"], want)
+    sel = oracle.contrastive_select(lp, want, run.r, w.gamma, w.B, w.N)
+    assert np.array_equal(sel["token"], out["token"]) and np.array_equal(sel["expert"], out["expert"])
+    # later steps keep it
+    assert np.array_equal(run.beta, want)
+    run.step()
+    assert np.array_equal(run.beta, want)
