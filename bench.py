@@ -43,6 +43,8 @@ def parse_args():
     p.add_argument("--secondary", default="llama32", help="second workload timed on the value path ('none' skips)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-dynamic-beta", action="store_true",
+                   help="skip timing the first step with dynamic contrast strength")
     p.add_argument("--profile-steps", type=int, default=4, help="replays with per-launch events (roofline)")
     return p.parse_args()
 
@@ -288,6 +290,38 @@ def run_e2e(dec, w, dev, steps):
     return el, h2d, d2h
 
 
+def time_dynamic_beta_first_step(w, dev, reps=3):
+    """Device time of the first step of a decode with dynamic contrast strength
+    and of the regular step after it (eager calls, CUDA events), median of
+    `reps` fresh decoders."""
+    import torch
+    import paper_2601_08670_gb300 as pced
+    import synth
+    S = w.B * (w.N + 1)
+    pced.adacad_beta(torch.zeros((S, w.V), dtype=torch.float32, device=dev), w.B, w.N)  # load the kernel
+    first, regular, status = [], [], 0
+    for _ in range(reps):
+        t = synth.device_inputs(w, dev, extra_steps=4)
+        dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
+        dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=4, bos=w.bos, dynamic_beta=True)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        torch.cuda.synchronize()
+        ev[0].record()
+        dec.step()
+        ev[1].record()
+        dec.step()
+        ev[2].record()
+        torch.cuda.synchronize()
+        first.append(ev[0].elapsed_time(ev[1]) * 1e3)
+        regular.append(ev[1].elapsed_time(ev[2]) * 1e3)
+        status |= dec.status()
+        del dec, t
+    f, r = statistics.median(first), statistics.median(regular)
+    return {"first_step_us": f, "next_step_us": r, "extra_us": f - r, "reps": reps,
+            "path": "pced_step with beta_from_step: LM head writes the log-probs, pced_adacad_beta kernel, "
+                    "then the fused LM head and selection with that beta"}, status
+
+
 def cpu_baseline(w, budget_s=20.0, max_steps=3):
     import oracle
     from oracle.run import OracleRun
@@ -391,6 +425,14 @@ def run_ours(args):
     del dec, g
     torch.cuda.empty_cache()
 
+    # first step with dynamic contrast strength (log-probs materialised, beta
+    # from their divergences, then the fused path) against the next, regular step
+    dyn = None
+    if not args.no_dynamic_beta:
+        dyn, st = time_dynamic_beta_first_step(w, dev)
+        status |= st
+        torch.cuda.empty_cache()
+
     secondary = None
     if args.secondary != "none":
         w2 = synth.get(args.secondary)
@@ -420,7 +462,7 @@ def run_ours(args):
                                                        "frac_of_measured": step_gbs / hbm_peak if hbm_peak else None,
                                                        "algorithmic_bytes_per_step": tot_bytes / args.steps},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches * args.steps,
-            "clocks": clk, "device_status": status, "secondary": secondary}
+            "clocks": clk, "device_status": status, "secondary": secondary, "dynamic_beta_first_step": dyn}
     if rank == 0:
         print(json.dumps(line), flush=True)
     dist.close()

@@ -159,6 +159,22 @@ pced_status pced_contrastive_select(const float* logprobs, const float* beta, co
                                     void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * pced_adacad_beta -- dynamic contrast strength for the first generated
+ * token (Sec. 3 after Eq. 2: beta_0 is computed as in AdaCAD for the first
+ * generated token and kept fixed thereafter).  Reading: one beta per
+ * contextual expert, the Jensen-Shannon divergence in bits between the
+ * expert's distribution p_k = exp(lp_k) and the amateur's p_0 = exp(lp_0),
+ *   beta[b][k-1] = 1/2 sum_v [p_k log2(p_k/m) + p_0 log2(p_0/m)],  m = (p_k + p_0)/2,
+ * so 0 <= beta <= 1.
+ *   logprobs fp32 [B*(N+1)][V]  query-major, amateur first (device)
+ *   beta     fp32 [B][N]        output (device)
+ * Deterministic (fixed summation order).
+ * ------------------------------------------------------------------------ */
+size_t pced_adacad_beta_workspace_size(int32_t B, int32_t N, int32_t V);
+pced_status pced_adacad_beta(const float* logprobs, int32_t B, int32_t N, int32_t V, float* beta, void* workspace,
+                             size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * pced_step -- one full greedy decode step of all B queries (Sec. 3,
  * Eq. 2, Eq. 3 and the shared-history append) on the weight-free layer
  * chain used for synthetic workloads:
@@ -208,6 +224,15 @@ typedef struct pced_step_args {
    * fewer events) disables recording. */
   void* const* stage_events;
   int32_t n_stage_events;
+  /* Dynamic contrast strength: when beta_from_step is nonzero this call
+   * computes beta from this step's distributions (as pced_adacad_beta), writes
+   * it to beta_out (device fp32 [B][N], may be the array `beta` points to)
+   * and uses it for this step's selection; the caller passes it as `beta` to
+   * the later steps.  Meant for the first step of a decode; such a call runs
+   * the LM head twice (once to materialise the log-probabilities in the
+   * workspace) and records no stage events. */
+  int32_t beta_from_step;
+  float* beta_out;
 } pced_step_args;
 
 size_t pced_step_workspace_size(const pced_dims* dims);

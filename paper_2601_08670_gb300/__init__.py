@@ -44,7 +44,7 @@ class StepArgs(ctypes.Structure):
                 ("attn_scale", ctypes.c_float), ("rms_eps", ctypes.c_float), ("bos_token", ctypes.c_int32),
                 ("hidden_out", ctypes.c_void_p), ("lse_out", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
                 ("workspace_bytes", ctypes.c_size_t), ("stage_events", ctypes.c_void_p),
-                ("n_stage_events", ctypes.c_int32)]
+                ("n_stage_events", ctypes.c_int32), ("beta_from_step", ctypes.c_int32), ("beta_out", ctypes.c_void_p)]
 
 
 _lib = None
@@ -76,6 +76,10 @@ def lib(path: str = LIB_PATH):
         L.pced_contrastive_select_workspace_size.restype = SZ
         L.pced_contrastive_select.argtypes = [P, P, P, F, I32, I32, I32, P, P, P, P, SZ, P]
         L.pced_contrastive_select.restype = I32
+        L.pced_adacad_beta_workspace_size.argtypes = [I32, I32, I32]
+        L.pced_adacad_beta_workspace_size.restype = SZ
+        L.pced_adacad_beta.argtypes = [P, I32, I32, I32, P, P, SZ, P]
+        L.pced_adacad_beta.restype = I32
         L.pced_step_workspace_size.argtypes = [ctypes.POINTER(Dims)]
         L.pced_step_workspace_size.restype = SZ
         L.pced_step.argtypes = [ctypes.POINTER(StepArgs), P]
@@ -197,6 +201,18 @@ def contrastive_select(logprobs, beta, r, gamma: float, ws=None, stream=None):
     return token, expert, score
 
 
+def adacad_beta(logprobs, B: int, N: int, ws=None, stream=None):
+    """pced_adacad_beta: per-expert Jensen-Shannon divergence (bits) between
+    each expert's distribution and its query's amateur, fp32 [B, N]."""
+    V = logprobs.shape[1]
+    beta = torch.empty((B, N), dtype=torch.float32, device=logprobs.device)
+    if ws is None:
+        ws = workspace(int(lib().pced_adacad_beta_workspace_size(B, N, V)), logprobs.device)
+    _check(lib().pced_adacad_beta(_ptr(logprobs), B, N, V, _ptr(beta), _ptr(ws), ws.numel(), _stream(stream)),
+           "pced_adacad_beta")
+    return beta
+
+
 def dims(B, N, L, Hq, Hkv, D, V) -> Dims:
     return Dims(B, N, L, Hq, Hkv, D, V)
 
@@ -222,7 +238,7 @@ class Decoder:
 
     def __init__(self, dm: Dims, *, embed, w_unembed, k_cache, v_cache, layer_elems: int, kv_offset, cap, seq_len,
                  beta, r, gamma: float, max_steps: int, total_cap: int, bos: int = 0, attn_scale=None,
-                 rms_eps: float = 1e-6, keep_hidden: bool = False):
+                 rms_eps: float = 1e-6, keep_hidden: bool = False, dynamic_beta: bool = False):
         dev = k_cache.device
         self.dm = dm
         B, S, d = dm.B, dm.B * (dm.N + 1), dm.Hq * dm.D
@@ -243,9 +259,16 @@ class Decoder:
             float(1.0 / math.sqrt(dm.D) if attn_scale is None else attn_scale), float(rms_eps), int(bos),
             _ptr(self.hidden), _ptr(self.lse), _ptr(self.ws), self.ws.numel())
         self.max_steps = max_steps
+        # dynamic contrast strength: the first step computes beta (into the
+        # `beta` tensor, which the later steps read) from its distributions
+        if dynamic_beta:
+            assert beta.dtype == torch.float32 and beta.is_contiguous()
+            self.args.beta_from_step = 1
+            self.args.beta_out = _ptr(beta)
 
     def step(self, stream=None):
         _check(lib().pced_step(ctypes.byref(self.args), _stream(stream)), "pced_step")
+        self.args.beta_from_step = 0
 
     def set_stage_events(self, events):
         """Record one torch.cuda.Event before and after every launch of each
@@ -272,7 +295,7 @@ class Decoder:
 
 
 def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos: int = 0, keep_hidden=False,
-                        attn_scale=None, rms_eps: float = 1e-6) -> Decoder:
+                        attn_scale=None, rms_eps: float = 1e-6, dynamic_beta: bool = False) -> Decoder:
     """Decoder over a dict of device tensors with the keys k_cache, v_cache,
     kv_offset, cap, seq_len, embed, w_unembed, beta, r, and the host layout
     values layer_elems / total_cap (or a `layout` object carrying them)."""
@@ -282,4 +305,4 @@ def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos:
     return Decoder(dm, embed=t["embed"], w_unembed=t["w_unembed"], k_cache=t["k_cache"], v_cache=t["v_cache"],
                    layer_elems=layer_elems, kv_offset=t["kv_offset"], cap=t["cap"], seq_len=t["seq_len"],
                    beta=t["beta"], r=t["r"], gamma=gamma, max_steps=max_steps, total_cap=total_cap, bos=bos,
-                   attn_scale=attn_scale, rms_eps=rms_eps, keep_hidden=keep_hidden)
+                   attn_scale=attn_scale, rms_eps=rms_eps, keep_hidden=keep_hidden, dynamic_beta=dynamic_beta)

@@ -465,9 +465,14 @@ cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, con
 }
 
 // ------------------------------------------------------------ mode-0 finish
+// grid (chunks, S): every CTA of row s forms lse[s] from the row's tile
+// records (the same fixed order in each) and turns its chunk of logits into
+// log-probabilities in place; chunk 0 stores lse.
+constexpr int LSE_CHUNK = 16384;
+
 __global__ void __launch_bounds__(256) lm_lse_finalize_kernel(float* logits, const float2* rec_stats, float* lse,
                                                               int32_t V, int32_t nrec) {
-  const int s = blockIdx.x, tid = threadIdx.x;
+  const int c = blockIdx.x, s = blockIdx.y, tid = threadIdx.x;
   __shared__ float2 red[8];
   __shared__ float Ls;
   float M = -INFINITY, sum = 0.f;
@@ -486,17 +491,19 @@ __global__ void __launch_bounds__(256) lm_lse_finalize_kernel(float* logits, con
     float m = -INFINITY, su = 0.f;
     for (int w = 0; w < 8; ++w) lse_merge(m, su, red[w].x, red[w].y);
     Ls = m + logf(su);
-    lse[s] = Ls;
+    if (c == 0) lse[s] = Ls;
   }
   __syncthreads();
   const float L = Ls;
   float* row = logits + (int64_t)s * V;
-  for (int v = tid; v < V; v += 256) row[v] -= L;
+  const int v1 = min(V, (c + 1) * LSE_CHUNK);
+  for (int v = c * LSE_CHUNK + tid; v < v1; v += 256) row[v] -= L;
 }
 
 cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float* lse, int32_t S, int32_t V,
                                    int32_t nrec, cudaStream_t stream) {
-  lm_lse_finalize_kernel<<<S, 256, 0, stream>>>(logits, rec_stats, lse, V, nrec);
+  lm_lse_finalize_kernel<<<dim3((V + LSE_CHUNK - 1) / LSE_CHUNK, S), 256, 0, stream>>>(logits, rec_stats, lse, V,
+                                                                                      nrec);
   return cudaGetLastError();
 }
 

@@ -11,6 +11,7 @@
 #include <math.h>
 #include <stdlib.h>
 
+#include "adacad.cuh"
 #include "attention.cuh"
 #include "lm_head.cuh"
 
@@ -26,6 +27,8 @@ struct StepLayout {
   float* sel_L;
   float* sel_u;
   int32_t* sel_tok;
+  float* lp;              // [S][V] log-probabilities of a dynamic-beta first step
+  void* ada;              // scratch of the beta kernel (counters zero between uses)
   uint64_t* part_ss;
   uint64_t* resid;
   uint64_t* rec_o;
@@ -60,6 +63,8 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   L.sel_L = c.take<float>((size_t)S);
   L.sel_u = c.take<float>((size_t)S);
   L.sel_tok = c.take<int32_t>((size_t)S);
+  L.lp = c.take<float>((size_t)S * dm->V);
+  L.ada = c.take<char>(adacad_scratch_bytes(dm->B, dm->N, dm->V));
   L.bytes = c.used() + 4 * (4096 - 256);  // room for the 4 KB alignment of four arrays
   return L;
 }
@@ -87,7 +92,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (!p) return fail(PCED_ERR_INVALID_ARG, "pced_step: null args");
   const pced_dims dm = p->dims;
   if (!p->embed || !p->w_unembed || !p->k_cache || !p->v_cache || !p->kv_offset || !p->cap || !p->seq_len ||
-      !p->step || !p->history || !p->beta || !p->r || !p->workspace)
+      !p->step || !p->history || !p->beta || !p->r || !p->workspace || (p->beta_from_step && !p->beta_out))
     return fail(PCED_ERR_INVALID_ARG, "pced_step: null pointer");
   if (dm.B < 1 || dm.N < 1 || dm.L < 1 || dm.Hq < 1 || dm.Hkv < 1 || dm.D < 1 || dm.V < 1 || dm.Hq % dm.Hkv != 0 ||
       2 * dm.Hkv > dm.Hq || dm.L > ATT_MAX_LAYERS || p->max_steps < 1 || p->layer_elems < dm.D || p->total_cap < 1)
@@ -120,7 +125,8 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (st == PCED_OK) st = make_tmap_2d(&hmap, W.h, (uint64_t)S, (uint64_t)d, (uint32_t)g.chunk_n, LM_TILE_K, false);
   if (st != PCED_OK) return st;
   cudaStream_t s = (cudaStream_t)stream;
-  const bool timed = p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
+  const bool dyn = p->beta_from_step != 0;
+  const bool timed = !dyn && p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
   cudaStreamCaptureStatus cap_status = cudaStreamCaptureStatusNone;
   if (timed && cudaStreamIsCapturing(s, &cap_status) != cudaSuccess) return cuda_status(cudaGetLastError(), "capture query");
   int mark_i = 0;
@@ -174,6 +180,39 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "attention launch");
 
+  // dynamic contrast strength: materialise this step's log-probabilities,
+  // beta from their divergences, then the usual fused LM head with that beta
+  const float* beta = p->beta;
+  if (dyn) {
+    LmArgs lz = {};
+    lz.mode = 0;
+    lz.S = S;
+    lz.N = 0;
+    lz.V = dm.V;
+    lz.ntiles = g.ntiles;
+    lz.nks = g.nks;
+    lz.slabs = g.slabs;
+    lz.nst = g.nst;
+    lz.nbeta = 0;
+    lz.stages = g.stages;
+    lz.acc_bufs = g.acc_bufs;
+    lz.S_pad = g.S_pad;
+    lz.nchunk = g.nchunk;
+    lz.chunk_n = g.chunk_n;
+    lz.tmem_cols = g.tmem_cols;
+    lz.logits = W.lp;
+    lz.rec_stats = W.lm_stats;
+    lz.tile_ctr = W.lm_tile_ctr;
+    lz.status = W.status;
+    lz.pdl = 0;
+    e = lm_head_launch(wmap, hmap, g, lz, s);
+    if (e == cudaSuccess) e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
+    // the JSD kernel also re-arms the LM head's tile counter for the fused pass
+    if (e == cudaSuccess) e = adacad_beta_launch(W.lp, dm.B, dm.N, dm.V, p->beta_out, W.ada, W.lm_tile_ctr, s);
+    if (e != cudaSuccess) return cuda_status(e, "dynamic beta launches");
+    beta = p->beta_out;
+  }
+
   LmArgs la = {};
   la.mode = 1;
   la.S = S;
@@ -193,9 +232,9 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.rec_stats = W.lm_stats;
   la.rec_arg = W.lm_arg;
   la.tile_ctr = W.lm_tile_ctr;
-  la.beta = p->beta;
+  la.beta = beta;
   la.status = W.status;
-  la.pdl = timed ? 0 : 1;  // stage events between the launches would break the overlap
+  la.pdl = (timed || dyn) ? 0 : 1;  // stage events between the launches would break the overlap
   e = lm_head_launch(wmap, hmap, g, la, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "lm head launch");
@@ -211,7 +250,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.sel_u = W.sel_u;
   sa.sel_tok = W.sel_tok;
   sa.qdone = W.sel_qdone;
-  sa.beta = p->beta;
+  sa.beta = beta;
   sa.r = p->r;
   sa.gamma = p->gamma;
   sa.lse_out = p->lse_out;
@@ -222,7 +261,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.max_steps = p->max_steps;
   sa.done_counter = W.done_counter;
   sa.status = W.status;
-  sa.pdl = timed ? 0 : 1;
+  sa.pdl = (timed || dyn) ? 0 : 1;
   e = select_from_records_launch(sa, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "select launch");

@@ -70,6 +70,25 @@ def test_select_rejects_bad_arguments(L):
     assert f(FAKE, FAKE, FAKE, 2.5, 1, 4, 100, FAKE, FAKE, FAKE, FAKE, 8, None) == 2
 
 
+def test_adacad_beta_rejects_bad_arguments(L):
+    f = L.pced_adacad_beta
+    big = 1 << 30
+    assert f(None, 1, 2, 100, FAKE, FAKE, big, None) == 1
+    assert f(FAKE, 1, 2, 100, None, FAKE, big, None) == 1
+    assert f(FAKE, 0, 2, 100, FAKE, FAKE, big, None) == 1
+    assert f(FAKE, 1, 0, 100, FAKE, FAKE, big, None) == 1
+    assert f(FAKE, 1, 2, 0, FAKE, FAKE, big, None) == 1
+    assert f(FAKE + 2, 1, 2, 100, FAKE, FAKE, big, None) == 1  # misaligned
+    assert f(FAKE, 1, 2, 100, FAKE, FAKE, 8, None) == 2        # workspace too small
+    assert L.pced_adacad_beta_workspace_size(1, 2, 100) > 0
+
+
+def test_step_dynamic_beta_needs_its_output(L):
+    import paper_2601_08670_gb300 as pced
+    a = step_args(pced, beta_from_step=1)
+    assert L.pced_step(ctypes.byref(a), None) == 1
+
+
 def step_args(pced, **kw):
     dm = pced.dims(1, 8, 32, 32, 8, 128, 128256)
     a = pced.StepArgs()
