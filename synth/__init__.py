@@ -101,6 +101,14 @@ WORKLOADS = {
         doc_len=("clipnormal", 1024.0, 256.0, 256, 2048),
         description="16 queries x (16 doc experts + amateur) = 272 sequences, doc KV N(1024,256) clipped "
                     "[256,2048]+32, Llama-3-8B shapes, 32 steps"),
+    "llama8_k64": Workload(
+        "llama8_k64", B=1, N=64, L=32, Hq=32, Hkv=8, D=128, V=128256, steps=16,
+        doc_len=("fixed", 2048),
+        description="Llama-3-8B shapes, top-k = 64 doc experts of KV 2048+32 + amateur, vocab 128256, 16 steps"),
+    "llama8_k128": Workload(
+        "llama8_k128", B=1, N=128, L=32, Hq=32, Hkv=8, D=128, V=128256, steps=16,
+        doc_len=("fixed", 2048),
+        description="Llama-3-8B shapes, top-k = 128 doc experts of KV 2048+32 + amateur, vocab 128256, 16 steps"),
     "qwen_flat": Workload(
         "qwen_flat", B=1, N=16, L=28, Hq=28, Hkv=4, D=128, V=151936, steps=128,
         doc_len=("fixed", 4096), r_recipe=("flat", 0.5),

@@ -132,6 +132,15 @@ def test_llama32_ragged_full_size(cuda_ok):
     run_parity("llama32", 2, min_ram_gb=40)
 
 
+def test_llama8_top64_experts(cuda_ok):
+    # the paper scales the retrieved experts from k = 8 to k = 128 (App., top-k ablation)
+    run_parity("llama8_k64", 2, min_ram_gb=24)
+
+
+def test_llama8_top128_experts(cuda_ok):
+    run_parity("llama8_k128", 1, min_ram_gb=44)
+
+
 def test_cache_full_is_flagged_not_faulted(cuda_ok):
     import paper_2601_08670_gb300 as pced
     dev = torch.device("cuda")
