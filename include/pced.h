@@ -56,6 +56,7 @@ typedef enum pced_status {
 #define PCED_DEV_TIMEOUT 0x4u     /* a bounded in-kernel wait expired */
 #define PCED_DEV_BAD_TOKEN 0x8u   /* history token outside [0, V) */
 #define PCED_DEV_STEP_LIMIT 0x10u /* step counter reached max_steps */
+#define PCED_DEV_BAD_BLOCK 0x20u  /* paged caches: a needed block-table entry is missing or outside the pool */
 
 /* Static description of a status code (host). */
 const char* pced_status_string(int32_t status);
@@ -233,6 +234,20 @@ typedef struct pced_step_args {
    * workspace) and records no stage events. */
   int32_t beta_from_step;
   float* beta_out;
+  /* Paged caches (PagedAttention-style, as the paper serves): when
+   * block_table is not NULL, k_cache / v_cache hold per layer a pool of
+   * layer_elems / (Hkv*block_rows*D) blocks of [Hkv][block_rows][D]; row pos
+   * of (sequence s, kv-head h) is row pos % block_rows of block
+   * block_table[s*max_blocks + pos / block_rows].  kv_offset is then unused
+   * (may be NULL); cap[s] still bounds the length and must not exceed
+   * max_blocks*block_rows.  block_rows: a multiple of 64 (else
+   * PCED_ERR_INVALID_ARG); S*max_blocks must stay below 2^31 (else
+   * PCED_ERR_UNSUPPORTED).  A table entry outside [0, number of blocks) sets
+   * PCED_DEV_BAD_BLOCK: its keys read as zeros and the appended row is not
+   * stored.  The table is read, never written. */
+  const int32_t* block_table;
+  int32_t block_rows;
+  int32_t max_blocks;
 } pced_step_args;
 
 size_t pced_step_workspace_size(const pced_dims* dims);

@@ -21,6 +21,7 @@ PCED_DEV_CACHE_FULL = 0x2
 PCED_DEV_TIMEOUT = 0x4
 PCED_DEV_BAD_TOKEN = 0x8
 PCED_DEV_STEP_LIMIT = 0x10
+PCED_DEV_BAD_BLOCK = 0x20
 
 
 class PcedError(RuntimeError):
@@ -44,7 +45,8 @@ class StepArgs(ctypes.Structure):
                 ("attn_scale", ctypes.c_float), ("rms_eps", ctypes.c_float), ("bos_token", ctypes.c_int32),
                 ("hidden_out", ctypes.c_void_p), ("lse_out", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
                 ("workspace_bytes", ctypes.c_size_t), ("stage_events", ctypes.c_void_p),
-                ("n_stage_events", ctypes.c_int32), ("beta_from_step", ctypes.c_int32), ("beta_out", ctypes.c_void_p)]
+                ("n_stage_events", ctypes.c_int32), ("beta_from_step", ctypes.c_int32), ("beta_out", ctypes.c_void_p),
+                ("block_table", ctypes.c_void_p), ("block_rows", ctypes.c_int32), ("max_blocks", ctypes.c_int32)]
 
 
 _lib = None
@@ -238,7 +240,8 @@ class Decoder:
 
     def __init__(self, dm: Dims, *, embed, w_unembed, k_cache, v_cache, layer_elems: int, kv_offset, cap, seq_len,
                  beta, r, gamma: float, max_steps: int, total_cap: int, bos: int = 0, attn_scale=None,
-                 rms_eps: float = 1e-6, keep_hidden: bool = False, dynamic_beta: bool = False):
+                 rms_eps: float = 1e-6, keep_hidden: bool = False, dynamic_beta: bool = False, block_table=None,
+                 block_rows: int = 0):
         dev = k_cache.device
         self.dm = dm
         B, S, d = dm.B, dm.B * (dm.N + 1), dm.Hq * dm.D
@@ -249,7 +252,7 @@ class Decoder:
         self.hidden = torch.zeros((S, d), dtype=torch.bfloat16, device=dev) if keep_hidden else None
         self.lse = torch.zeros(S, dtype=torch.float32, device=dev)
         self.ws = workspace(step_workspace_size(dm), dev)
-        self._keep = (embed, w_unembed, k_cache, v_cache, kv_offset, cap, seq_len, beta, r)
+        self._keep = (embed, w_unembed, k_cache, v_cache, kv_offset, cap, seq_len, beta, r, block_table)
         self.seq_len = seq_len
         self.beta, self.r = beta, r
         self.args = StepArgs(
@@ -259,6 +262,11 @@ class Decoder:
             float(1.0 / math.sqrt(dm.D) if attn_scale is None else attn_scale), float(rms_eps), int(bos),
             _ptr(self.hidden), _ptr(self.lse), _ptr(self.ws), self.ws.numel())
         self.max_steps = max_steps
+        if block_table is not None:  # paged caches
+            assert block_table.dtype == torch.int32 and block_table.is_contiguous() and block_table.dim() == 2
+            self.args.block_table = _ptr(block_table)
+            self.args.block_rows = int(block_rows)
+            self.args.max_blocks = int(block_table.shape[1])
         # dynamic contrast strength: the first step computes beta (into the
         # `beta` tensor, which the later steps read) from its distributions
         if dynamic_beta:
@@ -305,4 +313,5 @@ def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos:
     return Decoder(dm, embed=t["embed"], w_unembed=t["w_unembed"], k_cache=t["k_cache"], v_cache=t["v_cache"],
                    layer_elems=layer_elems, kv_offset=t["kv_offset"], cap=t["cap"], seq_len=t["seq_len"],
                    beta=t["beta"], r=t["r"], gamma=gamma, max_steps=max_steps, total_cap=total_cap, bos=bos,
-                   attn_scale=attn_scale, rms_eps=rms_eps, keep_hidden=keep_hidden, dynamic_beta=dynamic_beta)
+                   attn_scale=attn_scale, rms_eps=rms_eps, keep_hidden=keep_hidden, dynamic_beta=dynamic_beta,
+                   block_table=t.get("block_table"), block_rows=int(t.get("block_rows", 0)))

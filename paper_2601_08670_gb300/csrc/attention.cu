@@ -115,12 +115,42 @@ __device__ __forceinline__ Piece find_piece(const int64_t* pre, const int32_t* l
   return pc;
 }
 
-// exclusive prefix of ext[i] = lens[i] + extra into pre[0..S] (one warp)
-__device__ __forceinline__ void prefix_extents(const int32_t* lens, int32_t S, int32_t extra, int64_t* pre, int lane) {
+// The piece after prev when prev ended at its segment's end p (< end): the
+// next segment of the same position space, so no search is needed (find_piece
+// at p gives the same piece, as every segment spans at least one position).
+__device__ __forceinline__ Piece next_piece(const Piece& prev, const int64_t* pre, const int32_t* lens,
+                                            int32_t s_lo, int32_t s_hi, int64_t T, int64_t p, int64_t end,
+                                            int32_t lead = 0) {
+  Piece pc;
+  pc.s = prev.s + 1;
+  pc.h = prev.h;
+  if (pc.s >= s_hi) {
+    pc.s = s_lo;
+    ++pc.h;
+  }
+  const int64_t seg_end = (int64_t)pc.h * T + pre[pc.s + 1] - pre[s_lo];
+  const int64_t e = seg_end < end ? seg_end : end;
+  pc.adv = e - p;
+  const int64_t len = lens[pc.s];
+  const int64_t k1 = pc.adv - lead < len ? pc.adv - lead : len;  // keys start at offset lead
+  if (k1 > 0) {
+    pc.k0 = 0;
+    pc.k1 = (int32_t)k1;
+  } else {
+    pc.k0 = pc.k1 = 0;
+  }
+  return pc;
+}
+
+// exclusive prefix of ext[i] = roundup(lens[i], align) + extra into pre[0..S]
+// (one warp; align a power of two)
+__device__ __forceinline__ void prefix_extents(const int32_t* lens, int32_t S, int32_t extra, int64_t* pre, int lane,
+                                               int32_t align = 1) {
   const int chunk = (S + 31) / 32;
   const int b0 = lane * chunk, b1 = min(S, b0 + chunk);
+  const int64_t am = align - 1;
   int64_t sum = 0;
-  for (int i = b0; i < b1; ++i) sum += (int64_t)lens[i] + extra;
+  for (int i = b0; i < b1; ++i) sum += (((int64_t)lens[i] + am) & ~am) + extra;
   int64_t incl = sum;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -130,7 +160,7 @@ __device__ __forceinline__ void prefix_extents(const int32_t* lens, int32_t S, i
   int64_t run = incl - sum;
   for (int i = b0; i < b1; ++i) {
     pre[i] = run;
-    run += (int64_t)lens[i] + extra;
+    run += (((int64_t)lens[i] + am) & ~am) + extra;
   }
   if (lane == 31) pre[S] = incl;
 }
@@ -574,9 +604,13 @@ struct GroupPlan {
 };
 
 // Cut the sequences into min(want, S) contiguous groups of about equal weight
-// (pre: prefix of the extents) and partition each over the grid.
+// (pre: prefix of the extents) and partition each over the grid.  align (a
+// power of two dividing every extent): CTA c of a group takes positions
+// [c*P, (c+1)*P) rounded down to multiples of align, with P at least align,
+// so every CTA range is a whole number of tiles and none inside a segment is
+// empty (the CTAs holding a segment's keys stay consecutive).
 __device__ __forceinline__ void plan_groups(GroupPlan& gp, const int64_t* pre, int32_t S, int32_t Hkv, int want,
-                                            int64_t grid, int64_t cta) {
+                                            int64_t grid, int64_t cta, int32_t align = 1) {
   int ng = want < 1 ? 1 : (want > ATT_MAX_GROUPS ? ATT_MAX_GROUPS : want);
   if (ng > S) ng = S;
   const int64_t T = pre[S];
@@ -591,26 +625,68 @@ __device__ __forceinline__ void plan_groups(GroupPlan& gp, const int64_t* pre, i
   for (int g = 0; g < ng; ++g) {
     const int64_t Tg = pre[gp.s_lo[g + 1]] - pre[gp.s_lo[g]];
     const int64_t tot = (int64_t)Hkv * Tg;
-    const int64_t Pg = (tot + grid - 1) / grid;
+    int64_t Pg = (tot + grid - 1) / grid;
+    if (Pg < align) Pg = align;
+    const int64_t am = ~(int64_t)(align - 1);
     gp.T[g] = Tg;
     gp.P[g] = Pg;
-    gp.cb[g] = min(tot, cta * Pg);
-    gp.ce[g] = min(tot, gp.cb[g] + Pg);
+    gp.cb[g] = min(tot, cta * Pg) & am;
+    gp.ce[g] = min(tot, (cta + 1) * Pg) & am;
   }
   gp.n = ng;
 }
 
+// Block index of key x (paged caches).
+__device__ __forceinline__ int32_t block_of(const StepAttArgs& a, int32_t x) {
+  return a.block_shift >= 0 ? x >> a.block_shift : (int32_t)((uint32_t)x / (uint32_t)a.block_rows);
+}
+
+// Row, within a layer's region of the tensor maps, of key 0 of kv-head h in
+// block blk (of [Hkv][P][D]); -1 for a block id outside the pool (flagged).
+__device__ __forceinline__ int32_t block_base_of(const StepAttArgs& a, int32_t blk, int32_t h) {
+  if (blk < 0 || blk >= a.num_blocks) {
+    dev_flag(a.status, PCED_DEV_BAD_BLOCK);
+    return -1;
+  }
+  return (blk * a.Hkv + h) * a.block_rows;  // below rows_per_layer < 2^31
+}
+
+// block_base_of for block j of (sequence s, kv-head h): entry i of the CTA's
+// shared copy (built once per launch for the pieces of one layer, ptab_n
+// entries) or, past the copy, from the table in global memory.
+__device__ __forceinline__ int32_t block_base(const StepAttArgs& a, int32_t s, int32_t h, int32_t j, int32_t i,
+                                              const int32_t* ptab, int32_t ptab_n) {
+  if (i < ptab_n) return ptab[i];
+  return block_base_of(a, j < a.max_blocks ? __ldg(a.block_table + (int64_t)s * a.max_blocks + j) : -1, h);
+}
+
+// The CTA whose range (as plan_groups cuts it) holds position x.
+__device__ __forceinline__ int64_t part_cta(int64_t x, int64_t Pg, int32_t align) {
+  return udiv_pos((x & ~(int64_t)(align - 1)) + align - 1, Pg);
+}
+
 // Tile cursor over a CTA's ranges through all layers and groups (the
-// producer's order: layer by layer, group by group).
+// producer's order: layer by layer, group by group), carrying the
+// tensor-map row of its tile.  Slab caches: the slab's row + kt.  Paged
+// caches: pieces start on 64-key boundaries (tile-aligned partition), so a
+// tile never straddles two blocks, and the row is row kt % P of block
+// table[s][kt / P], advanced without a division and looked up once per block.  A bad block id (flagged) points the tile past
+// the last row of the tensor map, where the loads read zeros.
 struct TileCursor {
   int32_t l, g, kt;
-  int64_t p, row0;  // row0: tensor-map row of key 0 of the current piece
+  int32_t row;      // tensor-map row of the tile
+  bool bad;         // paged caches: the tile's block id is outside the pool
+  int64_t p;
+  int32_t kin, bj;  // paged caches: key offset of the tile in its block, the block's index
+  int32_t bi, ptn;  // paged caches: block-table copy entry of block bj; of the next piece's first block
   Piece pc;
   bool ok;
 };
 
+// cont: c.pc is the piece before position c.p in the same group
 __device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
-                                            const int32_t* lens, const GroupPlan& gp, int D) {
+                                            const int32_t* lens, const GroupPlan& gp, int D, const int32_t* ptab,
+                                            int32_t ptab_n, bool cont) {
   while (true) {
     if (c.p >= gp.ce[c.g]) {
       if (++c.g >= gp.n) {
@@ -619,33 +695,68 @@ __device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a,
           c.ok = false;
           return;
         }
+        c.ptn = 0;  // every layer visits the same pieces
       }
       c.p = gp.cb[c.g];
+      cont = false;
       continue;
     }
-    c.pc = find_piece(pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead);
+    c.pc = cont ? next_piece(c.pc, pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead)
+                : find_piece(pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead);
+    cont = true;
     if (c.pc.k0 < c.pc.k1) {
-      c.kt = c.pc.k0;
-      c.row0 = (int64_t)c.l * a.rows_per_layer + (a.kv_offset[c.pc.s] + (int64_t)c.pc.h * a.cap[c.pc.s] * D) / D;
+      if (!a.block_table) {
+        c.kt = c.pc.k0;
+        c.row = (int32_t)((int64_t)c.l * a.rows_per_layer +
+                          (__ldg(a.kv_offset + c.pc.s) + (int64_t)c.pc.h * __ldg(a.cap + c.pc.s) * D) / D + c.kt);
+        c.bad = false;
+        return;
+      }
+      c.kt = c.pc.k0;  // a multiple of 64 (tile-aligned partition)
+      c.bj = block_of(a, c.kt);
+      c.kin = c.kt - c.bj * a.block_rows;
+      c.bi = c.ptn;
+      c.ptn += block_of(a, c.pc.k1 - 1) - c.bj + 1;
+      const int32_t b0 = block_base(a, c.pc.s, c.pc.h, c.bj, c.bi, ptab, ptab_n);
+      c.bad = b0 < 0;
+      c.row = (int32_t)(c.bad ? (int64_t)a.L * a.rows_per_layer : (int64_t)c.l * a.rows_per_layer + b0 + c.kin);
       return;
     }
     c.p += c.pc.adv;
   }
 }
 __device__ __forceinline__ void cursor_begin(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
-                                             const int32_t* lens, const GroupPlan& gp, int D) {
+                                             const int32_t* lens, const GroupPlan& gp, int D, const int32_t* ptab,
+                                             int32_t ptab_n) {
   c.l = 0;
   c.g = 0;
   c.p = gp.cb[0];
+  c.ptn = 0;
   c.ok = a.L > 0;
-  if (c.ok) cursor_seek(c, a, pre, lens, gp, D);
+  if (c.ok) cursor_seek(c, a, pre, lens, gp, D, ptab, ptab_n, false);
 }
 __device__ __forceinline__ void cursor_next(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
-                                            const int32_t* lens, const GroupPlan& gp, int D) {
+                                            const int32_t* lens, const GroupPlan& gp, int D, const int32_t* ptab,
+                                            int32_t ptab_n) {
   c.kt += ATT_BLOCK_N;
-  if (c.kt < c.pc.k1) return;
+  if (c.kt < c.pc.k1) {
+    if (a.block_table) {
+      c.kin += ATT_BLOCK_N;
+      if (c.kin == a.block_rows) {
+        c.kin = 0;
+        ++c.bj;
+        ++c.bi;
+        const int32_t b0 = block_base(a, c.pc.s, c.pc.h, c.bj, c.bi, ptab, ptab_n);
+        c.bad = b0 < 0;
+        c.row = (int32_t)(c.bad ? (int64_t)a.L * a.rows_per_layer : (int64_t)c.l * a.rows_per_layer + b0);
+        return;
+      }
+    }
+    if (!c.bad) c.row += ATT_BLOCK_N;
+    return;
+  }
   c.p += c.pc.adv;
-  cursor_seek(c, a, pre, lens, gp, D);
+  cursor_seek(c, a, pre, lens, gp, D, ptab, ptab_n, true);
 }
 
 // 1/rms of x_l[s] from its Hkv per-group sums of squares (waits for all of
@@ -694,6 +805,7 @@ struct StepSmem {
   uint32_t pbuf, pslot; // [2] partial hand-off slots: ms[8][8], ls[8][8], os[8][G][D + 4]
   uint32_t misc;        // flags
   uint32_t tables;      // pre[ATT_MAX_S+1] int64, GroupPlan, lens[ATT_MAX_S] int32, apnd[ATT_MAX_S] u8
+  uint32_t ptab;        // block-table copy: ptab[ATT_PTAB] int32, its entry count, ptab_h[ATT_PTAB] u8
   uint32_t total;       // bytes to request, alignment slack included
 };
 __host__ __device__ inline StepSmem step_smem(int D, int G) {
@@ -711,7 +823,8 @@ __host__ __device__ inline StepSmem step_smem(int D, int G) {
     L.pbuf = L.qbuf + 2u * L.qslot;
     L.misc = L.pbuf + 2u * L.pslot;
     L.tables = L.misc + 64u;
-    L.total = 1024u + L.tables + tables;
+    L.ptab = L.tables + ((tables + 15u) & ~15u);
+    L.total = 1024u + L.ptab + ATT_PTAB * 5u + 16u;
     if (L.total <= 227u * 1024u) break;
   }
   return L;
@@ -770,6 +883,9 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   GroupPlan& gp = *reinterpret_cast<GroupPlan*>(pre + ATT_MAX_S + 1);
   int32_t* lens = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(&gp) + ((sizeof(GroupPlan) + 7) & ~(size_t)7));
   uint8_t* apnd = reinterpret_cast<uint8_t*>(lens + ATT_MAX_S);
+  int32_t* ptab = reinterpret_cast<int32_t*>(gbase + SL.ptab);
+  int32_t* ptab_cnt = ptab + ATT_PTAB;
+  uint8_t* ptab_h = reinterpret_cast<uint8_t*>(ptab_cnt + 4);  // kv-head of each entry (while building)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int32_t epoch = *a.epoch;
@@ -814,10 +930,45 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     apnd[i] = ap ? 1 : 0;
   }
   __syncthreads();
-  if (warp == 0) prefix_extents(lens, S, a.seg_cost, pre, lane);
+  const int32_t align = a.block_table ? ATT_BLOCK_N : 1;
+  if (warp == 0) prefix_extents(lens, S, a.seg_cost, pre, lane, align);
   __syncthreads();
-  if (tid == 0) plan_groups(gp, pre, S, Hkv, a.groups, gridDim.x, blockIdx.x);
+  if (tid == 0) plan_groups(gp, pre, S, Hkv, a.groups, gridDim.x, blockIdx.x, align);
   __syncthreads();
+  if (a.block_table) {
+    // paged caches: for the blocks of this CTA's pieces (the same in every
+    // layer), in the cursor's order, keep the block's row base for the
+    // piece's kv-head (block_base_of) in shared memory, so the producer and
+    // the input warp never wait on a table read in the loop
+    if (warp == 0) {
+      if (lane == 0) {
+        int32_t n = 0;
+        for (int gi = 0; gi < gp.n && n < ATT_PTAB; ++gi) {
+          Piece pc;
+          pc.adv = -1;  // none yet
+          for (int64_t pp = gp.cb[gi]; pp < gp.ce[gi] && n < ATT_PTAB;) {
+            pc = pc.adv < 0
+                     ? find_piece(pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead)
+                     : next_piece(pc, pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead);
+            pp += pc.adv;
+            if (pc.k0 == pc.k1) continue;
+            const int32_t j0 = block_of(a, pc.k0), j1 = block_of(a, pc.k1 - 1);
+            for (int32_t j = j0; j <= j1 && n < ATT_PTAB; ++j) {
+              ptab_h[n] = (uint8_t)pc.h;
+              ptab[n++] = j < a.max_blocks ? pc.s * a.max_blocks + j : -1;
+            }
+          }
+        }
+        *ptab_cnt = n;
+      }
+      __syncwarp();
+      const int32_t n = *ptab_cnt;
+      for (int32_t i = lane; i < n; i += 32)
+        ptab[i] = block_base_of(a, ptab[i] < 0 ? -1 : __ldg(a.block_table + ptab[i]), ptab_h[i]);
+    }
+    __syncthreads();
+  }
+  const int32_t ptab_n = a.block_table ? *ptab_cnt : 0;
 
   if (warp == STEP_PRODUCER) {
     // ------------------------------------------------------------ producer
@@ -826,12 +977,14 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     if (lane == 0) {
       const uint64_t pol = policy_evict_first();
       TileCursor ld, pf;
-      cursor_begin(ld, a, pre, lens, gp, D);
-      cursor_begin(pf, a, pre, lens, gp, D);
+      cursor_begin(ld, a, pre, lens, gp, D, ptab, ptab_n);
+      cursor_begin(pf, a, pre, lens, gp, D, ptab, ptab_n);
       for (int i = 0; i < a.pf_tiles && pf.ok; ++i) {
-        tma_prefetch_l2_3d(&kmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
-        tma_prefetch_l2_3d(&vmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
-        cursor_next(pf, a, pre, lens, gp, D);
+        if (!pf.bad) {
+          tma_prefetch_l2_3d(&kmap, 0, pf.row, 0);
+          tma_prefetch_l2_3d(&vmap, 0, pf.row, 0);
+        }
+        cursor_next(pf, a, pre, lens, gp, D, ptab, ptab_n);
       }
       uint32_t it = 0, st = 0, ph = 0;
       bool ok = true;
@@ -843,19 +996,20 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         const uint32_t fb = bar_full + 8 * st;
         const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
         mbar_arrive_expect_tx(fb, C::STAGE_BYTES);
-        const int32_t row = (int32_t)(ld.row0 + ld.kt);
-        tma_load_3d(sk, &kmap, fb, 0, row, 0, pol);
-        tma_load_3d(sv, &vmap, fb, 0, row, 0, pol);
+        tma_load_3d(sk, &kmap, fb, 0, ld.row, 0, pol);
+        tma_load_3d(sv, &vmap, fb, 0, ld.row, 0, pol);
         ++it;
         if (++st == NST) {
           st = 0;
           ph ^= 1u;
         }
-        cursor_next(ld, a, pre, lens, gp, D);
+        cursor_next(ld, a, pre, lens, gp, D, ptab, ptab_n);
         if (pf.ok) {
-          tma_prefetch_l2_3d(&kmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
-          tma_prefetch_l2_3d(&vmap, 0, (int32_t)(pf.row0 + pf.kt), 0);
-          cursor_next(pf, a, pre, lens, gp, D);
+          if (!pf.bad) {
+            tma_prefetch_l2_3d(&kmap, 0, pf.row, 0);
+            tma_prefetch_l2_3d(&vmap, 0, pf.row, 0);
+          }
+          cursor_next(pf, a, pre, lens, gp, D, ptab, ptab_n);
         }
       }
       if (!ok) {
@@ -878,11 +1032,22 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     for (int l = 0; l < a.L && ok; ++l) {
       const int par = l & 1;
       const uint32_t tag = step_tag(epoch, l);
-      for (int gi = 0; gi < gp.n && ok; ++gi)
+      int32_t ptn = 0;  // block-table copy: entry of the next piece's first block (as the producer's cursor)
+      for (int gi = 0; gi < gp.n && ok; ++gi) {
+      Piece pc;
+      pc.adv = -1;  // none yet
       for (int64_t pp = gp.cb[gi]; pp < gp.ce[gi] && ok;) {
-        const Piece pc = find_piece(pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead);
+        pc = pc.adv < 0 ? find_piece(pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead)
+                        : next_piece(pc, pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead);
         pp += pc.adv;
         if (pc.k0 == pc.k1) continue;
+        int32_t pt = 0, j0 = 0;
+        if (a.block_table) {
+          if (pc.k0 & (ATT_BLOCK_N - 1)) dev_flag(a.status, PCED_DEV_BAD_BLOCK);  // the partition guarantees it
+          j0 = block_of(a, pc.k0);
+          pt = ptn;
+          ptn += block_of(a, pc.k1 - 1) - j0 + 1;
+        }
         const uint32_t slot = p & 1u, u = p >> 1;
         ++p;
         if (u > 0 && !mbar_wait(bar_qempty + 8 * slot, (u - 1u) & 1u, a.status)) {
@@ -949,8 +1114,17 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           const uint64_t* xv = xs + ((int64_t)Hkv + pc.h) * D;
           uint32_t* kr = qw + 8 * QW;
           uint32_t* vr = kr + D / 2;
-          const int64_t grow = (int64_t)l * a.layer_elems + a.kv_offset[pc.s] +
-                               ((int64_t)pc.h * a.cap[pc.s] + lens[pc.s] - 1) * D;
+          int64_t arow;
+          if (a.block_table) {
+            const int32_t key = lens[pc.s] - 1, j = block_of(a, key);
+            const int32_t b0 = block_base(a, pc.s, pc.h, j, pt + (j - j0), ptab, ptab_n);
+            arow = b0 < 0 ? -1 : (int64_t)l * a.rows_per_layer + b0 + (key - j * a.block_rows);
+          } else {
+            arow = (int64_t)l * a.rows_per_layer + (a.kv_offset[pc.s] + (int64_t)pc.h * a.cap[pc.s] * D) / D +
+                   lens[pc.s] - 1;
+          }
+          const bool wrow = arow >= 0;  // a bad block id was flagged: keep the cache untouched
+          const int64_t grow = (wrow ? arow : 0) * D;
           constexpr int RW = (D / 2 + 31) / 32;  // word pairs per lane
           float k0[RW], k1[RW], w0[RW], w1[RW];
           uint64_t t0 = 0;
@@ -983,8 +1157,10 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
             const uint32_t vb = pack_bf16(w0[j] * inv, w1[j] * inv);
             kr[i] = kb;
             vr[i] = vb;
-            reinterpret_cast<uint32_t*>(a.k_cache + grow)[i] = kb;
-            reinterpret_cast<uint32_t*>(a.v_cache + grow)[i] = vb;
+            if (wrow) {
+              reinterpret_cast<uint32_t*>(a.k_cache + grow)[i] = kb;
+              reinterpret_cast<uint32_t*>(a.v_cache + grow)[i] = vb;
+            }
           }
         }
         if (lane == 0) {
@@ -996,13 +1172,14 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           dsc->k1 = pc.k1;
           dsc->l = l;
           dsc->gi = gi;
-          dsc->c0 = (int32_t)udiv_pos(pa, gp.P[gi]);
-          dsc->c1 = (int32_t)udiv_pos(pa + lens[pc.s] - 1, gp.P[gi]);
+          dsc->c0 = (int32_t)part_cta(pa, gp.P[gi], align);
+          dsc->c1 = (int32_t)part_cta(pa + lens[pc.s] - 1, gp.P[gi], align);
           dsc->app_row = app ? lens[pc.s] - 1 : -1;
           dsc->end = 0;
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(bar_qfull + 8 * slot);
+      }
       }
     }
     // end marker for the consumers
@@ -1259,21 +1436,45 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     ss = warp_sum(ss);
     uint64_t* ps = a.part_ss + ((int64_t)nx * S + pc.s) * Hkv * ATT_CONSUMERS;
     if (lane == 0) st_tagged(ps + pc.h * ATT_CONSUMERS + warp, ss, ntag);
-    if (l + 1 < a.L) continue;
-    // after the last layer: head group h of the final hidden state
-    float inv;
-    if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, ntag, d, a.rms_eps, lane, a.status, inv)) {
-      ok = false;
-      break;
-    }
-    if (own) {
-      __nv_bfloat16* hs = a.hidden + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0;
-      __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0 : nullptr;
+  }
+  // Final hidden state, head group h of every segment this CTA completed at
+  // the last layer.  It needs the sums of all the sequence's head groups, so
+  // it waits here, after this CTA has done all its merges: a wait inside the
+  // loop could close a cycle (two CTAs each waiting for a merge the other
+  // would only do later).  The CTA's pieces are walked again to find them.
+  if (ok && a.L > 0) {
+    const int nx = a.L & 1;
+    const uint32_t ntag = step_tag(epoch, a.L);
+    const bool own = tid < GD / 4;
+    const int idx0 = own ? 4 * tid : 0;
+    for (int gi = 0; gi < gp.n && ok; ++gi) {
+      Piece pc;
+      pc.adv = -1;  // none yet
+      for (int64_t pp = gp.cb[gi]; pp < gp.ce[gi] && ok;) {
+        pc = pc.adv < 0 ? find_piece(pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead)
+                        : next_piece(pc, pre, lens, gp.s_lo[gi], gp.s_lo[gi + 1], gp.T[gi], pp, gp.ce[gi], a.seg_lead);
+        pp += pc.adv;
+        if (pc.k0 == pc.k1) continue;
+        const int64_t pa = (int64_t)pc.h * gp.T[gi] + pre[pc.s] - pre[gp.s_lo[gi]] + a.seg_lead;  // first key
+        if (part_cta(pa, gp.P[gi], align) != (int64_t)blockIdx.x) continue;  // completed by another CTA
+        const uint64_t* ps = a.part_ss + ((int64_t)nx * S + pc.s) * Hkv * ATT_CONSUMERS;
+        float inv;
+        if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, ntag, d, a.rms_eps, lane, a.status, inv)) {
+          ok = false;
+          break;
+        }
+        if (own) {
+          // x_L as this thread stored it when it completed the segment
+          const uint64_t* xn = a.resid + ((int64_t)nx * S + pc.s) * d + (int64_t)pc.h * GD + idx0;
+          __nv_bfloat16* hs = a.hidden + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0;
+          __nv_bfloat16* hc = a.hidden_copy ? a.hidden_copy + (int64_t)pc.s * d + (int64_t)pc.h * GD + idx0 : nullptr;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const __nv_bfloat16 hv2 = __float2bfloat16_rn(xv[j] * inv);
-        hs[j] = hv2;
-        if (hc) hc[j] = hv2;
+          for (int j = 0; j < 4; ++j) {
+            const __nv_bfloat16 hv2 = __float2bfloat16_rn(tv_value(xn[j]) * inv);
+            hs[j] = hv2;
+            if (hc) hc[j] = hv2;
+          }
+        }
       }
     }
   }

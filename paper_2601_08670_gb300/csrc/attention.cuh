@@ -15,6 +15,7 @@ constexpr int ATT_MAX_G = 8;        // query heads per kv-head (mma N = 8)
 constexpr int ATT_MAX_CTAS = 1024;  // upper bound of the grid (sizes the partial-record pool)
 constexpr float ATT_RESCALE_SLACK = 8.f;  // log2 units the online-softmax reference may trail the max
 constexpr int ATT_MAX_GROUPS = 4;   // sequence groups of the step kernel
+constexpr int ATT_PTAB = 1024;       // block-table entries a step-kernel CTA keeps in shared memory
 
 // ---------------------------------------------------------------- one layer
 // Partition of all (kv-head, sequence, key) positions into equal contiguous
@@ -65,7 +66,10 @@ cudaError_t att_combine_launch(const CombineArgs& a, cudaStream_t stream);
 // Partition: head-major positions as above, but each segment (h, s) spans
 // len[s] + seg_cost positions; the last seg_cost hold no keys and stand for
 // the fixed cost of a piece (query formation, partial merge, record), so CTAs
-// that cover many short segments get fewer keys.  The partition is the same
+// that cover many short segments get fewer keys.  With paged caches the
+// extents are rounded up to whole 64-key tiles and the CTA boundaries down to
+// multiples of 64 positions, so every piece starts on a tile boundary and no
+// tile straddles two blocks (blocks hold a multiple of 64 rows).  The partition is the same
 // at every layer, so the producer warp streams K/V tiles straight through all
 // layers (a shared-memory ring plus L2 prefetch ahead of it) while the
 // consumers wait for the layer dependency.
@@ -103,8 +107,11 @@ struct StepAttArgs {
   int32_t seg_lead;           // how many of the seg_cost positions come before the keys (the rest after)
   int32_t pf_tiles;           // tiles prefetched into L2 ahead of the shared-memory ring
   int32_t groups;             // sequence groups (1..ATT_MAX_GROUPS), each partitioned over all CTAs
-  const int64_t* kv_offset;   // [S]
+  const int64_t* kv_offset;   // [S] (slab layout)
   const int32_t* cap;         // [S]
+  const int32_t* block_table; // [S][max_blocks] (paged layout) or null
+  int32_t block_rows, max_blocks, num_blocks;
+  int32_t block_shift;        // log2(block_rows) when it is a power of two, else -1
   int32_t* seq_len;           // [S] +1 per launch for every sequence with room
   const int32_t* step;        // [1] step counter t (token y_{t-1} = history[b][t-1])
   const int32_t* history;     // [B][max_steps]

@@ -91,7 +91,8 @@ extern "C" const char* pced_step_launch_kind(const pced_dims* dm, int32_t i) {
 extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (!p) return fail(PCED_ERR_INVALID_ARG, "pced_step: null args");
   const pced_dims dm = p->dims;
-  if (!p->embed || !p->w_unembed || !p->k_cache || !p->v_cache || !p->kv_offset || !p->cap || !p->seq_len ||
+  const bool paged = p->block_table != nullptr;
+  if (!p->embed || !p->w_unembed || !p->k_cache || !p->v_cache || (!paged && !p->kv_offset) || !p->cap || !p->seq_len ||
       !p->step || !p->history || !p->beta || !p->r || !p->workspace || (p->beta_from_step && !p->beta_out))
     return fail(PCED_ERR_INVALID_ARG, "pced_step: null pointer");
   if (dm.B < 1 || dm.N < 1 || dm.L < 1 || dm.Hq < 1 || dm.Hkv < 1 || dm.D < 1 || dm.V < 1 || dm.Hq % dm.Hkv != 0 ||
@@ -108,6 +109,18 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (d > 8192) return fail(PCED_ERR_UNSUPPORTED, "pced_step: hidden size %d > 8192", d);
   if (p->layer_elems % dm.D != 0 || (int64_t)dm.L * (p->layer_elems / dm.D) >= ((int64_t)1 << 31))
     return fail(PCED_ERR_UNSUPPORTED, "pced_step: cache too large for 32-bit row coordinates");
+  int64_t num_blocks = 0;
+  if (paged) {
+    if (p->block_rows < ATT_BLOCK_N || p->block_rows % ATT_BLOCK_N != 0 || p->max_blocks < 1)
+      return fail(PCED_ERR_INVALID_ARG, "pced_step: block_rows must be a positive multiple of %d", ATT_BLOCK_N);
+    if ((int64_t)S * p->max_blocks >= ((int64_t)1 << 31))
+      return fail(PCED_ERR_UNSUPPORTED, "pced_step: block table too large for 32-bit entry indices");
+    const int64_t block_elems = (int64_t)dm.Hkv * p->block_rows * dm.D;
+    if (p->layer_elems % block_elems != 0)
+      return fail(PCED_ERR_INVALID_ARG, "pced_step: layer_elems is not a whole number of blocks");
+    num_blocks = p->layer_elems / block_elems;
+    if (num_blocks >= ((int64_t)1 << 31)) return fail(PCED_ERR_UNSUPPORTED, "pced_step: too many blocks");
+  }
   LmGeom g;
   if (!lm_geometry(S, d, dm.V, &g)) return fail(PCED_ERR_UNSUPPORTED, "pced_step: LM-head shape unsupported");
   if ((((uintptr_t)p->k_cache) | ((uintptr_t)p->v_cache) | ((uintptr_t)p->w_unembed) | ((uintptr_t)p->embed)) & 15u)
@@ -159,8 +172,23 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   at.pf_tiles = att_step_pf_tiles();
   at.groups = att_step_groups();
   at.seg_lead = att_step_seg_lead(at.seg_cost);
+  if (paged) {
+    // whole tiles: with every extent, lead and CTA share a multiple of the
+    // tile size, each piece starts on a tile (and so block) boundary
+    at.seg_cost = (at.seg_cost + ATT_BLOCK_N - 1) & ~(ATT_BLOCK_N - 1);
+    at.seg_lead = (at.seg_lead + ATT_BLOCK_N - 1) & ~(ATT_BLOCK_N - 1);
+    if (at.seg_lead > at.seg_cost) at.seg_lead = at.seg_cost;
+  }
   at.kv_offset = p->kv_offset;
   at.cap = p->cap;
+  at.block_table = p->block_table;
+  at.block_rows = paged ? p->block_rows : 0;
+  at.max_blocks = paged ? p->max_blocks : 0;
+  at.num_blocks = (int32_t)num_blocks;
+  at.block_shift = -1;
+  if (paged && (p->block_rows & (p->block_rows - 1)) == 0)
+    for (at.block_shift = 0; (1 << at.block_shift) < p->block_rows; ++at.block_shift) {
+    }
   at.seq_len = p->seq_len;
   at.step = p->step;
   at.history = p->history;

@@ -201,6 +201,45 @@ def cache_layout(w: Workload, base_len: np.ndarray, extra: int | None = None) ->
     return CacheLayout(cap=cap, kv_offset=off, layer_elems=int(sizes.sum()), L=w.L, Hkv=w.Hkv, D=w.D)
 
 
+@dataclass
+class PagedLayout:
+    """Paged KV layout: each layer's pool is num_blocks blocks of [Hkv][P][D];
+    row pos of (sequence s, kv-head h) lives in block table[s][pos // P], row
+    pos % P.  Blocks are handed out in a seeded random order (a serving
+    allocator's scattered pages)."""
+    P: int
+    table: np.ndarray      # [S][max_blocks] int32 (-1 past a sequence's blocks)
+    num_blocks: int
+    cap: np.ndarray        # [S] int32 logical capacity (rows)
+    layer_elems: int
+    L: int
+    Hkv: int
+    D: int
+
+    @property
+    def max_blocks(self) -> int:
+        return int(self.table.shape[1])
+
+    @property
+    def total_elems(self) -> int:
+        return self.L * self.layer_elems
+
+
+def paged_layout(w: Workload, base_len: np.ndarray, P: int, extra: int | None = None) -> PagedLayout:
+    extra = w.steps if extra is None else extra
+    cap = (base_len.astype(np.int64) + extra).astype(np.int32)
+    nblk = (cap.astype(np.int64) + P - 1) // P
+    num_blocks = int(nblk.sum())
+    order = np.random.default_rng([w.seed, 0x9A6E]).permutation(num_blocks).astype(np.int32)
+    table = np.full((len(cap), int(nblk.max())), -1, np.int32)
+    at = 0
+    for s, n in enumerate(nblk):
+        table[s, :n] = order[at:at + n]
+        at += n
+    return PagedLayout(P=P, table=table, num_blocks=num_blocks, cap=cap,
+                       layer_elems=num_blocks * w.Hkv * P * w.D, L=w.L, Hkv=w.Hkv, D=w.D)
+
+
 def kv_bytes_per_token(L: int, Hkv: int, D: int, elem_bytes: int = 2) -> int:
     """K and V bytes one token occupies across all layers."""
     return L * 2 * Hkv * D * elem_bytes
@@ -278,6 +317,8 @@ def dev_lib():
                                     ctypes.c_uint32, ctypes.c_float)
         lib.synth_dev_fill_cache.argtypes = [P, I64, P, P, P, P, I32, I32, I32, I32, U64, U32, F, P]
         lib.synth_dev_fill_cache.restype = ctypes.c_int
+        lib.synth_dev_fill_cache_paged.argtypes = [P, I64, P, I32, I32, P, P, I32, I32, I32, I32, U64, U32, F, P]
+        lib.synth_dev_fill_cache_paged.restype = ctypes.c_int
         lib.synth_dev_fill_matrix.argtypes = [P, I64, I64, I64, U64, U32, F, P]
         lib.synth_dev_fill_matrix.restype = ctypes.c_int
         _dev = lib
@@ -352,26 +393,42 @@ def host_normal_bf16(n: int, seed: int, sigma: float = 1.0) -> np.ndarray:
     return out
 
 
-def device_inputs(w: Workload, device="cuda", extra_steps: int | None = None, stream=None) -> dict:
+def device_inputs(w: Workload, device="cuda", extra_steps: int | None = None, stream=None,
+                  paged: int = 0) -> dict:
     """All inputs of workload `w` as device tensors: caches with generated
     prefixes (zeros after), embedding, unembedding, lengths, layout tables,
-    beta and r.  Generated on the device with the same bits as the host fills."""
+    beta and r.  Generated on the device with the same bits as the host fills.
+    paged = P > 0 stores the caches in the paged layout with P-row blocks
+    (keys "block_table", "block_rows", "paged_layout"); the logical cache
+    contents are the same."""
     import torch
     stream = torch.cuda.current_stream() if stream is None else stream
     sp = stream.cuda_stream
     bl = base_lengths(w)
-    lay = cache_layout(w, bl, extra_steps)
+    lay = paged_layout(w, bl, paged, extra_steps) if paged else cache_layout(w, bl, extra_steps)
     k = torch.zeros(lay.total_elems, dtype=torch.bfloat16, device=device)
     v = torch.zeros(lay.total_elems, dtype=torch.bfloat16, device=device)
-    kv_off = torch.from_numpy(lay.kv_offset).to(device)
     cap = torch.from_numpy(lay.cap).to(device)
     base = torch.from_numpy(bl).to(device)
     ids = torch.arange(w.S, dtype=torch.int32, device=device)
-    dev_fill_caches(w, lay.layer_elems, k, v, kv_off, cap, base, ids, sp)
+    extra = {}
+    if paged:
+        table = torch.from_numpy(lay.table).to(device)
+        kv_off = torch.zeros(w.S, dtype=torch.int64, device=device)
+        for tensor, buf in ((T_KCACHE, k), (T_VCACHE, v)):
+            rc = dev_lib().synth_dev_fill_cache_paged(buf.data_ptr(), int(lay.layer_elems), table.data_ptr(),
+                                                      lay.max_blocks, paged, base.data_ptr(), ids.data_ptr(), w.S,
+                                                      w.L, w.Hkv, w.D, w.seed, tensor, normal_scale(SIGMA_KV), sp)
+            if rc != 0:
+                raise RuntimeError(f"synth_dev_fill_cache_paged failed: cuda error {rc}")
+        extra = dict(block_table=table, block_rows=paged, paged_layout=lay)
+    else:
+        kv_off = torch.from_numpy(lay.kv_offset).to(device)
+        dev_fill_caches(w, lay.layer_elems, k, v, kv_off, cap, base, ids, sp)
     emb = torch.empty((w.V, w.d), dtype=torch.bfloat16, device=device)
     wu = torch.empty((w.V, w.d), dtype=torch.bfloat16, device=device)
     dev_fill_matrix(w, T_EMBED, emb, sp)
     dev_fill_matrix(w, T_UNEMBED, wu, sp)
     return dict(k_cache=k, v_cache=v, kv_offset=kv_off, cap=cap, seq_len=base.clone(), base_len=bl, layout=lay,
                 embed=emb, w_unembed=wu, beta=torch.from_numpy(betas(w)).to(device),
-                r=torch.from_numpy(retrieval_scores(w)).to(device))
+                r=torch.from_numpy(retrieval_scores(w)).to(device), **extra)
