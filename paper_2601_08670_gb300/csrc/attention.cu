@@ -666,25 +666,30 @@ __device__ __forceinline__ int64_t part_cta(int64_t x, int64_t Pg, int32_t align
 }
 
 // Tile cursor over a CTA's ranges through all layers and groups (the
-// producer's order: layer by layer, group by group), carrying the
-// tensor-map row of its tile.  Slab caches: the slab's row + kt.  Paged
-// caches: pieces start on 64-key boundaries (tile-aligned partition), so a
-// tile never straddles two blocks, and the row is row kt % P of block
-// table[s][kt / P], advanced without a division and looked up once per block.  A bad block id (flagged) points the tile past
-// the last row of the tensor map, where the loads read zeros.
+// producer's order: layer by layer, group by group).  Slab caches: the tile's
+// tensor-map row is the slab's first row + kt.  Paged caches (PAGED): pieces
+// start on 64-key boundaries (tile-aligned partition), so a tile never
+// straddles two blocks; the row, row kt % P of block table[s][kt / P], is
+// advanced without a division, the block is looked up once (in the CTA's
+// shared copy) and the next piece is found without a search.  A bad block id
+// (flagged) points the tile past the last row of the tensor map, where the
+// loads read zeros.
+template <bool PAGED>
 struct TileCursor {
   int32_t l, g, kt;
-  int32_t row;      // tensor-map row of the tile
+  int64_t p, row0;  // slab caches: tensor-map row of key 0 of the current piece
+  int32_t row;      // paged caches: tensor-map row of the tile
   bool bad;         // paged caches: the tile's block id is outside the pool
-  int64_t p;
   int32_t kin, bj;  // paged caches: key offset of the tile in its block, the block's index
   int32_t bi, ptn;  // paged caches: block-table copy entry of block bj; of the next piece's first block
   Piece pc;
   bool ok;
+  __device__ __forceinline__ int32_t tile_row() const { return PAGED ? row : (int32_t)(row0 + kt); }
 };
 
-// cont: c.pc is the piece before position c.p in the same group
-__device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
+// cont (paged caches): c.pc is the piece before position c.p in the same group
+template <bool PAGED>
+__device__ __forceinline__ void cursor_seek(TileCursor<PAGED>& c, const StepAttArgs& a, const int64_t* pre,
                                             const int32_t* lens, const GroupPlan& gp, int D, const int32_t* ptab,
                                             int32_t ptab_n, bool cont) {
   while (true) {
@@ -701,19 +706,18 @@ __device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a,
       cont = false;
       continue;
     }
-    c.pc = cont ? next_piece(c.pc, pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead)
-                : find_piece(pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead);
+    if (PAGED && cont)
+      c.pc = next_piece(c.pc, pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead);
+    else
+      c.pc = find_piece(pre, lens, gp.s_lo[c.g], gp.s_lo[c.g + 1], gp.T[c.g], c.p, gp.ce[c.g], a.seg_lead);
     cont = true;
     if (c.pc.k0 < c.pc.k1) {
-      if (!a.block_table) {
-        c.kt = c.pc.k0;
-        c.row = (int32_t)((int64_t)c.l * a.rows_per_layer +
-                          (__ldg(a.kv_offset + c.pc.s) + (int64_t)c.pc.h * __ldg(a.cap + c.pc.s) * D) / D + c.kt);
-        c.bad = false;
+      c.kt = c.pc.k0;
+      if (!PAGED) {
+        c.row0 = (int64_t)c.l * a.rows_per_layer + (a.kv_offset[c.pc.s] + (int64_t)c.pc.h * a.cap[c.pc.s] * D) / D;
         return;
       }
-      c.kt = c.pc.k0;  // a multiple of 64 (tile-aligned partition)
-      c.bj = block_of(a, c.kt);
+      c.bj = block_of(a, c.kt);  // kt is a multiple of 64 (tile-aligned partition)
       c.kin = c.kt - c.bj * a.block_rows;
       c.bi = c.ptn;
       c.ptn += block_of(a, c.pc.k1 - 1) - c.bj + 1;
@@ -725,22 +729,25 @@ __device__ __forceinline__ void cursor_seek(TileCursor& c, const StepAttArgs& a,
     c.p += c.pc.adv;
   }
 }
-__device__ __forceinline__ void cursor_begin(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
+template <bool PAGED>
+__device__ __forceinline__ void cursor_begin(TileCursor<PAGED>& c, const StepAttArgs& a, const int64_t* pre,
                                              const int32_t* lens, const GroupPlan& gp, int D, const int32_t* ptab,
                                              int32_t ptab_n) {
   c.l = 0;
   c.g = 0;
   c.p = gp.cb[0];
   c.ptn = 0;
+  c.bad = false;
   c.ok = a.L > 0;
   if (c.ok) cursor_seek(c, a, pre, lens, gp, D, ptab, ptab_n, false);
 }
-__device__ __forceinline__ void cursor_next(TileCursor& c, const StepAttArgs& a, const int64_t* pre,
+template <bool PAGED>
+__device__ __forceinline__ void cursor_next(TileCursor<PAGED>& c, const StepAttArgs& a, const int64_t* pre,
                                             const int32_t* lens, const GroupPlan& gp, int D, const int32_t* ptab,
                                             int32_t ptab_n) {
   c.kt += ATT_BLOCK_N;
   if (c.kt < c.pc.k1) {
-    if (a.block_table) {
+    if (PAGED) {
       c.kin += ATT_BLOCK_N;
       if (c.kin == a.block_rows) {
         c.kin = 0;
@@ -749,14 +756,67 @@ __device__ __forceinline__ void cursor_next(TileCursor& c, const StepAttArgs& a,
         const int32_t b0 = block_base(a, c.pc.s, c.pc.h, c.bj, c.bi, ptab, ptab_n);
         c.bad = b0 < 0;
         c.row = (int32_t)(c.bad ? (int64_t)a.L * a.rows_per_layer : (int64_t)c.l * a.rows_per_layer + b0);
-        return;
+      } else if (!c.bad) {
+        c.row += ATT_BLOCK_N;
       }
     }
-    if (!c.bad) c.row += ATT_BLOCK_N;
     return;
   }
   c.p += c.pc.adv;
   cursor_seek(c, a, pre, lens, gp, D, ptab, ptab_n, true);
+}
+
+// The producer: K/V tiles of every layer in consumption order into the
+// NST-stage ring; the L2 prefetch cursor runs pf_tiles ahead so HBM keeps
+// streaming while the ring is full.  One thread.
+template <int D, bool PAGED>
+__device__ __forceinline__ void produce_tiles(const CUtensorMap* kmap, const CUtensorMap* vmap, const StepAttArgs& a,
+                                              const int64_t* pre, const int32_t* lens, const GroupPlan& gp,
+                                              const int32_t* ptab, int32_t ptab_n, uint32_t base, uint32_t NST,
+                                              uint32_t bar_full, uint32_t bar_empty) {
+  using C = AttCfg<D>;
+  const uint64_t pol = policy_evict_first();
+  TileCursor<PAGED> ld, pf;
+  cursor_begin(ld, a, pre, lens, gp, D, ptab, ptab_n);
+  cursor_begin(pf, a, pre, lens, gp, D, ptab, ptab_n);
+  for (int i = 0; i < a.pf_tiles && pf.ok; ++i) {
+    if (!pf.bad) {
+      tma_prefetch_l2_3d(kmap, 0, pf.tile_row(), 0);
+      tma_prefetch_l2_3d(vmap, 0, pf.tile_row(), 0);
+    }
+    cursor_next(pf, a, pre, lens, gp, D, ptab, ptab_n);
+  }
+  uint32_t it = 0, st = 0, ph = 0;
+  bool ok = true;
+  while (ld.ok) {
+    if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
+      ok = false;
+      break;
+    }
+    const uint32_t fb = bar_full + 8 * st;
+    const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
+    mbar_arrive_expect_tx(fb, C::STAGE_BYTES);
+    const int32_t row = ld.tile_row();
+    tma_load_3d(sk, kmap, fb, 0, row, 0, pol);
+    tma_load_3d(sv, vmap, fb, 0, row, 0, pol);
+    ++it;
+    if (++st == NST) {
+      st = 0;
+      ph ^= 1u;
+    }
+    cursor_next(ld, a, pre, lens, gp, D, ptab, ptab_n);
+    if (pf.ok) {
+      if (!pf.bad) {
+        tma_prefetch_l2_3d(kmap, 0, pf.tile_row(), 0);
+        tma_prefetch_l2_3d(vmap, 0, pf.tile_row(), 0);
+      }
+      cursor_next(pf, a, pre, lens, gp, D, ptab, ptab_n);
+    }
+  }
+  if (!ok) {
+    for (uint32_t j = (it >= NST ? it - NST : 0); j < it; ++j)
+      mbar_wait(bar_full + 8 * (j % NST), (j / NST) & 1u, a.status);
+  }
 }
 
 // 1/rms of x_l[s] from its Hkv per-group sums of squares (waits for all of
@@ -972,50 +1032,11 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
 
   if (warp == STEP_PRODUCER) {
     // ------------------------------------------------------------ producer
-    // K/V tiles of every layer in consumption order; the L2 prefetch cursor
-    // runs pf_tiles ahead so HBM keeps streaming while the ring is full
     if (lane == 0) {
-      const uint64_t pol = policy_evict_first();
-      TileCursor ld, pf;
-      cursor_begin(ld, a, pre, lens, gp, D, ptab, ptab_n);
-      cursor_begin(pf, a, pre, lens, gp, D, ptab, ptab_n);
-      for (int i = 0; i < a.pf_tiles && pf.ok; ++i) {
-        if (!pf.bad) {
-          tma_prefetch_l2_3d(&kmap, 0, pf.row, 0);
-          tma_prefetch_l2_3d(&vmap, 0, pf.row, 0);
-        }
-        cursor_next(pf, a, pre, lens, gp, D, ptab, ptab_n);
-      }
-      uint32_t it = 0, st = 0, ph = 0;
-      bool ok = true;
-      while (ld.ok) {
-        if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
-          ok = false;
-          break;
-        }
-        const uint32_t fb = bar_full + 8 * st;
-        const uint32_t sk = base + st * C::STAGE_BYTES, sv = sk + C::TILE_BYTES;
-        mbar_arrive_expect_tx(fb, C::STAGE_BYTES);
-        tma_load_3d(sk, &kmap, fb, 0, ld.row, 0, pol);
-        tma_load_3d(sv, &vmap, fb, 0, ld.row, 0, pol);
-        ++it;
-        if (++st == NST) {
-          st = 0;
-          ph ^= 1u;
-        }
-        cursor_next(ld, a, pre, lens, gp, D, ptab, ptab_n);
-        if (pf.ok) {
-          if (!pf.bad) {
-            tma_prefetch_l2_3d(&kmap, 0, pf.row, 0);
-            tma_prefetch_l2_3d(&vmap, 0, pf.row, 0);
-          }
-          cursor_next(pf, a, pre, lens, gp, D, ptab, ptab_n);
-        }
-      }
-      if (!ok) {
-        for (uint32_t j = (it >= NST ? it - NST : 0); j < it; ++j)
-          mbar_wait(bar_full + 8 * (j % NST), (j / NST) & 1u, a.status);
-      }
+      if (a.block_table)
+        produce_tiles<D, true>(&kmap, &vmap, a, pre, lens, gp, ptab, ptab_n, base, NST, bar_full, bar_empty);
+      else
+        produce_tiles<D, false>(&kmap, &vmap, a, pre, lens, gp, ptab, ptab_n, base, NST, bar_full, bar_empty);
     }
     return;
   }
