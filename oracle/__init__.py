@@ -39,7 +39,8 @@ def build(force: bool = False) -> str:
 class _Dims(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("N", ctypes.c_int32), ("L", ctypes.c_int32), ("Hq", ctypes.c_int32),
                 ("Hkv", ctypes.c_int32), ("D", ctypes.c_int32), ("V", ctypes.c_int32),
-                ("gamma", ctypes.c_double), ("rms_eps", ctypes.c_double), ("attn_scale", ctypes.c_double)]
+                ("gamma", ctypes.c_double), ("rms_eps", ctypes.c_double), ("attn_scale", ctypes.c_double),
+                ("rope_theta", ctypes.c_double)]
 
 
 _lib = None
@@ -69,6 +70,8 @@ def lib():
         L.oracle_decode_step_ex.restype = I32
         L.oracle_adacad_beta.argtypes = [P, I32, I32, I32, P]
         L.oracle_adacad_beta.restype = I32
+        L.oracle_rope.argtypes = [P, I32, I64, F64, P]
+        L.oracle_rope.restype = None
         _lib = L
     return _lib
 
@@ -153,6 +156,15 @@ def contrastive_select(lp, beta, r, gamma, B, N):
     return dict(token=tok, expert=exp_, score=sc, token_gap=tg, expert_gap=eg)
 
 
+def rope(x, pos: int, theta: float) -> np.ndarray:
+    """Rotary embedding of one head x [D] at position pos (rotate-half
+    pairing, fp32 angles; see oracle_rope)."""
+    x = _c(x, np.float64)
+    y = np.empty_like(x)
+    lib().oracle_rope(_p(x), x.size, int(pos), float(theta), _p(y))
+    return y
+
+
 def adacad_beta(lp, B, N):
     """Dynamic contrast strength (Sec. 3 after Eq. 2, as in AdaCAD): per
     expert, the Jensen-Shannon divergence in bits between its distribution
@@ -173,7 +185,7 @@ def decode_step(dims: dict, kc, vc, layer_elems, kv_off, cap, lens, emb_rows, w_
     (adacad_beta, rounded to fp32; returned as "beta")."""
     dm = _Dims(dims["B"], dims["N"], dims["L"], dims["Hq"], dims["Hkv"], dims["D"], dims["V"],
                float(dims["gamma"]), float(dims.get("rms_eps", RMS_EPS)),
-               float(dims.get("attn_scale", 1.0 / math.sqrt(dims["D"]))))
+               float(dims.get("attn_scale", 1.0 / math.sqrt(dims["D"]))), float(dims.get("rope_theta", 0.0)))
     B, N = dims["B"], dims["N"]
     S, d = B * (N + 1), dims["Hq"] * dims["D"]
     for a, t in ((kc, np.uint16), (vc, np.uint16), (lens, np.int32)):

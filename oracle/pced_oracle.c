@@ -266,6 +266,18 @@ int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, in
                                score, token_gap, expert_gap, h_out, lse_out, NULL, nthreads);
 }
 
+void oracle_rope(const double* x, int32_t D, int64_t pos, double theta, double* y) {
+  const int32_t half = D / 2;
+  for (int32_t f = 0; f < half; ++f) {
+    const float inv_freq = (float)pow(theta, -2.0 * (double)f / (double)D);
+    const float angle = (float)pos * inv_freq; /* fp32 product, as the models compute it */
+    const double c = cos((double)angle), sn = sin((double)angle);
+    const double a = x[f], b = x[f + half];
+    y[f] = a * c - b * sn;
+    y[f + half] = b * c + a * sn;
+  }
+}
+
 int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, int64_t layer_elems,
                               const int64_t* kv_off, const int32_t* cap, int32_t* len, const uint16_t* emb_rows,
                               const uint16_t* w, const float* beta, const float* r, int32_t* token, int32_t* expert,
@@ -276,18 +288,20 @@ int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc,
     return -1;
   const int32_t B = dm->B, N = dm->N, L = dm->L, Hq = dm->Hq, Hkv = dm->Hkv, D = dm->D, V = dm->V;
   if (B < 1 || N < 1 || L < 1 || Hkv < 1 || Hq % Hkv != 0 || 2 * Hkv > Hq || D < 1 || V < 1) return -1;
+  if (dm->rope_theta < 0.0 || (dm->rope_theta > 0.0 && D % 2 != 0)) return -1;
   const int32_t S = B * (N + 1), d = Hq * D;
   for (int32_t s = 0; s < S; ++s)
     if (len[s] < 0 || len[s] >= cap[s]) return -2;
 
   double* x = (double*)malloc(sizeof(double) * (size_t)S * d);  /* residual stream */
   double* xn = (double*)malloc(sizeof(double) * (size_t)d);
+  double* xq = (double*)malloc(sizeof(double) * (size_t)d); /* rotated query heads */
   uint16_t* u = (uint16_t*)malloc(sizeof(uint16_t) * (size_t)S * d); /* bf16 layer input */
   double* o = (double*)malloc(sizeof(double) * (size_t)S * d);
   double* lp = (double*)malloc(sizeof(double) * (size_t)S * V);
   double* lse = (double*)malloc(sizeof(double) * (size_t)S);
-  if (!x || !xn || !u || !o || !lp || !lse) {
-    free(x); free(xn); free(u); free(o); free(lp); free(lse);
+  if (!x || !xn || !xq || !u || !o || !lp || !lse) {
+    free(x); free(xn); free(xq); free(u); free(o); free(lp); free(lse);
     return -1;
   }
 
@@ -303,13 +317,19 @@ int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc,
     uint16_t* Vc = vc + (int64_t)l * layer_elems;
     for (int32_t s = 0; s < S; ++s) {
       oracle_rmsnorm(x + (int64_t)s * d, d, dm->rms_eps, xn);
-      for (int32_t i = 0; i < d; ++i) u[(int64_t)s * d + i] = oracle_round_bf16(xn[i]);
-      int64_t pos = len[s] - 1;
+      const int64_t pos = len[s] - 1; /* the new token's position */
+      for (int32_t hq = 0; hq < Hq; ++hq) {
+        if (dm->rope_theta > 0.0)
+          oracle_rope(xn + (int64_t)hq * D, D, pos, dm->rope_theta, xq + (int64_t)hq * D);
+        else
+          memcpy(xq + (int64_t)hq * D, xn + (int64_t)hq * D, sizeof(double) * (size_t)D);
+      }
+      for (int32_t i = 0; i < d; ++i) u[(int64_t)s * d + i] = oracle_round_bf16(xq[i]);
       for (int32_t h = 0; h < Hkv; ++h) {
         uint16_t* kr = K + kv_off[s] + ((int64_t)h * cap[s] + pos) * D;
         uint16_t* vr = Vc + kv_off[s] + ((int64_t)h * cap[s] + pos) * D;
         memcpy(kr, u + (int64_t)s * d + (int64_t)h * D, sizeof(uint16_t) * (size_t)D);
-        memcpy(vr, u + (int64_t)s * d + (int64_t)(Hkv + h) * D, sizeof(uint16_t) * (size_t)D);
+        for (int32_t i = 0; i < D; ++i) vr[i] = oracle_round_bf16(xn[(int64_t)(Hkv + h) * D + i]);
       }
     }
     oracle_attention(u, K, Vc, kv_off, cap, len, S, Hq, Hkv, D, dm->attn_scale, o, nthreads);
@@ -341,6 +361,6 @@ int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc,
   if (rc == 0)
     oracle_contrastive_select(lp, beta, r, dm->gamma, B, N, V, token, expert, score, token_gap, expert_gap);
 
-  free(x); free(xn); free(u); free(o); free(lp); free(lse);
+  free(x); free(xn); free(xq); free(u); free(o); free(lp); free(lse);
   return rc;
 }

@@ -62,18 +62,32 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
  * so 0 <= beta <= 1.  lp [S][V] as in oracle_contrastive_select. */
 int32_t oracle_adacad_beta(const double* lp, int32_t B, int32_t N, int32_t V, double* beta);
 
+/* Rotary position embedding of one head (the decoder LLM's positional
+ * encoding; the paper runs Llama / Qwen models, which use it), rotate-half
+ * pairing: for f < D/2, with angle a_f = fp32(pos * fp32(theta^(-2f/D)))
+ * (the fp32 angle of the models' reference implementations),
+ *   y[f]       = x[f] cos a_f - x[f + D/2] sin a_f,
+ *   y[f + D/2] = x[f + D/2] cos a_f + x[f] sin a_f,
+ * cos and sin evaluated in double.  D even, pos >= 0, theta > 0. */
+void oracle_rope(const double* x, int32_t D, int64_t pos, double theta, double* y);
+
 typedef struct oracle_dims {
   int32_t B, N, L, Hq, Hkv, D, V; /* S = B*(N+1), d = Hq*D, requires 2*Hkv <= Hq */
   double gamma;                   /* retrieval-prior weight of Eq. 2 */
   double rms_eps;                 /* RMSNorm epsilon */
   double attn_scale;              /* softmax scale, 1/sqrt(D) */
+  double rope_theta;              /* rotary base; 0: no rotary embedding */
 } oracle_dims;
 
 /* One full decode step of the synthetic PCED model.
  *   x_0[s]    = emb_rows[b]            (embedding of query b's previous token)
- *   per layer l:  u = bf16(rmsnorm(x_l[s]));  K_l[s][h][len] = u[h], V_l[s][h][len] = u[Hkv + h]
- *                 (h < Hkv, appended at the old length; the length grows by one per step)
- *                 x_{l+1}[s] = x_l[s] + attention(u as [Hq][D], K_l, V_l)
+ *   per layer l:  n = rmsnorm(x_l[s]);  q = bf16(R(n)) as [Hq][D];
+ *                 K_l[s][h][len] = q[h], V_l[s][h][len] = bf16(n[Hkv + h])
+ *                 (h < Hkv, appended at the old length = the token's position p;
+ *                 the length grows by one per step)
+ *                 x_{l+1}[s] = x_l[s] + attention(q, K_l, V_l)
+ *                 R: oracle_rope at position p on every head when
+ *                 rope_theta > 0, else the identity
  *   h[s]      = bf16(rmsnorm(x_L[s]))
  *   then the unembedding/log-softmax and Eq. 2 + Eq. 3 selection.
  * kc/vc span L layers of layer_elems elements (slab layout as in

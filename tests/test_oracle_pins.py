@@ -410,6 +410,85 @@ def test_step_appends_chosen_token_to_every_expert():
     assert 1 <= o2["expert"][0] <= w.N
 
 
+# --------------------------------------------------- rotary position embedding
+# The decoder LLMs the paper runs (Llama, Qwen) rotate queries and keys by
+# position.  Reading: rotate-half pairing (f, f + D/2), inverse frequency
+# theta^(-2f/D), angle pos * inv_freq in fp32 as the models compute it.
+def test_rope_position_zero_is_identity():
+    x = rng0.normal(size=64)
+    assert np.array_equal(oracle.rope(x, 0, 5e5), x)
+
+
+def test_rope_two_dims_is_a_plane_rotation_by_the_position():
+    # D = 2: the only inverse frequency is theta^0 = 1, so the angle is pos
+    x = np.array([0.75, -1.25])
+    for pos in (1, 2, 7, 1000):
+        c, s_ = math.cos(pos), math.sin(pos)
+        want = np.array([x[0] * c - x[1] * s_, x[1] * c + x[0] * s_])
+        assert np.allclose(oracle.rope(x, pos, 1e4), want, rtol=0, atol=1e-15)
+
+
+def test_rope_frequencies_and_rotate_half_pairing():
+    # theta = 2^16, D = 16: inverse frequencies 4^-f are exact in fp32, so the
+    # angles are exactly pos * 4^-f; a unit vector on dimension f moves towards
+    # f + D/2 (and f + D/2 towards f, with the opposite sign)
+    D, theta, pos = 16, 65536.0, 37
+    for f in range(D // 2):
+        a = pos * 4.0 ** -f
+        e = np.zeros(D); e[f] = 1.0
+        y = oracle.rope(e, pos, theta)
+        want = np.zeros(D); want[f] = math.cos(a); want[f + D // 2] = math.sin(a)
+        assert np.allclose(y, want, rtol=0, atol=1e-15)
+        e = np.zeros(D); e[f + D // 2] = 1.0
+        y = oracle.rope(e, pos, theta)
+        want = np.zeros(D); want[f] = -math.sin(a); want[f + D // 2] = math.cos(a)
+        assert np.allclose(y, want, rtol=0, atol=1e-15)
+
+
+def test_rope_scores_depend_on_relative_position_only():
+    D, theta = 16, 65536.0  # exact angles, see above
+    q, k = rng0.normal(size=D), rng0.normal(size=D)
+    for m, n, t in ((5, 2, 11), (0, 9, 100), (300, 300, 7)):
+        a = oracle.rope(q, m, theta) @ oracle.rope(k, n, theta)
+        b = oracle.rope(q, m + t, theta) @ oracle.rope(k, n + t, theta)
+        assert abs(a - b) < 1e-12
+    # and it is a rotation: every (f, f + D/2) pair keeps its length
+    y = oracle.rope(q, 12345, 5e5)
+    assert np.allclose(np.hypot(y[:D // 2], y[D // 2:]), np.hypot(q[:D // 2], q[D // 2:]), rtol=1e-14)
+
+
+def test_step_with_rope_rotates_queries_and_keys_at_the_token_position_not_values():
+    # Two zero prefix rows, then this step's token at position 2.  The new K row
+    # is bf16(rope(n[h], 2)), the V row bf16(n[Hkv + h]) unrotated; attention of
+    # query head hq over keys (0, 0, k) gives e^s / (2 + e^s) * v with
+    # s = scale * (rotated q) . (rotated k).
+    dims, kc, vc, lay, off, cap, lens, emb, w = empty_prefix_case(1)
+    dims["rope_theta"] = 1e4
+    lens[:] = 2
+    Hq, Hkv, D = dims["Hq"], dims["Hkv"], dims["D"]
+    G = Hq // Hkv
+    beta = np.full((1, 1), 0.5, np.float32)
+    r = np.full((1, 1), 0.8, np.float32)
+    out = oracle.decode_step(dims, kc, vc, lay, off, cap, lens, emb, w, beta, r)
+    x = oracle.bf16_to_f64(emb[0])
+    n = (x / math.sqrt(np.mean(x * x) + oracle.RMS_EPS)).reshape(Hq, D)
+    q = np.stack([oracle.bf16_to_f64(bf16_bits(oracle.rope(n[hq], 2, 1e4))) for hq in range(Hq)])
+    v = np.stack([oracle.bf16_to_f64(bf16_bits(n[Hkv + h])) for h in range(Hkv)])
+    for s in range(2):
+        for h in range(Hkv):
+            base = off[s] + (h * cap[s] + 2) * D
+            assert np.array_equal(oracle.bf16_to_f64(kc[base:base + D]), q[h])
+            assert np.array_equal(oracle.bf16_to_f64(vc[base:base + D]), v[h])
+    scale = 1.0 / math.sqrt(D)
+    o = []
+    for hq in range(Hq):
+        sc = scale * (q[hq] @ q[hq // G])
+        o.append(math.exp(sc) / (2.0 + math.exp(sc)) * v[hq // G])
+    x1 = x + np.concatenate(o)
+    h = bf16_bits(x1 / math.sqrt(np.mean(x1 * x1) + oracle.RMS_EPS))
+    assert np.array_equal(out["h"][0], h) and np.array_equal(out["h"][1], h)
+
+
 # --------------------------------------------------------------- paper figures
 def test_kv_storage_example_from_paper():
     import json, os
