@@ -248,6 +248,14 @@ typedef struct pced_step_args {
   const int32_t* block_table;
   int32_t block_rows;
   int32_t max_blocks;
+  /* Rotary position embedding (the paper's decoders, Llama-3.1 / Mistral /
+   * Qwen3, are rotary models): when rope_theta > 0 the queries and the
+   * appended key row of every layer are rotated by the new token's position
+   * p = seq_len[s] before the step (its row in the cache), rotate-half
+   * pairing (f, f + D/2) with angle fp32(p * fp32(rope_theta^(-2f/D))); the
+   * value row is not rotated and the cached rows are taken as stored (already
+   * rotated).  0: no rotation.  Negative or non-finite: PCED_ERR_INVALID_ARG. */
+  float rope_theta;
 } pced_step_args;
 
 size_t pced_step_workspace_size(const pced_dims* dims);

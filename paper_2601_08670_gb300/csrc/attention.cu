@@ -843,6 +843,26 @@ __device__ __forceinline__ bool wait_inv_rms(const uint64_t* part, int n, uint32
   }
 }
 
+// Rotary embedding of two rotate-half pairs: (a0, b0) at frequency f and
+// (a1, b1) at f + 1 (elements f, f + 1 and their partners f + D/2,
+// f + 1 + D/2); r = (cos, sin) of the two angles fp32(pos * inv_freq).
+struct RopePair {
+  float c0, s0, c1, s1;
+};
+__device__ __forceinline__ RopePair rope_angles(int f, float posf, const float* rope_f) {
+  RopePair r;
+  sincosf(__fmul_rn(posf, rope_f[f]), &r.s0, &r.c0);
+  sincosf(__fmul_rn(posf, rope_f[f + 1]), &r.s1, &r.c1);
+  return r;
+}
+__device__ __forceinline__ void rope_rotate(float& a0, float& a1, float& b0, float& b1, const RopePair& r) {
+  const float x0 = a0, x1 = a1;
+  a0 = x0 * r.c0 - b0 * r.s0;
+  b0 = b0 * r.c0 + x0 * r.s0;
+  a1 = x1 * r.c1 - b1 * r.s1;
+  b1 = b1 * r.c1 + x1 * r.s1;
+}
+
 // What the input warp tells the consumers about the piece in a hand-off slot
 // (the consumers take their pieces from the slots, in the input warp's order).
 struct PieceDesc {
@@ -866,6 +886,7 @@ struct StepSmem {
   uint32_t misc;        // flags
   uint32_t tables;      // pre[ATT_MAX_S+1] int64, GroupPlan, lens[ATT_MAX_S] int32, apnd[ATT_MAX_S] u8
   uint32_t ptab;        // block-table copy: ptab[ATT_PTAB] int32, its entry count, ptab_h[ATT_PTAB] u8
+  uint32_t rope;        // rotary inverse frequencies [D/2] fp32
   uint32_t total;       // bytes to request, alignment slack included
 };
 __host__ __device__ inline StepSmem step_smem(int D, int G) {
@@ -884,7 +905,8 @@ __host__ __device__ inline StepSmem step_smem(int D, int G) {
     L.misc = L.pbuf + 2u * L.pslot;
     L.tables = L.misc + 64u;
     L.ptab = L.tables + ((tables + 15u) & ~15u);
-    L.total = 1024u + L.ptab + ATT_PTAB * 5u + 16u;
+    L.rope = (L.ptab + ATT_PTAB * 5u + 16u + 15u) & ~15u;
+    L.total = 1024u + L.rope + 4u * (uint32_t)(D / 2);
     if (L.total <= 227u * 1024u) break;
   }
   return L;
@@ -946,6 +968,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   int32_t* ptab = reinterpret_cast<int32_t*>(gbase + SL.ptab);
   int32_t* ptab_cnt = ptab + ATT_PTAB;
   uint8_t* ptab_h = reinterpret_cast<uint8_t*>(ptab_cnt + 4);  // kv-head of each entry (while building)
+  float* rope_f = reinterpret_cast<float*>(gbase + SL.rope);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int32_t epoch = *a.epoch;
@@ -971,6 +994,8 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   // the next grid (LM head) may be scheduled as SMs free up; it waits for
   // this grid's completion before reading the hidden states
   pdl_launch_dependents();
+  // rotary inverse frequencies theta^(-2f/D), rounded to fp32
+  if (a.rope_theta > 0.f && tid < D / 2) rope_f[tid] = (float)pow((double)a.rope_theta, -2.0 * tid / D);
   // lengths after this step's append (a full cache appends nothing)
   for (int i = tid; i < S; i += STEP_THREADS) {
     int32_t n = a.seq_len[i];
@@ -1082,29 +1107,42 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         uint32_t* qw = reinterpret_cast<uint32_t*>(gbase + SL.qbuf + slot * SL.qslot);
         float* xr = reinterpret_cast<float*>(qw + 8 * QW + D);  // x_l of the head group, for the completing CTA
         float inv = 0.f;
-        // query pairs (lane handles element pairs 2i, 2i+1 of the head group);
-        // the first chunk's poll also covers the group sums (one round trip)
-        for (int i0 = 0; i0 < GD / 2 && ok; i0 += 32 * 8) {
-          float v0[8], v1[8], t = 0.f;
+        // query elements by rotary quads: lane takes elements 2k, 2k+1 of head
+        // g and their rotate-half partners 2k + D/2, 2k + 1 + D/2 (quad
+        // m = g*D/4 + k); the first chunk's poll also covers the group sums
+        // (one round trip)
+        const bool rope = a.rope_theta > 0.f;
+        // this lane's two rotary frequencies are 2k, 2k + 1 with k = lane mod D/4
+        // for every quad it takes (D/4 divides 32); their angles only depend
+        // on the position, so they are found before the wait for x_l
+        static_assert(32 % (D / 4) == 0, "rotary quads per lane assume D/4 divides 32");
+        RopePair rp = {1.f, 0.f, 1.f, 0.f};
+        if (rope) rp = rope_angles(2 * (lane % (D / 4)), (float)(lens[pc.s] - apnd[pc.s]), rope_f);
+        for (int m0 = 0; m0 < GD / 4 && ok; m0 += 32 * 4) {
+          float v[4][4], t = 0.f;
           uint64_t t0 = 0;
           while (true) {
             bool good = true;
             t = 0.f;
-            if (i0 == 0)
+            if (m0 == 0)
               for (int i = lane; i < Hkv * ATT_CONSUMERS; i += 32) {
                 const uint64_t w = ld_tagged(ps + i);
                 good &= tv_ok(w, tag);
                 t += tv_value(w);
               }
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              const int i = i0 + lane + 32 * j;
-              v0[j] = v1[j] = 0.f;
-              if (i >= GD / 2) continue;
-              const uint64_t w0 = ld_tagged(xq + 2 * i), w1 = ld_tagged(xq + 2 * i + 1);
-              good &= tv_ok(w0, tag) && tv_ok(w1, tag);
-              v0[j] = tv_value(w0);
-              v1[j] = tv_value(w1);
+            for (int j = 0; j < 4; ++j) {
+              const int m = m0 + lane + 32 * j;
+              v[j][0] = v[j][1] = v[j][2] = v[j][3] = 0.f;
+              if (m >= GD / 4) continue;
+              const int e = (m / (D / 4)) * D + 2 * (m % (D / 4));
+              const uint64_t w0 = ld_tagged(xq + e), w1 = ld_tagged(xq + e + 1);
+              const uint64_t w2 = ld_tagged(xq + e + D / 2), w3 = ld_tagged(xq + e + D / 2 + 1);
+              good &= tv_ok(w0, tag) && tv_ok(w1, tag) && tv_ok(w2, tag) && tv_ok(w3, tag);
+              v[j][0] = tv_value(w0);
+              v[j][1] = tv_value(w1);
+              v[j][2] = tv_value(w2);
+              v[j][3] = tv_value(w3);
             }
             if (__all_sync(0xffffffffu, good)) break;
             if (!poll_again(t0, a.status)) {
@@ -1113,24 +1151,29 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
             }
           }
           if (!ok) break;
-          if (i0 == 0) {
+          if (m0 == 0) {
             // same summation order as every other user of these sums
             t = warp_sum(t);
             t = __shfl_sync(0xffffffffu, t, 0);
             inv = 1.0f / sqrtf(t / (float)d + a.rms_eps);
           }
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int i = i0 + lane + 32 * j;
-            if (i >= GD / 2) continue;
-            const int g = (2 * i) / D, dd = (2 * i) % D;
-            qw[g * QW + dd / 2] = pack_bf16(v0[j] * inv, v1[j] * inv);
-            xr[2 * i] = v0[j];
-            xr[2 * i + 1] = v1[j];
+          for (int j = 0; j < 4; ++j) {
+            const int m = m0 + lane + 32 * j;
+            if (m >= GD / 4) continue;
+            const int g = m / (D / 4), k = m % (D / 4), e = g * D + 2 * k;
+            float a0 = v[j][0] * inv, a1 = v[j][1] * inv, b0 = v[j][2] * inv, b1 = v[j][3] * inv;
+            if (rope) rope_rotate(a0, a1, b0, b1, rp);
+            qw[g * QW + k] = pack_bf16(a0, a1);
+            qw[g * QW + k + D / 4] = pack_bf16(b0, b1);
+            xr[e] = v[j][0];
+            xr[e + 1] = v[j][1];
+            xr[e + D / 2] = v[j][2];
+            xr[e + D / 2 + 1] = v[j][3];
           }
         }
         if (ok && app) {
-          // K row = head h of u, V row = head Hkv + h of u
+          // K row = head h of u (rotated like the queries), V row = head Hkv + h of u
           const uint64_t* xk = xs + (int64_t)pc.h * D;
           const uint64_t* xv = xs + ((int64_t)Hkv + pc.h) * D;
           uint32_t* kr = qw + 8 * QW;
@@ -1146,23 +1189,25 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           }
           const bool wrow = arow >= 0;  // a bad block id was flagged: keep the cache untouched
           const int64_t grow = (wrow ? arow : 0) * D;
-          constexpr int RW = (D / 2 + 31) / 32;  // word pairs per lane
-          float k0[RW], k1[RW], w0[RW], w1[RW];
+          constexpr int RQ = (D / 4 + 31) / 32;  // rotary quads per lane (as for the queries)
+          float kx[RQ][4], vx[RQ][4];
           uint64_t t0 = 0;
           while (true) {
             bool good = true;
 #pragma unroll
-            for (int j = 0; j < RW; ++j) {
-              const int i = lane + 32 * j;
-              k0[j] = k1[j] = w0[j] = w1[j] = 0.f;
-              if (i >= D / 2) continue;
-              const uint64_t a0 = ld_tagged(xk + 2 * i), a1 = ld_tagged(xk + 2 * i + 1);
-              const uint64_t b0 = ld_tagged(xv + 2 * i), b1 = ld_tagged(xv + 2 * i + 1);
-              good &= tv_ok(a0, tag) && tv_ok(a1, tag) && tv_ok(b0, tag) && tv_ok(b1, tag);
-              k0[j] = tv_value(a0);
-              k1[j] = tv_value(a1);
-              w0[j] = tv_value(b0);
-              w1[j] = tv_value(b1);
+            for (int j = 0; j < RQ; ++j) {
+              const int k = lane + 32 * j;
+#pragma unroll
+              for (int c = 0; c < 4; ++c) kx[j][c] = vx[j][c] = 0.f;
+              if (k >= D / 4) continue;
+              const int e[4] = {2 * k, 2 * k + 1, 2 * k + D / 2, 2 * k + 1 + D / 2};
+#pragma unroll
+              for (int c = 0; c < 4; ++c) {
+                const uint64_t wk = ld_tagged(xk + e[c]), wv = ld_tagged(xv + e[c]);
+                good &= tv_ok(wk, tag) && tv_ok(wv, tag);
+                kx[j][c] = tv_value(wk);
+                vx[j][c] = tv_value(wv);
+              }
             }
             if (__all_sync(0xffffffffu, good)) break;
             if (!poll_again(t0, a.status)) {
@@ -1171,16 +1216,24 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
             }
           }
 #pragma unroll
-          for (int j = 0; j < RW; ++j) {
-            const int i = lane + 32 * j;
-            if (!ok || i >= D / 2) continue;
-            const uint32_t kb = pack_bf16(k0[j] * inv, k1[j] * inv);
-            const uint32_t vb = pack_bf16(w0[j] * inv, w1[j] * inv);
-            kr[i] = kb;
-            vr[i] = vb;
+          for (int j = 0; j < RQ; ++j) {
+            const int k = lane + 32 * j;
+            if (!ok || k >= D / 4) continue;
+            float a0 = kx[j][0] * inv, a1 = kx[j][1] * inv, b0 = kx[j][2] * inv, b1 = kx[j][3] * inv;
+            if (rope) rope_rotate(a0, a1, b0, b1, rp);  // keys rotate, values do not
+            const uint32_t ka = pack_bf16(a0, a1), kb = pack_bf16(b0, b1);
+            const uint32_t va = pack_bf16(vx[j][0] * inv, vx[j][1] * inv), vb = pack_bf16(vx[j][2] * inv, vx[j][3] * inv);
+            kr[k] = ka;
+            kr[k + D / 4] = kb;
+            vr[k] = va;
+            vr[k + D / 4] = vb;
             if (wrow) {
-              reinterpret_cast<uint32_t*>(a.k_cache + grow)[i] = kb;
-              reinterpret_cast<uint32_t*>(a.v_cache + grow)[i] = vb;
+              uint32_t* gk = reinterpret_cast<uint32_t*>(a.k_cache + grow);
+              uint32_t* gv = reinterpret_cast<uint32_t*>(a.v_cache + grow);
+              gk[k] = ka;
+              gk[k + D / 4] = kb;
+              gv[k] = va;
+              gv[k + D / 4] = vb;
             }
           }
         }

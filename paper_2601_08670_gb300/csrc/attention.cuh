@@ -112,6 +112,7 @@ struct StepAttArgs {
   const int32_t* block_table; // [S][max_blocks] (paged layout) or null
   int32_t block_rows, max_blocks, num_blocks;
   int32_t block_shift;        // log2(block_rows) when it is a power of two, else -1
+  float rope_theta;           // rotary base (0: no rotary embedding)
   int32_t* seq_len;           // [S] +1 per launch for every sequence with room
   const int32_t* step;        // [1] step counter t (token y_{t-1} = history[b][t-1])
   const int32_t* history;     // [B][max_steps]

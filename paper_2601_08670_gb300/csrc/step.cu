@@ -8,6 +8,7 @@
 //   select     Eq. 2 + Eq. 3 per query, history[b][t] = y, t += 1
 // Every quantity that changes between steps (t, lengths, history) lives on
 // the device, so one captured call replays as the next step.
+#include <cmath>
 #include <math.h>
 #include <stdlib.h>
 
@@ -109,6 +110,8 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (d > 8192) return fail(PCED_ERR_UNSUPPORTED, "pced_step: hidden size %d > 8192", d);
   if (p->layer_elems % dm.D != 0 || (int64_t)dm.L * (p->layer_elems / dm.D) >= ((int64_t)1 << 31))
     return fail(PCED_ERR_UNSUPPORTED, "pced_step: cache too large for 32-bit row coordinates");
+  if (!(p->rope_theta >= 0.f) || !std::isfinite(p->rope_theta))
+    return fail(PCED_ERR_INVALID_ARG, "pced_step: rope_theta must be finite and >= 0");
   int64_t num_blocks = 0;
   if (paged) {
     if (p->block_rows < ATT_BLOCK_N || p->block_rows % ATT_BLOCK_N != 0 || p->max_blocks < 1)
@@ -185,6 +188,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   at.block_rows = paged ? p->block_rows : 0;
   at.max_blocks = paged ? p->max_blocks : 0;
   at.num_blocks = (int32_t)num_blocks;
+  at.rope_theta = p->rope_theta;
   at.block_shift = -1;
   if (paged && (p->block_rows & (p->block_rows - 1)) == 0)
     for (at.block_shift = 0; (1 << at.block_shift) < p->block_rows; ++at.block_shift) {
