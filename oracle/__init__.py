@@ -72,6 +72,8 @@ def lib():
         L.oracle_adacad_beta.restype = I32
         L.oracle_rope.argtypes = [P, I32, I64, F64, P]
         L.oracle_rope.restype = None
+        L.oracle_relevance.argtypes = [P, I32, P, I32, F64, P]
+        L.oracle_relevance.restype = I32
         _lib = L
     return _lib
 
@@ -163,6 +165,20 @@ def rope(x, pos: int, theta: float) -> np.ndarray:
     y = np.empty_like(x)
     lib().oracle_rope(_p(x), x.size, int(pos), float(theta), _p(y))
     return y
+
+
+def relevance(s, mode: int, z=None, eps: float = 1e-8) -> np.ndarray:
+    """Relevance scores from raw retrieval scores s (mode 0 dense/ColBERT,
+    1 sparse) and, if given, reranker logits z, fused by the harmonic mean
+    (see oracle_relevance)."""
+    s = _c(np.atleast_1d(s), np.float64)
+    zz = None if z is None else _c(np.atleast_1d(z), np.float64)
+    assert zz is None or zz.shape == s.shape
+    r = np.empty_like(s)
+    rc = lib().oracle_relevance(_p(s), int(mode), _p(zz), s.size, float(eps), _p(r))
+    if rc != 0:
+        raise ValueError(f"oracle_relevance rc={rc}")
+    return r
 
 
 def adacad_beta(lp, B, N):

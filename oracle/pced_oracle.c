@@ -266,6 +266,28 @@ int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, in
                                score, token_gap, expert_gap, h_out, lse_out, NULL, nthreads);
 }
 
+static double clip_unit(double x, double eps) {
+  if (x < 0.0) return 0.0;
+  if (x > 1.0 - eps) return 1.0 - eps;
+  return x;
+}
+
+int32_t oracle_relevance(const double* s, int32_t mode, const double* z, int32_t n, double eps, double* r) {
+  if (!s || !r || n < 0 || eps < 0.0 || (mode != 0 && mode != 1)) return -1;
+  const double pi = 3.14159265358979323846;
+  for (int32_t k = 0; k < n; ++k) {
+    const double rr = mode == 0 ? clip_unit((s[k] + 1.0) / 2.0, eps)
+                                : clip_unit(2.0 / pi * atan(s[k] > 0.0 ? s[k] : 0.0), eps);
+    if (!z) {
+      r[k] = rr;
+      continue;
+    }
+    const double rz = clip_unit(1.0 / (1.0 + exp(-z[k])), eps);
+    r[k] = 2.0 * rr * rz / (rr + rz + eps);
+  }
+  return 0;
+}
+
 void oracle_rope(const double* x, int32_t D, int64_t pos, double theta, double* y) {
   const int32_t half = D / 2;
   for (int32_t f = 0; f < half; ++f) {

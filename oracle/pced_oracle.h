@@ -71,6 +71,18 @@ int32_t oracle_adacad_beta(const double* lp, int32_t B, int32_t N, int32_t V, do
  * cos and sin evaluated in double.  D even, pos >= 0, theta > 0. */
 void oracle_rope(const double* x, int32_t D, int64_t pos, double theta, double* y);
 
+/* Relevance scores r_k in [0, 1) from a retriever's and a reranker's raw
+ * scores (Sec. 3 "Retrieval and relevance scoring", App. "Normalization of
+ * Retrieval and Reranker Scores"):
+ *   retrieval, mode 0 (dense / ColBERT): r_ret = clip((s + 1)/2, 0, 1 - eps)
+ *   retrieval, mode 1 (sparse):          r_ret = clip((2/pi) atan(max(s, 0)), 0, 1 - eps)
+ *   reranker logit z:                    r_rer = clip(1/(1 + exp(-z)), 0, 1 - eps)
+ *   fusion (harmonic mean, appendix form with eps in the denominator):
+ *                                        r = 2 r_ret r_rer / (r_ret + r_rer + eps)
+ * With z == NULL the result is r_ret alone.  n scores; returns 0, or -1 on bad
+ * arguments (mode not 0/1, n < 0, eps < 0). */
+int32_t oracle_relevance(const double* s, int32_t mode, const double* z, int32_t n, double eps, double* r);
+
 typedef struct oracle_dims {
   int32_t B, N, L, Hq, Hkv, D, V; /* S = B*(N+1), d = Hq*D, requires 2*Hkv <= Hq */
   double gamma;                   /* retrieval-prior weight of Eq. 2 */

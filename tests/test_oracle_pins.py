@@ -489,6 +489,55 @@ def test_step_with_rope_rotates_queries_and_keys_at_the_token_position_not_value
     assert np.array_equal(out["h"][0], h) and np.array_equal(out["h"][1], h)
 
 
+# ------------------------------------- relevance normalisation and fusion
+# App. "Normalization of Retrieval and Reranker Scores", eps = 1e-8.
+EPS = 1e-8
+
+
+def test_relevance_dense_endpoints_and_midpoint():
+    r = oracle.relevance([-1.0, 1.0, 0.0, -3.0, 2.0, 0.5], 0)
+    assert list(r) == [0.0, 1.0 - EPS, 0.5, 0.0, 1.0 - EPS, 0.75]
+
+
+def test_relevance_sparse_saturating_arctan():
+    r = oracle.relevance([0.0, -5.0, 1.0, math.tan(math.pi / 8), 1e30], 1)
+    assert r[0] == 0.0 and r[1] == 0.0           # max(s, 0) then atan(0) = 0
+    assert abs(r[2] - 0.5) < 1e-15                # (2/pi) atan(1) = 1/2
+    assert abs(r[3] - 0.25) < 1e-15               # (2/pi)(pi/8)
+    assert r[4] == 1.0 - EPS                      # saturates below 1
+    xs = np.linspace(0, 50, 101)
+    assert np.all(np.diff(oracle.relevance(xs, 1)) > 0)  # monotone
+
+
+def test_relevance_reranker_sigmoid_and_harmonic_mean():
+    # dense s = 0 gives r_ret = 1/2; reranker z = 0 gives 1/2; HM(1/2, 1/2) = 1/(1 + eps)
+    r = oracle.relevance([0.0], 0, z=[0.0])
+    assert abs(r[0] - 0.5 / (1.0 + EPS)) < 1e-16
+    # z = ln 3: sigmoid = 3/4; with r_ret = 1/2: HM = 2 (3/8) / (5/4 + eps)
+    r = oracle.relevance([0.0], 0, z=[math.log(3.0)])
+    assert abs(r[0] - 0.75 / (1.25 + EPS)) < 1e-15
+    # a zero on either side gives zero; the fusion is symmetric
+    assert oracle.relevance([-1.0], 0, z=[0.3])[0] == 0.0
+    a = oracle.relevance([0.2], 0, z=[-0.7])[0]
+    b = oracle.relevance([2 * (1 / (1 + math.exp(0.7))) - 1], 0, z=[math.log(0.6 / 0.4)])[0]
+    assert abs(a - b) < 1e-15
+    # between the smaller input and the geometric mean, in [0, 1)
+    s = rng0.uniform(-1, 1, 50)
+    z = rng0.normal(size=50) * 3
+    r = oracle.relevance(s, 0, z=z)
+    rr = (s + 1) / 2
+    rz = 1 / (1 + np.exp(-z))
+    assert np.all(r <= np.sqrt(rr * rz) + 1e-15) and np.all(r >= np.minimum(rr, rz) * (1 - 1e-7) - 1e-15)
+    assert np.all((r >= 0) & (r < 1))
+
+
+def test_relevance_without_reranker_is_the_retrieval_score():
+    s = rng0.uniform(-1, 1, 20)
+    assert np.array_equal(oracle.relevance(s, 0), np.clip((s + 1) / 2, 0, 1 - EPS))
+    with pytest.raises(ValueError):
+        oracle.relevance(s, 2)
+
+
 # --------------------------------------------------------------- paper figures
 def test_kv_storage_example_from_paper():
     import json, os
