@@ -176,6 +176,28 @@ pced_status pced_adacad_beta(const float* logprobs, int32_t B, int32_t N, int32_
                              size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * pced_relevance -- relevance scores r in [0, 1) for the retrieval prior of
+ * Eq. 2 (Sec. 3 "Retrieval and relevance scoring": map retriever and
+ * reranker scores to [0, 1) and fuse them by the harmonic mean; App.
+ * "Normalization of Retrieval and Reranker Scores" gives the maps):
+ *   ret_mode PCED_RET_DENSE (dense / ColBERT similarity in [-1, 1]):
+ *       r_ret = clip((s + 1)/2, 0, 1 - eps)
+ *   ret_mode PCED_RET_SPARSE (sparse lexical score, >= 0, unbounded):
+ *       r_ret = clip((2/pi) atan(max(s, 0)), 0, 1 - eps)
+ *   reranker logit z:  r_rer = clip(1/(1 + exp(-z)), 0, 1 - eps)
+ *   r = 2 r_ret r_rer / (r_ret + r_rer + eps)   (the appendix's form, eps in the denominator)
+ *   ret_scores fp32 [n] (device), rer_logits fp32 [n] (device) or NULL
+ *   (then r = r_ret), r fp32 [n] output (device).  The paper uses eps = 1e-8.
+ * Evaluated in fp64, rounded to fp32 once.  n = 0 does nothing.  Errors:
+ * PCED_ERR_INVALID_ARG for n < 0, another mode, eps outside [0, 0.5), a
+ * null or misaligned pointer.
+ * ------------------------------------------------------------------------ */
+#define PCED_RET_DENSE 0
+#define PCED_RET_SPARSE 1
+pced_status pced_relevance(const float* ret_scores, int32_t ret_mode, const float* rer_logits, int32_t n, double eps,
+                           float* r, void* stream);
+
+/* ------------------------------------------------------------------------
  * pced_step -- one full greedy decode step of all B queries (Sec. 3,
  * Eq. 2, Eq. 3 and the shared-history append) on the weight-free layer
  * chain used for synthetic workloads:

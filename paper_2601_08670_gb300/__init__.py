@@ -83,6 +83,8 @@ def lib(path: str = LIB_PATH):
         L.pced_adacad_beta_workspace_size.restype = SZ
         L.pced_adacad_beta.argtypes = [P, I32, I32, I32, P, P, SZ, P]
         L.pced_adacad_beta.restype = I32
+        L.pced_relevance.argtypes = [P, I32, P, I32, ctypes.c_double, P, P]
+        L.pced_relevance.restype = I32
         L.pced_step_workspace_size.argtypes = [ctypes.POINTER(Dims)]
         L.pced_step_workspace_size.restype = SZ
         L.pced_step.argtypes = [ctypes.POINTER(StepArgs), P]
@@ -214,6 +216,23 @@ def adacad_beta(logprobs, B: int, N: int, ws=None, stream=None):
     _check(lib().pced_adacad_beta(_ptr(logprobs), B, N, V, _ptr(beta), _ptr(ws), ws.numel(), _stream(stream)),
            "pced_adacad_beta")
     return beta
+
+
+RET_DENSE, RET_SPARSE = 0, 1
+
+
+def relevance(ret_scores, ret_mode: int = RET_DENSE, rer_logits=None, eps: float = 1e-8, stream=None):
+    """pced_relevance: relevance scores in [0, 1) from raw retrieval scores
+    (dense/ColBERT or sparse) and optional reranker logits, fused by the
+    harmonic mean (fp32 tensors of one shape on the device)."""
+    assert ret_scores.dtype == torch.float32 and ret_scores.is_contiguous()
+    if rer_logits is not None:
+        assert rer_logits.dtype == torch.float32 and rer_logits.is_contiguous()
+        assert rer_logits.shape == ret_scores.shape
+    r = torch.empty_like(ret_scores)
+    _check(lib().pced_relevance(_ptr(ret_scores), int(ret_mode), _ptr(rer_logits), ret_scores.numel(), float(eps),
+                                _ptr(r), _stream(stream)), "pced_relevance")
+    return r
 
 
 def dims(B, N, L, Hq, Hkv, D, V) -> Dims:

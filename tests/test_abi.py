@@ -83,6 +83,26 @@ def test_adacad_beta_rejects_bad_arguments(L):
     assert L.pced_adacad_beta_workspace_size(1, 2, 100) > 0
 
 
+def test_relevance_rejects_bad_arguments(L):
+    f = L.pced_relevance
+    assert f(FAKE, 0, None, -1, 1e-8, FAKE, None) == 1      # n < 0
+    assert f(FAKE, 2, None, 4, 1e-8, FAKE, None) == 1       # no such retrieval mode
+    assert f(FAKE, 0, None, 4, -1.0, FAKE, None) == 1       # eps < 0
+    assert f(FAKE, 0, None, 4, float("nan"), FAKE, None) == 1
+    assert f(None, 0, None, 4, 1e-8, FAKE, None) == 1       # null scores
+    assert f(FAKE, 1, FAKE + 2, 4, 1e-8, FAKE, None) == 1   # misaligned reranker logits
+    assert f(None, 0, None, 0, 1e-8, None, None) == 0       # nothing to do
+
+
+def test_step_rejects_bad_rope_and_block_arguments(L):
+    import paper_2601_08670_gb300 as pced
+    f = lambda a: L.pced_step(ctypes.byref(a), None)
+    assert f(step_args(pced, rope_theta=-1.0)) == 1
+    assert f(step_args(pced, rope_theta=float("inf"))) == 1
+    assert f(step_args(pced, block_table=FAKE, block_rows=96, max_blocks=4)) == 1   # not a multiple of 64
+    assert f(step_args(pced, block_table=FAKE, block_rows=64, max_blocks=0)) == 1
+
+
 def test_step_dynamic_beta_needs_its_output(L):
     import paper_2601_08670_gb300 as pced
     a = step_args(pced, beta_from_step=1)
