@@ -40,7 +40,7 @@ class _Dims(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int32), ("N", ctypes.c_int32), ("L", ctypes.c_int32), ("Hq", ctypes.c_int32),
                 ("Hkv", ctypes.c_int32), ("D", ctypes.c_int32), ("V", ctypes.c_int32),
                 ("gamma", ctypes.c_double), ("rms_eps", ctypes.c_double), ("attn_scale", ctypes.c_double),
-                ("rope_theta", ctypes.c_double)]
+                ("rope_theta", ctypes.c_double), ("score_mode", ctypes.c_int32), ("aggregation", ctypes.c_int32)]
 
 
 _lib = None
@@ -74,6 +74,8 @@ def lib():
         L.oracle_rope.restype = None
         L.oracle_relevance.argtypes = [P, I32, P, I32, F64, P]
         L.oracle_relevance.restype = I32
+        L.oracle_aggregate_select.argtypes = [P, P, P, I32, I32, I32, I32, P, P, P, P]
+        L.oracle_aggregate_select.restype = I32
         _lib = L
     return _lib
 
@@ -181,6 +183,28 @@ def relevance(s, mode: int, z=None, eps: float = 1e-8) -> np.ndarray:
     return r
 
 
+MOE, POE = 1, 2
+
+
+def aggregate_select(lp, beta, r, rule: int):
+    """MoE (rule 1) / PoE (rule 2) aggregation of the contrastive expert
+    distributions (see oracle_aggregate_select).  lp: [B*(N+1), V]; beta, r:
+    [B, N].  Returns dict(token, expert, score, token_gap)."""
+    lp = _c(lp, np.float64)
+    beta = _c(beta, np.float32)
+    r = _c(r, np.float32)
+    B, N = beta.shape
+    V = lp.shape[1]
+    tok = np.empty(B, np.int32)
+    ex = np.empty(B, np.int32)
+    sc = np.empty(B, np.float64)
+    gap = np.empty(B, np.float64)
+    rc = lib().oracle_aggregate_select(_p(lp), _p(beta), _p(r), B, N, V, int(rule), _p(tok), _p(ex), _p(sc), _p(gap))
+    if rc != 0:
+        raise ValueError(f"oracle_aggregate_select rc={rc}")
+    return dict(token=tok, expert=ex, score=sc, token_gap=gap)
+
+
 def adacad_beta(lp, B, N):
     """Dynamic contrast strength (Sec. 3 after Eq. 2, as in AdaCAD): per
     expert, the Jensen-Shannon divergence in bits between its distribution
@@ -201,7 +225,8 @@ def decode_step(dims: dict, kc, vc, layer_elems, kv_off, cap, lens, emb_rows, w_
     (adacad_beta, rounded to fp32; returned as "beta")."""
     dm = _Dims(dims["B"], dims["N"], dims["L"], dims["Hq"], dims["Hkv"], dims["D"], dims["V"],
                float(dims["gamma"]), float(dims.get("rms_eps", RMS_EPS)),
-               float(dims.get("attn_scale", 1.0 / math.sqrt(dims["D"]))), float(dims.get("rope_theta", 0.0)))
+               float(dims.get("attn_scale", 1.0 / math.sqrt(dims["D"]))), float(dims.get("rope_theta", 0.0)),
+               int(dims.get("score_mode", 0)), int(dims.get("aggregation", 0)))
     B, N = dims["B"], dims["N"]
     S, d = B * (N + 1), dims["Hq"] * dims["D"]
     for a, t in ((kc, np.uint16), (vc, np.uint16), (lens, np.int32)):

@@ -234,6 +234,67 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
 
 /* ------------------------------------- dynamic contrast strength (AdaCAD) */
 
+int32_t oracle_aggregate_select(const double* lp, const float* beta, const float* r, int32_t B, int32_t N, int32_t V,
+                                int32_t rule, int32_t* token, int32_t* expert, double* score, double* token_gap) {
+  if (!lp || !beta || !r || !token || !expert || !score || B < 1 || N < 1 || V < 1 || (rule != 1 && rule != 2))
+    return -1;
+  double* c = (double*)malloc(sizeof(double) * (size_t)N * V); /* c_k(v) - LSE_k = log p_k(v) */
+  double* agg = (double*)malloc(sizeof(double) * (size_t)V);
+  double* w = (double*)malloc(sizeof(double) * (size_t)N);
+  if (!c || !agg || !w) {
+    free(c); free(agg); free(w);
+    return -1;
+  }
+  for (int32_t b = 0; b < B; ++b) {
+    const double* lp0 = lp + (int64_t)b * (N + 1) * V;
+    double wsum = 0.0;
+    for (int32_t k = 0; k < N; ++k) {
+      w[k] = clip_relevance(r[(int64_t)b * N + k]);
+      wsum += w[k];
+    }
+    for (int32_t k = 0; k < N; ++k) w[k] /= wsum;
+    for (int32_t k = 0; k < N; ++k) {
+      const double bt = (double)beta[(int64_t)b * N + k];
+      const double* lpk = lp + ((int64_t)b * (N + 1) + k + 1) * V;
+      double* ck = c + (int64_t)k * V;
+      double m = -INFINITY;
+      for (int32_t v = 0; v < V; ++v) {
+        ck[v] = (1.0 + bt) * lpk[v] - bt * lp0[v];
+        if (ck[v] > m) m = ck[v];
+      }
+      double se = 0.0;
+      for (int32_t v = 0; v < V; ++v) se += exp(ck[v] - m);
+      const double lse = m + log(se);
+      for (int32_t v = 0; v < V; ++v) ck[v] -= lse;
+    }
+    for (int32_t v = 0; v < V; ++v) {
+      double a = 0.0;
+      if (rule == 1) {
+        for (int32_t k = 0; k < N; ++k) a += w[k] * exp(c[(int64_t)k * V + v]);
+        a = log(a);
+      } else {
+        for (int32_t k = 0; k < N; ++k) a += w[k] * c[(int64_t)k * V + v];
+      }
+      agg[v] = a;
+    }
+    int32_t bv = 0;
+    for (int32_t v = 1; v < V; ++v)
+      if (agg[v] > agg[bv]) bv = v;
+    double runner = -INFINITY;
+    for (int32_t v = 0; v < V; ++v)
+      if (v != bv && agg[v] > runner) runner = agg[v];
+    int32_t bk = 0;
+    for (int32_t k = 1; k < N; ++k)
+      if (w[k] * exp(c[(int64_t)k * V + bv]) > w[bk] * exp(c[(int64_t)bk * V + bv])) bk = k;
+    token[b] = bv;
+    expert[b] = bk + 1;
+    score[b] = agg[bv];
+    if (token_gap) token_gap[b] = agg[bv] - runner;
+  }
+  free(c); free(agg); free(w);
+  return 0;
+}
+
 int32_t oracle_adacad_beta(const double* lp, int32_t B, int32_t N, int32_t V, double* beta) {
   if (!lp || !beta || B < 1 || N < 1 || V < 1) return -1;
   for (int32_t b = 0; b < B; ++b) {
@@ -311,6 +372,7 @@ int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc,
   const int32_t B = dm->B, N = dm->N, L = dm->L, Hq = dm->Hq, Hkv = dm->Hkv, D = dm->D, V = dm->V;
   if (B < 1 || N < 1 || L < 1 || Hkv < 1 || Hq % Hkv != 0 || 2 * Hkv > Hq || D < 1 || V < 1) return -1;
   if (dm->rope_theta < 0.0 || (dm->rope_theta > 0.0 && D % 2 != 0)) return -1;
+  if (dm->score_mode < 0 || dm->score_mode > 1 || dm->aggregation < 0 || dm->aggregation > 2) return -1;
   const int32_t S = B * (N + 1), d = Hq * D;
   for (int32_t s = 0; s < S; ++s)
     if (len[s] < 0 || len[s] >= cap[s]) return -2;
@@ -380,8 +442,16 @@ int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc,
       beta = beta_dyn;
     }
   }
-  if (rc == 0)
+  if (rc == 0 && dm->aggregation != 0) {
+    rc = oracle_aggregate_select(lp, beta, r, B, N, V, dm->aggregation, token, expert, score, token_gap);
+    if (expert_gap)
+      for (int32_t b = 0; b < B; ++b) expert_gap[b] = INFINITY;
+  } else if (rc == 0) {
+    if (dm->score_mode == 1) /* raw logits: z = lp + lse */
+      for (int32_t s = 0; s < S; ++s)
+        for (int32_t v = 0; v < V; ++v) lp[(int64_t)s * V + v] += lse[s];
     oracle_contrastive_select(lp, beta, r, dm->gamma, B, N, V, token, expert, score, token_gap, expert_gap);
+  }
 
   free(x); free(xn); free(xq); free(u); free(o); free(lp); free(lse);
   return rc;

@@ -53,6 +53,22 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
                                   int32_t N, int32_t V, int32_t* token, int32_t* expert, double* score,
                                   double* token_gap, double* expert_gap);
 
+/* Aggregation variants of the experts (App. "Ablation of Expert Aggregation
+ * Rule": Mixture-of-Experts, a weighted sum, and Product-of-Experts, a
+ * weighted product, in probability space, weights derived from retrieval
+ * scores).  Reading (the paper gives no formula): per contextual expert the
+ * contrastive scores c_k(v) = (1 + beta_k) lp_k(v) - beta_k lp_0(v) of Eq. 2
+ * without the prior, p_k = softmax_v(c_k), weights w_k = r~_k / sum_j r~_j
+ * with r~ clipped as in Eq. 2;
+ *   rule 1 (MoE): agg(v) = log sum_k w_k p_k(v)
+ *   rule 2 (PoE): agg(v) = sum_k w_k log p_k(v)
+ * token = argmax_v agg (lowest id on exact ties), score = agg(token),
+ * expert = argmax_k w_k p_k(token) (1-based, lowest k on ties),
+ * token_gap = agg(token) - max_{v != token} agg(v) (+inf when V = 1).
+ * lp [S][V] as in oracle_contrastive_select; gamma does not enter. */
+int32_t oracle_aggregate_select(const double* lp, const float* beta, const float* r, int32_t B, int32_t N, int32_t V,
+                                int32_t rule, int32_t* token, int32_t* expert, double* score, double* token_gap);
+
 /* Dynamic contrast strength (Sec. 3 after Eq. 2: beta_0 is computed as in
  * AdaCAD for the first generated token and kept fixed thereafter).  Reading
  * used here: one beta per contextual expert, the Jensen-Shannon divergence in
@@ -89,6 +105,8 @@ typedef struct oracle_dims {
   double rms_eps;                 /* RMSNorm epsilon */
   double attn_scale;              /* softmax scale, 1/sqrt(D) */
   double rope_theta;              /* rotary base; 0: no rotary embedding */
+  int32_t score_mode;             /* s_k of Eq. 2: 0 log-probabilities, 1 raw logits */
+  int32_t aggregation;            /* 0 max over experts (Eq. 3), 1 MoE, 2 PoE (oracle_aggregate_select) */
 } oracle_dims;
 
 /* One full decode step of the synthetic PCED model.
@@ -104,7 +122,11 @@ typedef struct oracle_dims {
  *   then the unembedding/log-softmax and Eq. 2 + Eq. 3 selection.
  * kc/vc span L layers of layer_elems elements (slab layout as in
  * oracle_attention); len[S] is updated in place; h_out (bf16 [S][d]) and
- * lse_out ([S]) may be NULL.  Returns 0, -1 on bad arguments, -2 when a
+ * lse_out ([S]) may be NULL.  score_mode 1 feeds the raw logits z = lp + lse
+ * to Eq. 2 instead of the log-probabilities (max rule; MoE / PoE do not
+ * depend on it: a per-expert constant drops out of the softmax); with
+ * aggregation 1 or 2 the token comes from oracle_aggregate_select and
+ * expert_gap is +inf.  Returns 0, -1 on bad arguments, -2 when a
  * cache is full. */
 int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, int64_t layer_elems,
                            const int64_t* kv_off, const int32_t* cap, int32_t* len, const uint16_t* emb_rows,

@@ -538,6 +538,104 @@ def test_relevance_without_reranker_is_the_retrieval_score():
         oracle.relevance(s, 2)
 
 
+# ------------------------------------------- aggregation variants (MoE / PoE)
+# App. "Ablation of Expert Aggregation Rule".  Reading: p_k = softmax of the
+# contrastive scores of Eq. 2 without the prior, weights r_k / sum r, MoE =
+# weighted sum of the p_k, PoE = weighted product (sum of weighted logs).
+def _lp(*rows):
+    return np.log(np.array(rows, np.float64))
+
+
+def test_aggregate_hand_worked_example_separates_max_moe_and_poe():
+    u = [1 / 3] * 3
+    lp = _lp(u, [0.7, 0.2, 0.1], [0.05, 0.35, 0.6])
+    beta = np.zeros((1, 2), np.float32)
+    r = np.full((1, 2), 0.5, np.float32)
+    moe = oracle.aggregate_select(lp, beta, r, oracle.MOE)
+    poe = oracle.aggregate_select(lp, beta, r, oracle.POE)
+    # MoE: (0.375, 0.275, 0.35) -> token 0, carried by expert 1
+    assert moe["token"][0] == 0 and moe["expert"][0] == 1
+    assert abs(moe["score"][0] - math.log(0.375)) < 1e-12
+    assert abs(moe["token_gap"][0] - math.log(0.375 / 0.35)) < 1e-12
+    # PoE: sqrt of (0.035, 0.07, 0.06) -> token 1, where expert 2 puts more mass
+    assert poe["token"][0] == 1 and poe["expert"][0] == 2
+    assert abs(poe["score"][0] - 0.5 * math.log(0.07)) < 1e-12
+    # Max (Eq. 3 with gamma = 0, beta = 0): the single most confident expert wins, token 0
+    mx = oracle.contrastive_select(lp, beta, r, 0.0, 1, 2)
+    assert mx["token"][0] == 0 and mx["expert"][0] == 1
+
+
+def test_aggregate_weights_are_normalised_retrieval_scores():
+    lp = _lp([0.25] * 4, [0.1, 0.6, 0.2, 0.1], [0.5, 0.1, 0.1, 0.3])
+    beta = np.zeros((1, 2), np.float32)
+    for scale in (1.0, 0.1):
+        r = (np.array([[0.9, 0.1]]) * scale).astype(np.float32)
+        moe = oracle.aggregate_select(lp, beta, r, oracle.MOE)
+        w = r[0].astype(np.float64) / r[0].astype(np.float64).sum()
+        mix = w[0] * np.array([0.1, 0.6, 0.2, 0.1]) + w[1] * np.array([0.5, 0.1, 0.1, 0.3])
+        assert moe["token"][0] == 1 and abs(moe["score"][0] - math.log(mix[1])) < 1e-12
+    # flipping the weights flips the winner
+    r = np.array([[0.1, 0.9]], np.float32)
+    assert oracle.aggregate_select(lp, beta, r, oracle.MOE)["token"][0] == 0
+
+
+def test_aggregate_contrast_sharpens_against_a_flat_amateur():
+    # uniform amateur: c_k = (1 + beta) log p_k + const, so p_k becomes p_k^(1+beta) renormalised
+    p1 = np.array([0.7, 0.2, 0.1])
+    lp = _lp([1 / 3] * 3, p1, [0.2, 0.5, 0.3])
+    beta = np.ones((1, 2), np.float32)
+    r = np.array([[1.0, 1e-30]], np.float32)  # clipped to 1e-8: expert 2 weighs ~1e-8
+    moe = oracle.aggregate_select(lp, beta, r, oracle.MOE)
+    sq = p1 ** 2 / (p1 ** 2).sum()
+    assert moe["token"][0] == 0 and abs(moe["score"][0] - math.log(sq[0])) < 1e-6
+
+
+def test_aggregate_single_expert_is_contrastive_greedy_and_permutation_invariant():
+    rng = np.random.default_rng(3)
+    V = 50
+    z = rng.normal(size=(2, V)) * 3
+    lp = z - np.log(np.exp(z).sum(1, keepdims=True))
+    beta = np.full((1, 1), 0.5, np.float32)
+    r = np.full((1, 1), 0.3, np.float32)
+    tok = oracle.contrastive_select(lp, beta, r, 0.0, 1, 1)["token"]
+    for rule in (oracle.MOE, oracle.POE):
+        out = oracle.aggregate_select(lp, beta, r, rule)
+        assert out["token"][0] == tok[0] and out["expert"][0] == 1
+    z = rng.normal(size=(4, V)) * 2
+    lp = z - np.log(np.exp(z).sum(1, keepdims=True))
+    beta = np.array([[0.2, 0.7, 0.4]], np.float32)
+    r = np.array([[0.5, 0.2, 0.9]], np.float32)
+    perm = [2, 0, 1]
+    for rule in (oracle.MOE, oracle.POE):
+        a = oracle.aggregate_select(lp, beta, r, rule)
+        b = oracle.aggregate_select(lp[[0] + [1 + p for p in perm]], beta[:, perm], r[:, perm], rule)
+        assert a["token"][0] == b["token"][0] and abs(a["score"][0] - b["score"][0]) < 1e-12
+        assert perm[b["expert"][0] - 1] + 1 == a["expert"][0]
+
+
+def test_step_raw_logit_mode_and_moe_in_closed_form():
+    # one expert over an empty prefix: expert and amateur see the same single
+    # token, so lp_1 = lp_0 and (1 + beta) s_1 - beta s_0 = s_1.  Log-prob mode
+    # scores z* - lse + gamma log r; raw-logit mode z* + gamma log r; MoE picks
+    # the same token with score log p(token) and no prior.
+    outs = {}
+    case = empty_prefix_case(1)
+    for key, extra in (("lp", {}), ("raw", dict(score_mode=1)), ("moe", dict(aggregation=1)),
+                       ("poe", dict(aggregation=2))):
+        dims, kc, vc, lay, off, cap, lens, emb, w = [x.copy() if hasattr(x, "copy") else x for x in case]
+        dims.update(extra)
+        beta = np.full((1, 1), 0.5, np.float32)
+        r = np.full((1, 1), 0.8, np.float32)
+        outs[key] = oracle.decode_step(dims, kc, vc, lay, off, cap, lens, emb, w, beta, r)
+    lse = outs["lp"]["lse"][1]
+    assert all(outs[k]["token"][0] == outs["lp"]["token"][0] for k in outs)
+    assert abs(outs["raw"]["score"][0] - outs["lp"]["score"][0] - lse) < 1e-9
+    prior = 2.5 * math.log(float(np.float32(0.8)))
+    for k in ("moe", "poe"):
+        assert abs(outs[k]["score"][0] - (outs["lp"]["score"][0] - prior)) < 1e-9
+        assert outs[k]["expert"][0] == 1
+
+
 # --------------------------------------------------------------- paper figures
 def test_kv_storage_example_from_paper():
     import json, os
