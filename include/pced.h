@@ -278,7 +278,27 @@ typedef struct pced_step_args {
    * value row is not rotated and the cached rows are taken as stored (already
    * rotated).  0: no rotation.  Negative or non-finite: PCED_ERR_INVALID_ARG. */
   float rope_theta;
+  /* s_k of Eq. 2 (Sec. 3 "per-expert logits"): PCED_SCORE_LOGPROB (0, the
+   * default reading: log-softmax) or PCED_SCORE_LOGIT (1: raw logits, so the
+   * per-expert constant is gamma log r alone).  Used by the max rule. */
+  int32_t score_mode;
+  /* How experts are combined (appendix "Ablation of Expert Aggregation
+   * Rule"): PCED_AGG_MAX (0, Eq. 3), PCED_AGG_MOE (1) or PCED_AGG_POE (2).
+   * MoE / PoE read: p_k = softmax_v((1 + beta_k) lp_k - beta_k lp_0), weights
+   * w_k = r_k / sum_j r_j (r clipped to [1e-8, 1]); MoE picks
+   * argmax_v log sum_k w_k p_k(v), PoE argmax_v sum_k w_k log p_k(v); the
+   * expert reported is argmax_k w_k p_k(token), the score the aggregate;
+   * gamma and score_mode do not enter (a per-expert constant drops out of the
+   * softmax).  These rules materialise the log-probabilities (S x V fp32 in
+   * the workspace) and take five launches; stage events are not recorded. */
+  int32_t aggregation;
 } pced_step_args;
+
+#define PCED_SCORE_LOGPROB 0
+#define PCED_SCORE_LOGIT 1
+#define PCED_AGG_MAX 0
+#define PCED_AGG_MOE 1
+#define PCED_AGG_POE 2
 
 size_t pced_step_workspace_size(const pced_dims* dims);
 pced_status pced_step(const pced_step_args* args, void* stream);

@@ -47,7 +47,7 @@ class StepArgs(ctypes.Structure):
                 ("workspace_bytes", ctypes.c_size_t), ("stage_events", ctypes.c_void_p),
                 ("n_stage_events", ctypes.c_int32), ("beta_from_step", ctypes.c_int32), ("beta_out", ctypes.c_void_p),
                 ("block_table", ctypes.c_void_p), ("block_rows", ctypes.c_int32), ("max_blocks", ctypes.c_int32),
-                ("rope_theta", ctypes.c_float)]
+                ("rope_theta", ctypes.c_float), ("score_mode", ctypes.c_int32), ("aggregation", ctypes.c_int32)]
 
 
 _lib = None
@@ -219,6 +219,8 @@ def adacad_beta(logprobs, B: int, N: int, ws=None, stream=None):
 
 
 RET_DENSE, RET_SPARSE = 0, 1
+SCORE_LOGPROB, SCORE_LOGIT = 0, 1
+AGG_MAX, AGG_MOE, AGG_POE = 0, 1, 2
 
 
 def relevance(ret_scores, ret_mode: int = RET_DENSE, rer_logits=None, eps: float = 1e-8, stream=None):
@@ -261,7 +263,7 @@ class Decoder:
     def __init__(self, dm: Dims, *, embed, w_unembed, k_cache, v_cache, layer_elems: int, kv_offset, cap, seq_len,
                  beta, r, gamma: float, max_steps: int, total_cap: int, bos: int = 0, attn_scale=None,
                  rms_eps: float = 1e-6, keep_hidden: bool = False, dynamic_beta: bool = False, block_table=None,
-                 block_rows: int = 0, rope_theta: float = 0.0):
+                 block_rows: int = 0, rope_theta: float = 0.0, score_mode: int = 0, aggregation: int = 0):
         dev = k_cache.device
         self.dm = dm
         B, S, d = dm.B, dm.B * (dm.N + 1), dm.Hq * dm.D
@@ -283,6 +285,8 @@ class Decoder:
             _ptr(self.hidden), _ptr(self.lse), _ptr(self.ws), self.ws.numel())
         self.max_steps = max_steps
         self.args.rope_theta = float(rope_theta)  # rotary base, 0: none
+        self.args.score_mode = int(score_mode)     # SCORE_LOGPROB / SCORE_LOGIT
+        self.args.aggregation = int(aggregation)   # AGG_MAX / AGG_MOE / AGG_POE
         if block_table is not None:  # paged caches
             assert block_table.dtype == torch.int32 and block_table.is_contiguous() and block_table.dim() == 2
             self.args.block_table = _ptr(block_table)
@@ -325,7 +329,7 @@ class Decoder:
 
 def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos: int = 0, keep_hidden=False,
                         attn_scale=None, rms_eps: float = 1e-6, dynamic_beta: bool = False,
-                        rope_theta: float = 0.0) -> Decoder:
+                        rope_theta: float = 0.0, score_mode: int = 0, aggregation: int = 0) -> Decoder:
     """Decoder over a dict of device tensors with the keys k_cache, v_cache,
     kv_offset, cap, seq_len, embed, w_unembed, beta, r, and the host layout
     values layer_elems / total_cap (or a `layout` object carrying them)."""
@@ -336,4 +340,5 @@ def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos:
                    layer_elems=layer_elems, kv_offset=t["kv_offset"], cap=t["cap"], seq_len=t["seq_len"],
                    beta=t["beta"], r=t["r"], gamma=gamma, max_steps=max_steps, total_cap=total_cap, bos=bos,
                    attn_scale=attn_scale, rms_eps=rms_eps, keep_hidden=keep_hidden, dynamic_beta=dynamic_beta,
-                   block_table=t.get("block_table"), block_rows=int(t.get("block_rows", 0)), rope_theta=rope_theta)
+                   block_table=t.get("block_table"), block_rows=int(t.get("block_rows", 0)), rope_theta=rope_theta,
+                   score_mode=score_mode, aggregation=aggregation)

@@ -1,0 +1,37 @@
+// aggregate.cuh -- MoE / PoE aggregation of the experts from materialised
+// log-probabilities (the appendix's aggregation-rule ablation).
+#pragma once
+#include "common.cuh"
+
+namespace pced {
+
+struct AggArgs {
+  const float* lp;      // [S][V] log-probabilities, query-major, amateur first
+  const float* beta;    // [B][N]
+  const float* r;       // [B][N] relevance scores
+  const float* lse;     // [S] log-sum-exps of the rows (copied to lse_out)
+  int32_t B, N, V, rule, nchunks;  // rule 1 MoE, 2 PoE
+  float2* part;         // [B][N][nchunks] (max, sum exp) of c_k over each chunk
+  float2* best;         // [B][nchunks] (aggregate, token) of each chunk
+  int32_t* qdone;       // [B] chunks finished (zero at launch; the last resets it)
+  int* tile_ctr;        // optional: the LM head's tile counter, reset for its next launch
+  int32_t* token;       // optional [B]
+  int32_t* expert;      // optional [B]
+  float* score;         // optional [B]
+  float* lse_out;       // optional [S]
+  // step bookkeeping (optional), as in the max-rule selection
+  int32_t* step;
+  int32_t* history;
+  int32_t* expert_trace;
+  float* score_trace;
+  int32_t max_steps;
+  int32_t* done_counter;
+  int* status;
+};
+
+constexpr int AGG_CHUNK = 8192;  // vocabulary entries per CTA
+constexpr int AGG_MAX_N = 512;   // experts per query (the LM head's row limit)
+inline int32_t agg_chunks(int32_t V) { return (V + AGG_CHUNK - 1) / AGG_CHUNK; }
+cudaError_t aggregate_launch(const AggArgs& a, cudaStream_t stream);
+
+}  // namespace pced

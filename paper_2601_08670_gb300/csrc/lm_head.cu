@@ -594,7 +594,7 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
     const int sk = b * n1 + 1 + k;
     const float btk = a.beta[b * N + k];
     const float rr = fminf(fmaxf(a.r[b * N + k], 1e-8f), 1.0f);
-    const float c = -(1.f + btk) * __ldcg(a.sel_L + sk) + btk * L0 + a.gamma * logf(rr);
+    const float c = (a.raw_logits ? 0.f : -(1.f + btk) * __ldcg(a.sel_L + sk) + btk * L0) + a.gamma * logf(rr);
     const float sc = __ldcg(a.sel_u + sk) + c;
     const int tk = __ldcg(a.sel_tok + sk);
     if (sc > bs || (sc == bs && (tk < bt || (tk == bt && k < bk)))) {

@@ -67,6 +67,7 @@ struct SelectArgs {
   int32_t* sel_tok;   // [S] its token
   int32_t* qdone;     // [B] rows of the query finished
   int pdl;            // launched as a programmatic dependent of the LM head
+  int raw_logits;     // s_k of Eq. 2 are the raw logits: c_k = gamma log r_k alone
   int* status;
 };
 cudaError_t select_from_records_launch(const SelectArgs& a, cudaStream_t stream);

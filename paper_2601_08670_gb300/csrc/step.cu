@@ -13,6 +13,7 @@
 #include <stdlib.h>
 
 #include "adacad.cuh"
+#include "aggregate.cuh"
 #include "attention.cuh"
 #include "lm_head.cuh"
 
@@ -30,6 +31,9 @@ struct StepLayout {
   int32_t* sel_tok;
   float* lp;              // [S][V] log-probabilities of a dynamic-beta first step
   void* ada;              // scratch of the beta kernel (counters zero between uses)
+  float2* agg_part;       // MoE / PoE: per (query, expert, chunk) statistics
+  float2* agg_best;       // MoE / PoE: per (query, chunk) best
+  int32_t* agg_qdone;     // MoE / PoE: chunks finished per query
   uint64_t* part_ss;
   uint64_t* resid;
   uint64_t* rec_o;
@@ -66,6 +70,9 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   L.sel_tok = c.take<int32_t>((size_t)S);
   L.lp = c.take<float>((size_t)S * dm->V);
   L.ada = c.take<char>(adacad_scratch_bytes(dm->B, dm->N, dm->V));
+  L.agg_part = c.take<float2>((size_t)dm->B * dm->N * agg_chunks(dm->V));
+  L.agg_best = c.take<float2>((size_t)dm->B * agg_chunks(dm->V));
+  L.agg_qdone = c.take<int32_t>((size_t)dm->B);
   L.bytes = c.used() + 4 * (4096 - 256);  // room for the 4 KB alignment of four arrays
   return L;
 }
@@ -110,6 +117,12 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (d > 8192) return fail(PCED_ERR_UNSUPPORTED, "pced_step: hidden size %d > 8192", d);
   if (p->layer_elems % dm.D != 0 || (int64_t)dm.L * (p->layer_elems / dm.D) >= ((int64_t)1 << 31))
     return fail(PCED_ERR_UNSUPPORTED, "pced_step: cache too large for 32-bit row coordinates");
+  if (p->score_mode != PCED_SCORE_LOGPROB && p->score_mode != PCED_SCORE_LOGIT)
+    return fail(PCED_ERR_INVALID_ARG, "pced_step: score_mode %d", p->score_mode);
+  if (p->aggregation < PCED_AGG_MAX || p->aggregation > PCED_AGG_POE)
+    return fail(PCED_ERR_INVALID_ARG, "pced_step: aggregation %d", p->aggregation);
+  if (p->aggregation != PCED_AGG_MAX && dm.N > AGG_MAX_N)
+    return fail(PCED_ERR_UNSUPPORTED, "pced_step: MoE / PoE take at most %d experts", AGG_MAX_N);
   if (!(p->rope_theta >= 0.f) || !std::isfinite(p->rope_theta))
     return fail(PCED_ERR_INVALID_ARG, "pced_step: rope_theta must be finite and >= 0");
   int64_t num_blocks = 0;
@@ -142,7 +155,8 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (st != PCED_OK) return st;
   cudaStream_t s = (cudaStream_t)stream;
   const bool dyn = p->beta_from_step != 0;
-  const bool timed = !dyn && p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
+  const bool agg = p->aggregation != PCED_AGG_MAX;
+  const bool timed = !dyn && !agg && p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
   cudaStreamCaptureStatus cap_status = cudaStreamCaptureStatusNone;
   if (timed && cudaStreamIsCapturing(s, &cap_status) != cudaSuccess) return cuda_status(cudaGetLastError(), "capture query");
   int mark_i = 0;
@@ -212,10 +226,11 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "attention launch");
 
-  // dynamic contrast strength: materialise this step's log-probabilities,
-  // beta from their divergences, then the usual fused LM head with that beta
+  // dynamic contrast strength or MoE / PoE: materialise this step's
+  // log-probabilities; beta from their divergences, then either the usual
+  // fused LM head with that beta or the aggregation kernels
   const float* beta = p->beta;
-  if (dyn) {
+  if (dyn || agg) {
     LmArgs lz = {};
     lz.mode = 0;
     lz.S = S;
@@ -240,9 +255,36 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     e = lm_head_launch(wmap, hmap, g, lz, s);
     if (e == cudaSuccess) e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
     // the JSD kernel also re-arms the LM head's tile counter for the fused pass
-    if (e == cudaSuccess) e = adacad_beta_launch(W.lp, dm.B, dm.N, dm.V, p->beta_out, W.ada, W.lm_tile_ctr, s);
-    if (e != cudaSuccess) return cuda_status(e, "dynamic beta launches");
-    beta = p->beta_out;
+    if (e == cudaSuccess && dyn) e = adacad_beta_launch(W.lp, dm.B, dm.N, dm.V, p->beta_out, W.ada, W.lm_tile_ctr, s);
+    if (e != cudaSuccess) return cuda_status(e, "log-probability launches");
+    if (dyn) beta = p->beta_out;
+  }
+  if (agg) {
+    AggArgs ag = {};
+    ag.lp = W.lp;
+    ag.beta = beta;
+    ag.r = p->r;
+    ag.lse = W.sel_L;
+    ag.B = dm.B;
+    ag.N = dm.N;
+    ag.V = dm.V;
+    ag.rule = p->aggregation;
+    ag.nchunks = agg_chunks(dm.V);
+    ag.part = W.agg_part;
+    ag.best = W.agg_best;
+    ag.qdone = W.agg_qdone;
+    ag.tile_ctr = W.lm_tile_ctr;
+    ag.lse_out = p->lse_out;
+    ag.step = p->step;
+    ag.history = p->history;
+    ag.expert_trace = p->expert_trace;
+    ag.score_trace = p->score_trace;
+    ag.max_steps = p->max_steps;
+    ag.done_counter = W.done_counter;
+    ag.status = W.status;
+    e = aggregate_launch(ag, s);
+    if (e != cudaSuccess) return cuda_status(e, "aggregation launches");
+    return PCED_OK;
   }
 
   LmArgs la = {};
@@ -294,6 +336,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.done_counter = W.done_counter;
   sa.status = W.status;
   sa.pdl = (timed || dyn) ? 0 : 1;
+  sa.raw_logits = p->score_mode == PCED_SCORE_LOGIT;
   e = select_from_records_launch(sa, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "select launch");

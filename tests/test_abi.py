@@ -101,6 +101,9 @@ def test_step_rejects_bad_rope_and_block_arguments(L):
     assert f(step_args(pced, rope_theta=float("inf"))) == 1
     assert f(step_args(pced, block_table=FAKE, block_rows=96, max_blocks=4)) == 1   # not a multiple of 64
     assert f(step_args(pced, block_table=FAKE, block_rows=64, max_blocks=0)) == 1
+    assert f(step_args(pced, score_mode=2)) == 1
+    assert f(step_args(pced, aggregation=3)) == 1
+    assert f(step_args(pced, aggregation=-1)) == 1
 
 
 def test_step_dynamic_beta_needs_its_output(L):
