@@ -47,6 +47,9 @@ def parse_args():
                    help="store the caches paged with blocks of this many rows (a multiple of 64; 0: slabs)")
     p.add_argument("--rope-theta", type=float, default=0.0,
                    help="rotate queries and appended keys with this rotary base (0: none)")
+    p.add_argument("--aggregation", choices=["max", "moe", "poe"], default="max",
+                   help="how experts are combined: Eq. 3's max (default) or the MoE / PoE variants")
+    p.add_argument("--raw-logits", action="store_true", help="Eq. 2 on raw logits instead of log-probabilities")
     p.add_argument("--no-dynamic-beta", action="store_true",
                    help="skip timing the first step with dynamic contrast strength")
     p.add_argument("--profile-steps", type=int, default=4, help="replays with per-launch events (roofline)")
@@ -198,12 +201,16 @@ def step_bytes(w, lens_after) -> int:
 
 
 # --------------------------------------------------------------- our GPU path
-def build_decoder(w, dev, capacity_steps, paged=0, rope_theta=0.0):
+AGGREGATIONS = {"max": 0, "moe": 1, "poe": 2}
+
+
+def build_decoder(w, dev, capacity_steps, paged=0, rope_theta=0.0, aggregation="max", raw_logits=False):
     import paper_2601_08670_gb300 as pced
     import synth
     t = synth.device_inputs(w, dev, extra_steps=capacity_steps, paged=paged)
     dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
-    dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=capacity_steps, bos=w.bos, rope_theta=rope_theta)
+    dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=capacity_steps, bos=w.bos, rope_theta=rope_theta,
+                                   aggregation=AGGREGATIONS[aggregation], score_mode=1 if raw_logits else 0)
     return dec, t
 
 
@@ -344,7 +351,7 @@ def cpu_baseline(w, budget_s=20.0, max_steps=3):
             "ms_per_step": 1e3 * el / n}
 
 
-def workload_config(w, graph=True, paged=0, rope_theta=0.0):
+def workload_config(w, graph=True, paged=0, rope_theta=0.0, aggregation="max", raw_logits=False):
     import synth
     bl = synth.base_lengths(w)
     return {"workload": f"{w.name}: {w.description}", "B": w.B, "N": w.N, "S": w.S, "L": w.L, "Hq": w.Hq,
@@ -354,7 +361,10 @@ def workload_config(w, graph=True, paged=0, rope_theta=0.0):
                    if step_bytes(w, bl + 1) > 129e6 else "step working set fits in L2 (not a bandwidth workload)"),
             "cuda_graph": graph, "parallelism": "one independent replica per GPU",
             "kv_layout": f"paged, {paged}-row blocks in a shuffled pool" if paged else "one slab per (sequence, kv-head)",
-            "rotary": f"queries and appended keys rotated, base {rope_theta:g}" if rope_theta > 0 else "none"}
+            "rotary": f"queries and appended keys rotated, base {rope_theta:g}" if rope_theta > 0 else "none",
+            "aggregation": {"max": "max over experts (Eq. 3)", "moe": "mixture of experts (weighted sum)",
+                            "poe": "product of experts (weighted product)"}[aggregation],
+            "scores": "raw logits" if raw_logits else "log-probabilities"}
 
 
 def run_ours(args):
@@ -369,7 +379,8 @@ def run_ours(args):
     w = synth.get(args.workload)
     e2e_steps = 0 if args.no_e2e else min(args.steps, 16)
     cap_steps = args.warmup * 2 + 1 + args.steps + args.profile_steps + e2e_steps + 2
-    dec, _ = build_decoder(w, dev, cap_steps, paged=args.paged, rope_theta=args.rope_theta)
+    dec, _ = build_decoder(w, dev, cap_steps, paged=args.paged, rope_theta=args.rope_theta,
+                           aggregation=args.aggregation, raw_logits=args.raw_logits)
     launches = dec.launches_per_step()
 
     clocks = ClockSampler(local)
@@ -463,7 +474,8 @@ def run_ours(args):
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded counter-based generator)",
-            "config": workload_config(w, paged=args.paged, rope_theta=args.rope_theta),
+            "config": workload_config(w, paged=args.paged, rope_theta=args.rope_theta, aggregation=args.aggregation,
+                                      raw_logits=args.raw_logits),
             "step_hbm": {"achieved_gbs": step_gbs,
                                                        "frac_of_8tbps": step_gbs / NOMINAL_HBM_GBS,
                                                        "frac_of_measured": step_gbs / hbm_peak if hbm_peak else None,

@@ -290,7 +290,9 @@ typedef struct pced_step_args {
    * expert reported is argmax_k w_k p_k(token), the score the aggregate;
    * gamma and score_mode do not enter (a per-expert constant drops out of the
    * softmax).  These rules materialise the log-probabilities (S x V fp32 in
-   * the workspace) and take five launches; stage events are not recorded. */
+   * the workspace) and take five launches; the stage events then bracket the
+   * attention, the logits pass with its log-sum-exp finalise, and the two
+   * aggregation kernels. */
   int32_t aggregation;
 } pced_step_args;
 

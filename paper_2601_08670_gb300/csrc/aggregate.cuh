@@ -29,7 +29,7 @@ struct AggArgs {
   int* status;
 };
 
-constexpr int AGG_CHUNK = 8192;  // vocabulary entries per CTA
+constexpr int AGG_CHUNK = 1024;  // vocabulary entries per CTA (about 125 CTAs per query at V = 128K)
 constexpr int AGG_MAX_N = 512;   // experts per query (the LM head's row limit)
 inline int32_t agg_chunks(int32_t V) { return (V + AGG_CHUNK - 1) / AGG_CHUNK; }
 cudaError_t aggregate_launch(const AggArgs& a, cudaStream_t stream);

@@ -156,7 +156,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   cudaStream_t s = (cudaStream_t)stream;
   const bool dyn = p->beta_from_step != 0;
   const bool agg = p->aggregation != PCED_AGG_MAX;
-  const bool timed = !dyn && !agg && p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
+  const bool timed = !dyn && p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
   cudaStreamCaptureStatus cap_status = cudaStreamCaptureStatusNone;
   if (timed && cudaStreamIsCapturing(s, &cap_status) != cudaSuccess) return cuda_status(cudaGetLastError(), "capture query");
   int mark_i = 0;
@@ -256,6 +256,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     if (e == cudaSuccess) e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
     // the JSD kernel also re-arms the LM head's tile counter for the fused pass
     if (e == cudaSuccess && dyn) e = adacad_beta_launch(W.lp, dm.B, dm.N, dm.V, p->beta_out, W.ada, W.lm_tile_ctr, s);
+    if (e == cudaSuccess && agg) e = mark();  // MoE / PoE: the "lm_head" stage is the logits pass and its finalise
     if (e != cudaSuccess) return cuda_status(e, "log-probability launches");
     if (dyn) beta = p->beta_out;
   }
@@ -283,6 +284,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ag.done_counter = W.done_counter;
     ag.status = W.status;
     e = aggregate_launch(ag, s);
+    if (e == cudaSuccess) e = mark();  // the "select" stage: the two aggregation kernels
     if (e != cudaSuccess) return cuda_status(e, "aggregation launches");
     return PCED_OK;
   }
