@@ -65,7 +65,9 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
  * token = argmax_v agg (lowest id on exact ties), score = agg(token),
  * expert = argmax_k w_k p_k(token) (1-based, lowest k on ties),
  * token_gap = agg(token) - max_{v != token} agg(v) (+inf when V = 1).
- * lp [S][V] as in oracle_contrastive_select; gamma does not enter. */
+ * lp [S][V] as in oracle_contrastive_select; gamma does not enter.
+ * Parity unpinned against the paper (it names the rules, not the weighting);
+ * the tests pin this reading by closed forms. */
 int32_t oracle_aggregate_select(const double* lp, const float* beta, const float* r, int32_t B, int32_t N, int32_t V,
                                 int32_t rule, int32_t* token, int32_t* expert, double* score, double* token_gap);
 
@@ -75,7 +77,9 @@ int32_t oracle_aggregate_select(const double* lp, const float* beta, const float
  * bits between the expert's next-token distribution and the amateur's,
  *   beta[b][k-1] = 1/2 sum_v [ p_k(v) log2(p_k(v)/m(v)) + p_0(v) log2(p_0(v)/m(v)) ],
  *   m = (p_k + p_0)/2,  p = exp(lp),  terms with p = 0 contribute 0,
- * so 0 <= beta <= 1.  lp [S][V] as in oracle_contrastive_select. */
+ * so 0 <= beta <= 1.  lp [S][V] as in oracle_contrastive_select.
+ * Parity unpinned against the paper (it names AdaCAD, not the formula); the
+ * tests pin the divergence itself. */
 int32_t oracle_adacad_beta(const double* lp, int32_t B, int32_t N, int32_t V, double* beta);
 
 /* Rotary position embedding of one head (the decoder LLM's positional
