@@ -69,3 +69,22 @@ def test_oracle_queries_are_independent():
         b = one.step()
         assert a["token"][2] == b["token"][0] and a["expert"][2] == b["expert"][0]
         assert np.array_equal(a["h"][6:9], b["h"])
+
+
+def test_paged_layout_hands_out_every_block_once():
+    # a seeded shuffled pool: every sequence gets ceil(cap / P) distinct blocks,
+    # the blocks of all sequences are a permutation of the pool, -1 pads the table
+    for name, P in (("tiny", 64), ("llama8", 256), ("manydoc", 64), ("tiny", 192)):
+        w = synth.get(name)
+        bl = synth.base_lengths(w)
+        lay = synth.paged_layout(w, bl, P)
+        nblk = (lay.cap.astype(np.int64) + P - 1) // P
+        assert lay.num_blocks == int(nblk.sum())
+        assert lay.layer_elems == lay.num_blocks * w.Hkv * P * w.D
+        used = np.concatenate([lay.table[s, :n] for s, n in enumerate(nblk)])
+        assert np.array_equal(np.sort(used), np.arange(lay.num_blocks))
+        for s, n in enumerate(nblk):
+            assert np.all(lay.table[s, n:] == -1)
+        assert np.all(lay.cap <= lay.max_blocks * P)
+        # same seed, same pool
+        assert np.array_equal(synth.paged_layout(w, bl, P).table, lay.table)
