@@ -189,7 +189,7 @@ MOE, POE = 1, 2
 def aggregate_select(lp, beta, r, rule: int):
     """MoE (rule 1) / PoE (rule 2) aggregation of the contrastive expert
     distributions (see oracle_aggregate_select).  lp: [B*(N+1), V]; beta, r:
-    [B, N].  Returns dict(token, expert, score, token_gap)."""
+    [B, N].  Returns dict(token, expert, score, token_gap, expert_gap)."""
     lp = _c(lp, np.float64)
     beta = _c(beta, np.float32)
     r = _c(r, np.float32)
@@ -199,10 +199,12 @@ def aggregate_select(lp, beta, r, rule: int):
     ex = np.empty(B, np.int32)
     sc = np.empty(B, np.float64)
     gap = np.empty(B, np.float64)
-    rc = lib().oracle_aggregate_select(_p(lp), _p(beta), _p(r), B, N, V, int(rule), _p(tok), _p(ex), _p(sc), _p(gap))
+    egap = np.empty(B, np.float64)
+    rc = lib().oracle_aggregate_select(_p(lp), _p(beta), _p(r), B, N, V, int(rule), _p(tok), _p(ex), _p(sc), _p(gap),
+                                       _p(egap))
     if rc != 0:
         raise ValueError(f"oracle_aggregate_select rc={rc}")
-    return dict(token=tok, expert=ex, score=sc, token_gap=gap)
+    return dict(token=tok, expert=ex, score=sc, token_gap=gap, expert_gap=egap)
 
 
 def adacad_beta(lp, B, N):

@@ -235,7 +235,8 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
 /* ------------------------------------- dynamic contrast strength (AdaCAD) */
 
 int32_t oracle_aggregate_select(const double* lp, const float* beta, const float* r, int32_t B, int32_t N, int32_t V,
-                                int32_t rule, int32_t* token, int32_t* expert, double* score, double* token_gap) {
+                                int32_t rule, int32_t* token, int32_t* expert, double* score, double* token_gap,
+                                double* expert_gap) {
   if (!lp || !beta || !r || !token || !expert || !score || B < 1 || N < 1 || V < 1 || (rule != 1 && rule != 2))
     return -1;
   double* c = (double*)malloc(sizeof(double) * (size_t)N * V); /* c_k(v) - LSE_k = log p_k(v) */
@@ -290,6 +291,16 @@ int32_t oracle_aggregate_select(const double* lp, const float* beta, const float
     expert[b] = bk + 1;
     score[b] = agg[bv];
     if (token_gap) token_gap[b] = agg[bv] - runner;
+    if (expert_gap) {
+      /* the attribution's margin in log units: log(w p) of the chosen
+       * expert at the token against the best other expert's */
+      double other = -INFINITY;
+      for (int32_t k = 0; k < N; ++k) {
+        const double lk = log(w[k]) + c[(int64_t)k * V + bv];
+        if (k != bk && lk > other) other = lk;
+      }
+      expert_gap[b] = log(w[bk]) + c[(int64_t)bk * V + bv] - other;
+    }
   }
   free(c); free(agg); free(w);
   return 0;
@@ -443,9 +454,7 @@ int32_t oracle_decode_step_ex(const oracle_dims* dm, uint16_t* kc, uint16_t* vc,
     }
   }
   if (rc == 0 && dm->aggregation != 0) {
-    rc = oracle_aggregate_select(lp, beta, r, B, N, V, dm->aggregation, token, expert, score, token_gap);
-    if (expert_gap)
-      for (int32_t b = 0; b < B; ++b) expert_gap[b] = INFINITY;
+    rc = oracle_aggregate_select(lp, beta, r, B, N, V, dm->aggregation, token, expert, score, token_gap, expert_gap);
   } else if (rc == 0) {
     if (dm->score_mode == 1) /* raw logits: z = lp + lse */
       for (int32_t s = 0; s < S; ++s)

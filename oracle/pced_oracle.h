@@ -64,12 +64,15 @@ int32_t oracle_contrastive_select(const double* lp, const float* beta, const flo
  *   rule 2 (PoE): agg(v) = sum_k w_k log p_k(v)
  * token = argmax_v agg (lowest id on exact ties), score = agg(token),
  * expert = argmax_k w_k p_k(token) (1-based, lowest k on ties),
- * token_gap = agg(token) - max_{v != token} agg(v) (+inf when V = 1).
+ * token_gap = agg(token) - max_{v != token} agg(v) (+inf when V = 1),
+ * expert_gap = log(w p)_expert(token) - max_{k != expert} log(w_k p_k(token))
+ * (+inf when N = 1; the near-tie margin of the attribution, in log units).
  * lp [S][V] as in oracle_contrastive_select; gamma does not enter.
  * Parity unpinned against the paper (it names the rules, not the weighting);
  * the tests pin this reading by closed forms. */
 int32_t oracle_aggregate_select(const double* lp, const float* beta, const float* r, int32_t B, int32_t N, int32_t V,
-                                int32_t rule, int32_t* token, int32_t* expert, double* score, double* token_gap);
+                                int32_t rule, int32_t* token, int32_t* expert, double* score, double* token_gap,
+                                double* expert_gap);
 
 /* Dynamic contrast strength (Sec. 3 after Eq. 2: beta_0 is computed as in
  * AdaCAD for the first generated token and kept fixed thereafter).  Reading
@@ -129,8 +132,8 @@ typedef struct oracle_dims {
  * lse_out ([S]) may be NULL.  score_mode 1 feeds the raw logits z = lp + lse
  * to Eq. 2 instead of the log-probabilities (max rule; MoE / PoE do not
  * depend on it: a per-expert constant drops out of the softmax); with
- * aggregation 1 or 2 the token comes from oracle_aggregate_select and
- * expert_gap is +inf.  Returns 0, -1 on bad arguments, -2 when a
+ * aggregation 1 or 2 the token, expert and both gaps come from
+ * oracle_aggregate_select.  Returns 0, -1 on bad arguments, -2 when a
  * cache is full. */
 int32_t oracle_decode_step(const oracle_dims* dm, uint16_t* kc, uint16_t* vc, int64_t layer_elems,
                            const int64_t* kv_off, const int32_t* cap, int32_t* len, const uint16_t* emb_rows,

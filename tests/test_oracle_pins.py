@@ -560,6 +560,10 @@ def test_aggregate_hand_worked_example_separates_max_moe_and_poe():
     # PoE: sqrt of (0.035, 0.07, 0.06) -> token 1, where expert 2 puts more mass
     assert poe["token"][0] == 1 and poe["expert"][0] == 2
     assert abs(poe["score"][0] - 0.5 * math.log(0.07)) < 1e-12
+    # attribution margins (log w p at the token): MoE 0.5*0.7 against 0.5*0.05,
+    # PoE 0.5*0.35 against 0.5*0.2
+    assert abs(moe["expert_gap"][0] - math.log(14.0)) < 1e-12
+    assert abs(poe["expert_gap"][0] - math.log(1.75)) < 1e-12
     # Max (Eq. 3 with gamma = 0, beta = 0): the single most confident expert wins, token 0
     mx = oracle.contrastive_select(lp, beta, r, 0.0, 1, 2)
     assert mx["token"][0] == 0 and mx["expert"][0] == 1
@@ -601,6 +605,13 @@ def test_aggregate_single_expert_is_contrastive_greedy_and_permutation_invariant
     for rule in (oracle.MOE, oracle.POE):
         out = oracle.aggregate_select(lp, beta, r, rule)
         assert out["token"][0] == tok[0] and out["expert"][0] == 1
+        assert out["expert_gap"][0] == math.inf  # no other expert to mistake it for
+    # two copies of one expert with equal scores: an exact attribution tie,
+    # margin 0, the lower index reported
+    lp2 = lp[[0, 1, 1]]
+    for rule in (oracle.MOE, oracle.POE):
+        out = oracle.aggregate_select(lp2, np.full((1, 2), 0.5, np.float32), np.full((1, 2), 0.3, np.float32), rule)
+        assert out["expert"][0] == 1 and out["expert_gap"][0] == 0.0
     z = rng.normal(size=(4, V)) * 2
     lp = z - np.log(np.exp(z).sum(1, keepdims=True))
     beta = np.array([[0.2, 0.7, 0.4]], np.float32)
