@@ -250,8 +250,7 @@ def time_graph(dec, dist, steps, warmup, dev, clocks=None):
 def profile_launches(dec, g_unused, dev, reps):
     """Per-launch device times from stage events recorded inside a captured step."""
     import torch
-    import paper_2601_08670_gb300 as pced
-    kinds = pced.step_launch_kinds(dec.dm)
+    kinds = dec.launch_kinds()
     n = len(kinds)
     events = [torch.cuda.Event(enable_timing=True) for _ in range(n + 1)]
     dec.set_stage_events(events)
@@ -526,6 +525,14 @@ def run_reference(args):
 
 def main():
     args = parse_args()
+    world = dist_env()[1]
+    if args.gpus != world:
+        # one rank per GPU comes from the launcher (torchrun); a mismatch
+        # would silently time fewer GPUs than asked for
+        print(f"bench.py: --gpus {args.gpus} but WORLD_SIZE={world}; launch one rank per GPU with "
+              f"python -m torch.distributed.run --nproc-per-node {args.gpus} bench.py --gpus {args.gpus}",
+              file=sys.stderr)
+        return 2
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)

@@ -240,11 +240,12 @@ typedef struct pced_step_args {
   float* lse_out;           /* optional fp32 [S]: log-sum-exp of each row of h W^T */
   void* workspace;
   size_t workspace_bytes;
-  /* Optional timing hooks: an array of pced_step_launch_count(&dims) + 1
+  /* Optional timing hooks: an array of pced_step_launch_count(args) + 1
    * cudaEvent_t handles (cast to void*).  Event 0 is recorded on `stream`
    * before the first launch and event i+1 right after launch i, so the time
-   * between consecutive events is the device time of that launch.  NULL (or
-   * fewer events) disables recording. */
+   * between consecutive events is the device time of that launch (the
+   * events keep consecutive launches from overlapping).  NULL (or fewer
+   * events) disables recording. */
   void* const* stage_events;
   int32_t n_stage_events;
   /* Dynamic contrast strength: when beta_from_step is nonzero this call
@@ -253,7 +254,7 @@ typedef struct pced_step_args {
    * and uses it for this step's selection; the caller passes it as `beta` to
    * the later steps.  Meant for the first step of a decode; such a call runs
    * the LM head twice (once to materialise the log-probabilities in the
-   * workspace) and records no stage events. */
+   * workspace). */
   int32_t beta_from_step;
   float* beta_out;
   /* Paged caches (PagedAttention-style, as the paper serves): when
@@ -290,9 +291,7 @@ typedef struct pced_step_args {
    * expert reported is argmax_k w_k p_k(token), the score the aggregate;
    * gamma and score_mode do not enter (a per-expert constant drops out of the
    * softmax).  These rules materialise the log-probabilities (S x V fp32 in
-   * the workspace) and take five launches; the stage events then bracket the
-   * attention, the logits pass with its log-sum-exp finalise, and the two
-   * aggregation kernels. */
+   * the workspace) and take five launches (see pced_step_launch_kind). */
   int32_t aggregation;
 } pced_step_args;
 
@@ -305,11 +304,17 @@ typedef struct pced_step_args {
 size_t pced_step_workspace_size(const pced_dims* dims);
 pced_status pced_step(const pced_step_args* args, void* stream);
 
-/* Number of kernel launches one pced_step call makes for these dimensions. */
-int32_t pced_step_launch_count(const pced_dims* dims);
-/* Kind of launch i of pced_step (0-based): "embed", "attn_split",
- * "attn_combine", "lm_head" or "select"; NULL when out of range (static storage). */
-const char* pced_step_launch_kind(const pced_dims* dims, int32_t i);
+/* Number of kernel launches one pced_step call with these arguments makes:
+ * 3 for the max rule with a fixed beta (attention, LM head, selection); a
+ * first step with beta_from_step adds a logits pass, its log-sum-exp
+ * finalise and the beta kernel (6); MoE / PoE run attention, the logits pass,
+ * the finalise and two aggregation kernels (5; 6 with beta_from_step).  Only
+ * the fields dims, beta_from_step and aggregation are read; NULL gives 0. */
+int32_t pced_step_launch_count(const pced_step_args* args);
+/* Kind of launch i (0-based) of such a call: "attention", "lm_head",
+ * "lse_finalize", "adacad_beta", "agg_partials", "agg_select" or "select";
+ * NULL when out of range (static storage). */
+const char* pced_step_launch_kind(const pced_step_args* args, int32_t i);
 
 #ifdef __cplusplus
 }

@@ -89,9 +89,9 @@ def lib(path: str = LIB_PATH):
         L.pced_step_workspace_size.restype = SZ
         L.pced_step.argtypes = [ctypes.POINTER(StepArgs), P]
         L.pced_step.restype = I32
-        L.pced_step_launch_count.argtypes = [ctypes.POINTER(Dims)]
+        L.pced_step_launch_count.argtypes = [ctypes.POINTER(StepArgs)]
         L.pced_step_launch_count.restype = I32
-        L.pced_step_launch_kind.argtypes = [ctypes.POINTER(Dims), I32]
+        L.pced_step_launch_kind.argtypes = [ctypes.POINTER(StepArgs), I32]
         L.pced_step_launch_kind.restype = ctypes.c_char_p
         _lib = L
     return _lib
@@ -245,12 +245,13 @@ def step_workspace_size(dm: Dims) -> int:
     return int(lib().pced_step_workspace_size(ctypes.byref(dm)))
 
 
-def step_launch_count(dm: Dims) -> int:
-    return int(lib().pced_step_launch_count(ctypes.byref(dm)))
+def step_launch_count(args) -> int:
+    """Kernel launches of one pced_step call with these StepArgs."""
+    return int(lib().pced_step_launch_count(ctypes.byref(args)))
 
 
-def step_launch_kinds(dm: Dims) -> list:
-    return [lib().pced_step_launch_kind(ctypes.byref(dm), i).decode() for i in range(step_launch_count(dm))]
+def step_launch_kinds(args) -> list:
+    return [lib().pced_step_launch_kind(ctypes.byref(args), i).decode() for i in range(step_launch_count(args))]
 
 
 class Decoder:
@@ -321,7 +322,11 @@ class Decoder:
         self.args.n_stage_events = len(events)
 
     def launches_per_step(self) -> int:
-        return step_launch_count(self.dm)
+        """Kernel launches of the next step() call."""
+        return step_launch_count(self.args)
+
+    def launch_kinds(self) -> list:
+        return step_launch_kinds(self.args)
 
     def status(self) -> int:
         return device_status(self.ws)

@@ -180,8 +180,12 @@ __global__ void __launch_bounds__(AGG_THREADS) agg_select_kernel(AggArgs a) {
   }
 }
 
-cudaError_t aggregate_launch(const AggArgs& a, cudaStream_t stream) {
+cudaError_t agg_partials_launch(const AggArgs& a, cudaStream_t stream) {
   agg_partials_kernel<<<dim3(a.nchunks, a.N, a.B), AGG_THREADS, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t agg_select_launch(const AggArgs& a, cudaStream_t stream) {
   agg_select_kernel<<<dim3(a.nchunks, a.B), AGG_THREADS, 0, stream>>>(a);
   return cudaGetLastError();
 }

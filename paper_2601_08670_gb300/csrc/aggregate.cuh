@@ -32,6 +32,8 @@ struct AggArgs {
 constexpr int AGG_CHUNK = 1024;  // vocabulary entries per CTA (about 125 CTAs per query at V = 128K)
 constexpr int AGG_MAX_N = 512;   // experts per query (the LM head's row limit)
 inline int32_t agg_chunks(int32_t V) { return (V + AGG_CHUNK - 1) / AGG_CHUNK; }
-cudaError_t aggregate_launch(const AggArgs& a, cudaStream_t stream);
+// (1) per (query, expert, chunk) statistics, (2) per (query, chunk) best and the pick
+cudaError_t agg_partials_launch(const AggArgs& a, cudaStream_t stream);
+cudaError_t agg_select_launch(const AggArgs& a, cudaStream_t stream);
 
 }  // namespace pced

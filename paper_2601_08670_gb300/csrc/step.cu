@@ -88,11 +88,36 @@ extern "C" size_t pced_step_workspace_size(const pced_dims* dm) {
   return step_layout(dm, nullptr).bytes;
 }
 
-extern "C" int32_t pced_step_launch_count(const pced_dims* dm) { return dm ? 3 : 0; }
+// The kernels one pced_step call with these arguments launches, in order
+// (kinds may be NULL); returns their number.
+static int32_t step_plan(const pced_step_args* p, const char** kinds) {
+  int32_t n = 0;
+  auto add = [&](const char* k) {
+    if (kinds) kinds[n] = k;
+    ++n;
+  };
+  const bool dyn = p->beta_from_step != 0, agg = p->aggregation != PCED_AGG_MAX;
+  add("attention");
+  if (dyn || agg) {
+    add("lm_head");  // logits mode: log-probabilities materialised
+    add("lse_finalize");
+    if (dyn) add("adacad_beta");
+  }
+  if (agg) {
+    add("agg_partials");
+    add("agg_select");
+  } else {
+    add("lm_head");  // fused log-softmax statistics and contrastive tile maxima
+    add("select");
+  }
+  return n;
+}
 
-extern "C" const char* pced_step_launch_kind(const pced_dims* dm, int32_t i) {
-  static const char* kinds[3] = {"attention", "lm_head", "select"};
-  if (!dm || i < 0 || i >= pced_step_launch_count(dm)) return nullptr;
+extern "C" int32_t pced_step_launch_count(const pced_step_args* p) { return p ? step_plan(p, nullptr) : 0; }
+
+extern "C" const char* pced_step_launch_kind(const pced_step_args* p, int32_t i) {
+  const char* kinds[8];
+  if (!p || i < 0 || i >= step_plan(p, kinds)) return nullptr;
   return kinds[i];
 }
 
@@ -156,7 +181,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   cudaStream_t s = (cudaStream_t)stream;
   const bool dyn = p->beta_from_step != 0;
   const bool agg = p->aggregation != PCED_AGG_MAX;
-  const bool timed = !dyn && p->stage_events && p->n_stage_events >= pced_step_launch_count(&dm) + 1;
+  const bool timed = p->stage_events && p->n_stage_events >= step_plan(p, nullptr) + 1;
   cudaStreamCaptureStatus cap_status = cudaStreamCaptureStatusNone;
   if (timed && cudaStreamIsCapturing(s, &cap_status) != cudaSuccess) return cuda_status(cudaGetLastError(), "capture query");
   int mark_i = 0;
@@ -253,10 +278,14 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     lz.status = W.status;
     lz.pdl = 0;
     e = lm_head_launch(wmap, hmap, g, lz, s);
+    if (e == cudaSuccess) e = mark();
     if (e == cudaSuccess) e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
+    if (e == cudaSuccess) e = mark();
     // the JSD kernel also re-arms the LM head's tile counter for the fused pass
-    if (e == cudaSuccess && dyn) e = adacad_beta_launch(W.lp, dm.B, dm.N, dm.V, p->beta_out, W.ada, W.lm_tile_ctr, s);
-    if (e == cudaSuccess && agg) e = mark();  // MoE / PoE: the "lm_head" stage is the logits pass and its finalise
+    if (e == cudaSuccess && dyn) {
+      e = adacad_beta_launch(W.lp, dm.B, dm.N, dm.V, p->beta_out, W.ada, W.lm_tile_ctr, s);
+      if (e == cudaSuccess) e = mark();
+    }
     if (e != cudaSuccess) return cuda_status(e, "log-probability launches");
     if (dyn) beta = p->beta_out;
   }
@@ -283,8 +312,10 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ag.max_steps = p->max_steps;
     ag.done_counter = W.done_counter;
     ag.status = W.status;
-    e = aggregate_launch(ag, s);
-    if (e == cudaSuccess) e = mark();  // the "select" stage: the two aggregation kernels
+    e = agg_partials_launch(ag, s);
+    if (e == cudaSuccess) e = mark();
+    if (e == cudaSuccess) e = agg_select_launch(ag, s);
+    if (e == cudaSuccess) e = mark();
     if (e != cudaSuccess) return cuda_status(e, "aggregation launches");
     return PCED_OK;
   }

@@ -146,11 +146,26 @@ def test_step_rejects_bad_arguments(L):
     assert f(step_args(pced, workspace_bytes=100)) == 2
 
 
-def test_launch_count_and_workspace_sizes(L):
+def test_launch_count_and_kinds_follow_the_mode(L):
+    import paper_2601_08670_gb300 as pced
+    assert pced.step_launch_kinds(step_args(pced)) == ["attention", "lm_head", "select"]
+    assert pced.step_launch_kinds(step_args(pced, beta_from_step=1)) == [
+        "attention", "lm_head", "lse_finalize", "adacad_beta", "lm_head", "select"]
+    for rule in (pced.AGG_MOE, pced.AGG_POE):
+        assert pced.step_launch_kinds(step_args(pced, aggregation=rule)) == [
+            "attention", "lm_head", "lse_finalize", "agg_partials", "agg_select"]
+        assert pced.step_launch_kinds(step_args(pced, aggregation=rule, beta_from_step=1)) == [
+            "attention", "lm_head", "lse_finalize", "adacad_beta", "agg_partials", "agg_select"]
+    a = step_args(pced, aggregation=pced.AGG_MOE)
+    assert pced.step_launch_count(a) == 5
+    assert L.pced_step_launch_kind(ctypes.byref(a), 5) is None
+    assert L.pced_step_launch_kind(ctypes.byref(a), -1) is None
+    assert L.pced_step_launch_count(None) == 0
+
+
+def test_workspace_sizes(L):
     import paper_2601_08670_gb300 as pced
     dm = pced.dims(1, 8, 32, 32, 8, 128, 128256)
-    assert pced.step_launch_count(dm) == 3
-    assert pced.step_launch_kinds(dm) == ["attention", "lm_head", "select"]
     assert pced.step_workspace_size(dm) > 0
     assert pced.step_workspace_size(pced.dims(1, 8, 32, 30, 8, 128, 100)) == 0
     assert L.pced_decode_attention_workspace_size(9, 32, 8, 128) > 0

@@ -58,7 +58,7 @@ def test_adacad_beta_degenerate_rows(cuda_ok):
 
 @pytest.mark.parametrize("name,steps,ram", [("tiny", 4, 0), ("llama8", 2, 8)])
 def test_step_with_dynamic_beta(cuda_ok, name, steps, ram):
-    from test_gpu_step import compare_step, host_ram_gb
+    from test_gpu_step import check_stats, compare_step, host_ram_gb, new_stats
     import paper_2601_08670_gb300 as pced
     if host_ram_gb() < ram:
         pytest.skip(f"needs {ram} GB of free host memory for the oracle's caches")
@@ -70,7 +70,7 @@ def test_step_with_dynamic_beta(cuda_ok, name, steps, ram):
                                    dynamic_beta=True)
     from oracle.run import OracleRun
     run = OracleRun(w, dynamic_beta=True)
-    stats = dict(lse=0.0, h=0.0, h_bits_diff=0, h_elems=0, near_ties=0)
+    stats = new_stats()
     for s in range(steps):
         dec.step()
         torch.cuda.synchronize()
@@ -82,3 +82,4 @@ def test_step_with_dynamic_beta(cuda_ok, name, steps, ram):
             assert not np.allclose(got, synth.betas(w))
         compare_step(dec, ref, run, s, stats)
     assert dec.status() == 0
+    check_stats(stats, name)

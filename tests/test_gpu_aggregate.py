@@ -9,7 +9,7 @@ import torch
 import synth
 from gpu_util import near_tie
 from oracle.run import OracleRun
-from test_gpu_step import compare_step, host_ram_gb
+from test_gpu_step import check_stats, compare_step, host_ram_gb, new_stats
 
 pytestmark = pytest.mark.gpu
 
@@ -25,7 +25,7 @@ def run_variant(name, steps, ram, **kw):
     dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
     dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=w.steps, bos=w.bos, keep_hidden=True, **kw)
     run = OracleRun(w, **kw)
-    stats = dict(lse=0.0, h=0.0, h_bits_diff=0, h_elems=0, near_ties=0)
+    stats = new_stats()
     for s in range(steps):
         dec.step()
         torch.cuda.synchronize()
@@ -36,6 +36,7 @@ def run_variant(name, steps, ram, **kw):
                 assert abs(sc[b] - ref["score"][j]) <= SCORE_TOL, f"step {s} query {b}: score {sc[b]} vs {ref['score'][j]}"
         compare_step(dec, ref, run, s, stats)
     assert dec.status() == 0
+    check_stats(stats, f"{name} {kw}")
     return stats
 
 
@@ -63,7 +64,7 @@ def test_moe_with_dynamic_beta_and_graph_replay(cuda_ok):
     dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=w.steps, bos=w.bos, keep_hidden=True,
                                    aggregation=1, dynamic_beta=True)
     run = OracleRun(w, aggregation=1, dynamic_beta=True)
-    stats = dict(lse=0.0, h=0.0, h_bits_diff=0, h_elems=0, near_ties=0)
+    stats = new_stats()
     dec.step()
     torch.cuda.synchronize()
     compare_step(dec, run.step(), run, 0, stats)
@@ -78,3 +79,4 @@ def test_moe_with_dynamic_beta_and_graph_replay(cuda_ok):
         torch.cuda.synchronize()
         compare_step(dec, run.step(), run, i, stats)
     assert dec.status() == 0
+    check_stats(stats, "tiny moe dynamic beta graph")

@@ -38,7 +38,7 @@ def test_paged_pool_holds_the_logical_cache(cuda_ok):
 def test_paged_step_matches_oracle(cuda_ok, name, P, steps, queries, ram):
     import paper_2601_08670_gb300 as pced
     from oracle.run import OracleRun
-    from test_gpu_step import compare_step, host_ram_gb
+    from test_gpu_step import check_stats, compare_step, host_ram_gb, new_stats
     if host_ram_gb() < ram:
         pytest.skip(f"needs {ram} GB of free host memory for the oracle's caches")
     w = synth.get(name)
@@ -46,12 +46,13 @@ def test_paged_step_matches_oracle(cuda_ok, name, P, steps, queries, ram):
     dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
     dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=w.steps, bos=w.bos, keep_hidden=True)
     run = OracleRun(w, queries=queries)
-    stats = dict(lse=0.0, h=0.0, h_bits_diff=0, h_elems=0, near_ties=0)
+    stats = new_stats()
     for s in range(steps):
         dec.step()
         torch.cuda.synchronize()
         compare_step(dec, run.step(), run, s, stats)
     assert dec.status() == 0
+    check_stats(stats, f"{name} paged {P}")
 
 
 def test_paged_agrees_with_slab(cuda_ok):

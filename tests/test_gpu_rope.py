@@ -10,7 +10,7 @@ import torch
 import synth
 from gpu_util import bf16_bits, bits_to_f64
 from oracle.run import OracleRun
-from test_gpu_step import compare_step, host_ram_gb
+from test_gpu_step import check_stats, compare_step, host_ram_gb, new_stats
 
 pytestmark = pytest.mark.gpu
 
@@ -31,7 +31,7 @@ def test_rope_step_matches_oracle(cuda_ok, name, theta, steps, paged, ram):
     dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=w.steps, bos=w.bos, keep_hidden=True,
                                    rope_theta=theta)
     run = OracleRun(w, rope_theta=theta)
-    stats = dict(lse=0.0, h=0.0, h_bits_diff=0, h_elems=0, near_ties=0)
+    stats = new_stats()
     for s in range(steps):
         pos = run.lens.copy()  # the new token's position in every sequence
         dec.step()
@@ -62,6 +62,7 @@ def test_rope_step_matches_oracle(cuda_ok, name, theta, steps, paged, ram):
                         total += a.size
         assert same >= 0.98 * total, f"{same}/{total} appended elements bit-equal"
     assert dec.status() == 0
+    check_stats(stats, f"{name} rope {theta}")
 
 
 def test_rope_changes_the_step_and_zero_theta_is_the_plain_step(cuda_ok):

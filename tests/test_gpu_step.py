@@ -18,6 +18,15 @@ from oracle.run import OracleRun
 pytestmark = pytest.mark.gpu
 
 LSE_TOL = 1e-2  # spec log-prob tolerance (absolute)
+# Hidden state h = bf16(rmsnorm(x_L)) after the whole attention chain: every
+# element within the spec attention bound, 2e-2 of the largest
+# magnitude of its (sequence, head) block, and most elements bit-equal (fp32
+# accumulation against fp64 moves a bf16 rounding only near a midpoint).
+H_REL_TOL = 2e-2
+H_BITS_MIN = 0.98
+# Selections within 1e-3 of a tie are not compared; a run where they are
+# more than a quarter of the comparisons proves too little.
+MAX_NEAR_TIE_FRAC = 0.25
 
 
 def host_ram_gb() -> float:
@@ -34,6 +43,25 @@ def make_decoder(w, dev):
     return pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=w.steps, bos=w.bos, keep_hidden=True), t
 
 
+def new_stats() -> dict:
+    return dict(lse=0.0, h=0.0, h_rel=0.0, h_bits_diff=0, h_elems=0, near_ties=0, compared=0)
+
+
+def compare_hidden(h_gpu, h_ref, Hq, what, stats):
+    """h_gpu, h_ref: bf16 bit patterns [rows, Hq*D]; asserts the block bound."""
+    g = bits_to_f64(h_gpu).reshape(h_gpu.shape[0], Hq, -1)
+    r = bits_to_f64(h_ref).reshape(h_ref.shape[0], Hq, -1)
+    err = np.abs(g - r).max(axis=2)
+    mag = np.abs(r).max(axis=2)
+    rel = err / np.maximum(mag, 1e-30)
+    stats["h"] = max(stats["h"], float(err.max()))
+    stats["h_rel"] = max(stats["h_rel"], float(rel.max()))
+    stats["h_bits_diff"] += int((h_gpu != h_ref).sum())
+    stats["h_elems"] += h_gpu.size
+    worst = np.unravel_index(np.argmax(rel), rel.shape)
+    assert np.all(err <= H_REL_TOL * mag), f"{what}: hidden state row {worst[0]} head {worst[1]} rel err {rel.max():.3e}"
+
+
 def compare_step(dec, ref, run, t, stats):
     w = run.w
     tok = dec.history[:, t].cpu().numpy()
@@ -46,10 +74,8 @@ def compare_step(dec, ref, run, t, stats):
         err = np.abs(lse[rows] - ref["lse"][lo]).max()
         stats["lse"] = max(stats["lse"], err)
         assert err <= LSE_TOL, f"step {t} query {b}: lse err {err:.3e}"
-        hd = np.abs(bits_to_f64(h[rows]) - bits_to_f64(ref["h"][lo]))
-        stats["h"] = max(stats["h"], float(hd.max()))
-        stats["h_bits_diff"] += int((h[rows] != ref["h"][lo]).sum())
-        stats["h_elems"] += h[rows].size
+        compare_hidden(h[rows], ref["h"][lo], w.Hq, f"step {t} query {b}", stats)
+        stats["compared"] += 1
         if near_tie(ref, j):
             stats["near_ties"] += 1
         else:
@@ -59,6 +85,18 @@ def compare_step(dec, ref, run, t, stats):
         dec.history[b, t] = int(ref["token"][j])
 
 
+def check_stats(stats, name=""):
+    """The run-level bounds: bf16 bit-equality of the hidden states and the
+    share of selections left uncompared as near ties."""
+    print(f"{name}: {stats}")
+    assert stats["compared"] > 0
+    eq = 1.0 - stats["h_bits_diff"] / max(1, stats["h_elems"])
+    assert eq >= H_BITS_MIN, f"{name}: only {eq:.4f} of the hidden-state elements bit-equal"
+    nt = stats["near_ties"]
+    assert nt < stats["compared"], f"{name}: every selection was a near tie"
+    assert nt <= MAX_NEAR_TIE_FRAC * stats["compared"], f"{name}: {nt} near ties in {stats['compared']} selections"
+
+
 def run_parity(name, steps, queries=None, graph=False, min_ram_gb=0.0):
     if host_ram_gb() < min_ram_gb:
         pytest.skip(f"needs {min_ram_gb} GB of free host memory for the oracle's caches")
@@ -66,7 +104,7 @@ def run_parity(name, steps, queries=None, graph=False, min_ram_gb=0.0):
     w = synth.get(name)
     dec, _ = make_decoder(w, dev)
     run = OracleRun(w, queries=queries)
-    stats = dict(lse=0.0, h=0.0, h_bits_diff=0, h_elems=0, near_ties=0)
+    stats = new_stats()
     g = None
     if graph:
         s = torch.cuda.Stream()
@@ -88,7 +126,7 @@ def run_parity(name, steps, queries=None, graph=False, min_ram_gb=0.0):
     assert int(dec.step_t.item()) == steps
     lens = dec.seq_len.cpu().numpy()
     assert np.array_equal(lens, synth.base_lengths(w) + steps)
-    print(f"{name}: {stats}")
+    check_stats(stats, name)
     return stats
 
 
@@ -101,7 +139,8 @@ def test_tiny_graph_replay(cuda_ok):
 
 
 def test_llama8_full_size(cuda_ok):
-    run_parity("llama8", 3, min_ram_gb=8)
+    # every step of the benchmarked workload (64), teacher-forced
+    run_parity("llama8", 64, min_ram_gb=8)
 
 
 def test_llama8_graph_replay(cuda_ok):
@@ -117,19 +156,19 @@ def test_llama8_sequence_groups(cuda_ok, monkeypatch, groups):
 
 
 def test_qwen_flat_full_size(cuda_ok):
-    run_parity("qwen_flat", 2, min_ram_gb=10)
+    run_parity("qwen_flat", 6, min_ram_gb=10)
 
 
 def test_qwen_onehot_full_size(cuda_ok):
-    run_parity("qwen_onehot", 2, min_ram_gb=10)
+    run_parity("qwen_onehot", 6, min_ram_gb=10)
 
 
-def test_manydoc_first_and_last_query(cuda_ok):
-    run_parity("manydoc", 2, queries=[0, 15], min_ram_gb=8)
+def test_manydoc_all_queries(cuda_ok):
+    run_parity("manydoc", 2, min_ram_gb=24)
 
 
 def test_llama32_ragged_full_size(cuda_ok):
-    run_parity("llama32", 2, min_ram_gb=40)
+    run_parity("llama32", 4, min_ram_gb=40)
 
 
 def test_llama8_top64_experts(cuda_ok):
@@ -138,7 +177,7 @@ def test_llama8_top64_experts(cuda_ok):
 
 
 def test_llama8_top128_experts(cuda_ok):
-    run_parity("llama8_k128", 1, min_ram_gb=44)
+    run_parity("llama8_k128", 2, min_ram_gb=44)
 
 
 def test_cache_full_is_flagged_not_faulted(cuda_ok):
