@@ -229,6 +229,14 @@ typedef struct pced_step_args {
   int32_t* history;         /* [B][max_steps] chosen tokens */
   int32_t* expert_trace;    /* [B][max_steps] winning expert (1-based), may be NULL */
   float* score_trace;       /* [B][max_steps] winning score, may be NULL */
+  /* [B][max_steps][2] near-tie margins of each choice (Eq. 3), may be NULL:
+   * the token gap, score minus the best score at any other token over all
+   * experts, and the expert gap, score minus the best other expert's score
+   * at the chosen token (+inf with one expert).  MoE / PoE report the
+   * aggregate's token gap and the attribution's margin in log(w p).  A
+   * choice within a small gap is a near tie: its token or expert could flip
+   * under a change of summation order. */
+  float* gap_trace;
   int32_t max_steps;
   const float* beta;        /* [B][N] */
   const float* r;           /* [B][N] relevance scores */
@@ -252,9 +260,10 @@ typedef struct pced_step_args {
    * computes beta from this step's distributions (as pced_adacad_beta), writes
    * it to beta_out (device fp32 [B][N], may be the array `beta` points to)
    * and uses it for this step's selection; the caller passes it as `beta` to
-   * the later steps.  Meant for the first step of a decode; such a call runs
-   * the LM head twice (once to materialise the log-probabilities in the
-   * workspace). */
+   * the later steps.  Meant for the first step of a decode; such a call
+   * materialises the log-probabilities (S x V fp32 in the workspace) in a
+   * logits pass of the LM head and selects from them (Eq. 3 on materialised
+   * log-probabilities). */
   int32_t beta_from_step;
   float* beta_out;
   /* Paged caches (PagedAttention-style, as the paper serves): when
@@ -293,6 +302,12 @@ typedef struct pced_step_args {
    * softmax).  These rules materialise the log-probabilities (S x V fp32 in
    * the workspace) and take five launches (see pced_step_launch_kind). */
   int32_t aggregation;
+  /* How long (ns) a warp of the attention kernel waits for another warp or
+   * CTA (a layer's input, a partial record, a pipeline stage) before it sets
+   * PCED_DEV_TIMEOUT and unwinds; the kernel then returns without its
+   * results.  0: 2 s.  A CTA still waits for its own tile copies in flight
+   * (up to 2 s) before it exits. */
+  uint64_t wait_limit_ns;
 } pced_step_args;
 
 #define PCED_SCORE_LOGPROB 0
@@ -306,10 +321,11 @@ pced_status pced_step(const pced_step_args* args, void* stream);
 
 /* Number of kernel launches one pced_step call with these arguments makes:
  * 3 for the max rule with a fixed beta (attention, LM head, selection); a
- * first step with beta_from_step adds a logits pass, its log-sum-exp
- * finalise and the beta kernel (6); MoE / PoE run attention, the logits pass,
- * the finalise and two aggregation kernels (5; 6 with beta_from_step).  Only
- * the fields dims, beta_from_step and aggregation are read; NULL gives 0. */
+ * first step with beta_from_step runs attention, a logits pass, its
+ * log-sum-exp finalise, the beta kernel and a selection from the
+ * log-probabilities (5); MoE / PoE run attention, the logits pass, the
+ * finalise and two aggregation kernels (5; 6 with beta_from_step).  Only the
+ * fields dims, beta_from_step and aggregation are read; NULL gives 0. */
 int32_t pced_step_launch_count(const pced_step_args* args);
 /* Kind of launch i (0-based) of such a call: "attention", "lm_head",
  * "lse_finalize", "adacad_beta", "agg_partials", "agg_select" or "select";

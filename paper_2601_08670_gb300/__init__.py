@@ -40,14 +40,16 @@ class StepArgs(ctypes.Structure):
                 ("k_cache", ctypes.c_void_p), ("v_cache", ctypes.c_void_p), ("layer_elems", ctypes.c_int64),
                 ("kv_offset", ctypes.c_void_p), ("cap", ctypes.c_void_p), ("total_cap", ctypes.c_int64),
                 ("seq_len", ctypes.c_void_p), ("step", ctypes.c_void_p), ("history", ctypes.c_void_p),
-                ("expert_trace", ctypes.c_void_p), ("score_trace", ctypes.c_void_p), ("max_steps", ctypes.c_int32),
+                ("expert_trace", ctypes.c_void_p), ("score_trace", ctypes.c_void_p), ("gap_trace", ctypes.c_void_p),
+                ("max_steps", ctypes.c_int32),
                 ("beta", ctypes.c_void_p), ("r", ctypes.c_void_p), ("gamma", ctypes.c_float),
                 ("attn_scale", ctypes.c_float), ("rms_eps", ctypes.c_float), ("bos_token", ctypes.c_int32),
                 ("hidden_out", ctypes.c_void_p), ("lse_out", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
                 ("workspace_bytes", ctypes.c_size_t), ("stage_events", ctypes.c_void_p),
                 ("n_stage_events", ctypes.c_int32), ("beta_from_step", ctypes.c_int32), ("beta_out", ctypes.c_void_p),
                 ("block_table", ctypes.c_void_p), ("block_rows", ctypes.c_int32), ("max_blocks", ctypes.c_int32),
-                ("rope_theta", ctypes.c_float), ("score_mode", ctypes.c_int32), ("aggregation", ctypes.c_int32)]
+                ("rope_theta", ctypes.c_float), ("score_mode", ctypes.c_int32), ("aggregation", ctypes.c_int32),
+                ("wait_limit_ns", ctypes.c_uint64)]
 
 
 _lib = None
@@ -264,7 +266,8 @@ class Decoder:
     def __init__(self, dm: Dims, *, embed, w_unembed, k_cache, v_cache, layer_elems: int, kv_offset, cap, seq_len,
                  beta, r, gamma: float, max_steps: int, total_cap: int, bos: int = 0, attn_scale=None,
                  rms_eps: float = 1e-6, keep_hidden: bool = False, dynamic_beta: bool = False, block_table=None,
-                 block_rows: int = 0, rope_theta: float = 0.0, score_mode: int = 0, aggregation: int = 0):
+                 block_rows: int = 0, rope_theta: float = 0.0, score_mode: int = 0, aggregation: int = 0,
+                 track_gaps: bool = True):
         dev = k_cache.device
         self.dm = dm
         B, S, d = dm.B, dm.B * (dm.N + 1), dm.Hq * dm.D
@@ -272,6 +275,8 @@ class Decoder:
         self.history = torch.zeros((B, max_steps), dtype=torch.int32, device=dev)
         self.expert_trace = torch.zeros((B, max_steps), dtype=torch.int32, device=dev)
         self.score_trace = torch.zeros((B, max_steps), dtype=torch.float32, device=dev)
+        # near-tie margins of every choice: [B, max_steps, 2] (token gap, expert gap)
+        self.gap_trace = torch.zeros((B, max_steps, 2), dtype=torch.float32, device=dev) if track_gaps else None
         self.hidden = torch.zeros((S, d), dtype=torch.bfloat16, device=dev) if keep_hidden else None
         self.lse = torch.zeros(S, dtype=torch.float32, device=dev)
         self.ws = workspace(step_workspace_size(dm), dev)
@@ -281,7 +286,8 @@ class Decoder:
         self.args = StepArgs(
             dm, _ptr(embed), _ptr(w_unembed), _ptr(k_cache), _ptr(v_cache), int(layer_elems), _ptr(kv_offset),
             _ptr(cap), int(total_cap), _ptr(seq_len), _ptr(self.step_t), _ptr(self.history),
-            _ptr(self.expert_trace), _ptr(self.score_trace), int(max_steps), _ptr(beta), _ptr(r), float(gamma),
+            _ptr(self.expert_trace), _ptr(self.score_trace), _ptr(self.gap_trace), int(max_steps), _ptr(beta), _ptr(r),
+            float(gamma),
             float(1.0 / math.sqrt(dm.D) if attn_scale is None else attn_scale), float(rms_eps), int(bos),
             _ptr(self.hidden), _ptr(self.lse), _ptr(self.ws), self.ws.numel())
         self.max_steps = max_steps
@@ -334,7 +340,8 @@ class Decoder:
 
 def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos: int = 0, keep_hidden=False,
                         attn_scale=None, rms_eps: float = 1e-6, dynamic_beta: bool = False,
-                        rope_theta: float = 0.0, score_mode: int = 0, aggregation: int = 0) -> Decoder:
+                        rope_theta: float = 0.0, score_mode: int = 0, aggregation: int = 0,
+                        track_gaps: bool = True) -> Decoder:
     """Decoder over a dict of device tensors with the keys k_cache, v_cache,
     kv_offset, cap, seq_len, embed, w_unembed, beta, r, and the host layout
     values layer_elems / total_cap (or a `layout` object carrying them)."""
@@ -346,4 +353,4 @@ def decoder_from_inputs(dm: Dims, t: dict, *, gamma: float, max_steps: int, bos:
                    beta=t["beta"], r=t["r"], gamma=gamma, max_steps=max_steps, total_cap=total_cap, bos=bos,
                    attn_scale=attn_scale, rms_eps=rms_eps, keep_hidden=keep_hidden, dynamic_beta=dynamic_beta,
                    block_table=t.get("block_table"), block_rows=int(t.get("block_rows", 0)), rope_theta=rope_theta,
-                   score_mode=score_mode, aggregation=aggregation)
+                   score_mode=score_mode, aggregation=aggregation, track_gaps=track_gaps)

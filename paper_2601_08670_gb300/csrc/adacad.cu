@@ -17,7 +17,7 @@
 namespace pced {
 
 constexpr int ADA_THREADS = 256;
-constexpr int ADA_CHUNK = 8192;  // vocabulary entries per CTA
+constexpr int ADA_CHUNK = 2048;  // vocabulary entries per CTA (about 500 CTAs at llama8: every SM busy)
 
 int32_t adacad_chunks(int32_t V) { return (V + ADA_CHUNK - 1) / ADA_CHUNK; }
 

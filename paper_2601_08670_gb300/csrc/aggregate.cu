@@ -8,11 +8,12 @@
 //   token = argmax_v agg (lowest id on ties), score = agg(token),
 //   expert = argmax_k w_k p_k(token) (lowest k on ties).
 // Two launches over the materialised log-probabilities (S x V fp32, a few MB,
-// L2-resident): (1) per (query, expert, chunk) the max and sum of exp of c_k;
-// (2) per (query, chunk) the best aggregate, every CTA first merging the
-// chunk statistics of its query into log-sum-exps; the last CTA of a query
-// picks the token across chunks and writes the step's results.  Every sum
-// runs in a fixed order, so results do not depend on timing.
+// L2-resident): (1) per (query, expert, chunk) the max and sum of exp of c_k,
+// merged into the expert's log-sum-exp by the last chunk to finish; (2) per
+// (query, chunk) the best aggregate and the best at another token; the last
+// CTA of a query picks the token across chunks, attributes the expert and
+// writes the step's results with both near-tie margins.  Every sum runs in a
+// fixed order, so results do not depend on timing.
 #include <math.h>
 
 #include "aggregate.cuh"
@@ -33,31 +34,56 @@ __device__ __forceinline__ void agg_lse_merge(float& m, float& s, float m2, floa
   m = M;
 }
 
-// grid (nchunks, N, B)
+// grid (nchunks, N, B): the chunk's (max, sum exp) of c_k; the last chunk CTA
+// of (query, expert) to finish merges them all into lse_k (strided, then a
+// fixed tree: the order does not depend on which CTA is last)
 __global__ void __launch_bounds__(AGG_THREADS) agg_partials_kernel(AggArgs a) {
   const int c = blockIdx.x, k = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int N = a.N, V = a.V;
   const float* lp0 = a.lp + (int64_t)b * (N + 1) * V;
   const float* lpk = lp0 + (int64_t)(k + 1) * V;
   const float bt = a.beta[b * N + k];
+  __shared__ float2 red[AGG_THREADS / 32];
+  __shared__ int last;
+  auto block_merge = [&](float m, float s) -> float2 {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
+      agg_lse_merge(m, s, m2, s2);
+    }
+    if ((tid & 31) == 0) red[tid >> 5] = make_float2(m, s);
+    __syncthreads();
+    float M = -INFINITY, Sm = 0.f;
+    for (int w = 0; w < AGG_THREADS / 32; ++w) agg_lse_merge(M, Sm, red[w].x, red[w].y);
+    __syncthreads();
+    return make_float2(M, Sm);
+  };
   float m = -INFINITY, s = 0.f;
   const int v1 = min(V, (c + 1) * AGG_CHUNK);
   for (int v = c * AGG_CHUNK + tid; v < v1; v += AGG_THREADS) {
     const float ck = (1.f + bt) * lpk[v] - bt * lp0[v];
     agg_lse_merge(m, s, ck, 1.f);
   }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
-    agg_lse_merge(m, s, m2, s2);
-  }
-  __shared__ float2 red[AGG_THREADS / 32];
-  if ((tid & 31) == 0) red[tid >> 5] = make_float2(m, s);
-  __syncthreads();
+  const float2 ms = block_merge(m, s);
+  const int64_t pk = (int64_t)b * N + k;
   if (tid == 0) {
-    float M = -INFINITY, Sm = 0.f;
-    for (int w = 0; w < AGG_THREADS / 32; ++w) agg_lse_merge(M, Sm, red[w].x, red[w].y);
-    a.part[((int64_t)b * N + k) * a.nchunks + c] = make_float2(M, Sm);
+    a.part[pk * a.nchunks + c] = ms;
+    __threadfence();
+    last = atomicAdd(a.kdone + pk, 1) == a.nchunks - 1;
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();  // the other chunks' statistics are visible
+  m = -INFINITY;
+  s = 0.f;
+  for (int j = tid; j < a.nchunks; j += AGG_THREADS) {
+    const float2 e = __ldcg(a.part + pk * a.nchunks + j);
+    agg_lse_merge(m, s, e.x, e.y);
+  }
+  const float2 t = block_merge(m, s);
+  if (tid == 0) {
+    a.lse_k[pk] = t.x + logf(t.y);
+    a.kdone[pk] = 0;
   }
 }
 
@@ -65,24 +91,42 @@ __global__ void __launch_bounds__(AGG_THREADS) agg_partials_kernel(AggArgs a) {
 __device__ __forceinline__ bool agg_better(float v2, int t2, float v1, int t1) {
   return v2 > v1 || (v2 == v1 && t2 < t1);
 }
+// top-2 over disjoint token sets: (b1, t1) best, b2 best value at another token
+__device__ __forceinline__ void agg_top2(float& b1, int& t1, float& b2, float r1, int rt, float r2) {
+  if (agg_better(r1, rt, b1, t1)) {
+    b2 = fmaxf(b1, r2);
+    b1 = r1;
+    t1 = rt;
+  } else {
+    b2 = fmaxf(b2, r1);
+  }
+}
 
-// grid (nchunks, B)
+// grid (nchunks, B).  rule 0 is Eq. 3 itself on the materialised
+// log-probabilities: per token the best expert's score of Eq. 2 (the first
+// step of a dynamic-beta decode selects this way, from the log-probabilities
+// it has written for beta anyway); rules 1 and 2 are MoE and PoE.
 __global__ void __launch_bounds__(AGG_THREADS) agg_select_kernel(AggArgs a) {
   const int c = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int N = a.N, V = a.V, n1 = N + 1;
   __shared__ float w_s[AGG_MAX_N], lse_s[AGG_MAX_N], beta_s[AGG_MAX_N];
   __shared__ float wsum;
-  __shared__ float bv_s[AGG_THREADS / 32];
+  __shared__ float bv_s[AGG_THREADS / 32], b2_s[AGG_THREADS / 32];
   __shared__ int bt_s[AGG_THREADS / 32];
   __shared__ int last;
   if (c == 0 && b == 0 && tid == 0 && a.tile_ctr) *a.tile_ctr = 0;  // the next LM head claims its tiles from 0
   for (int k = tid; k < N; k += AGG_THREADS) {
     w_s[k] = fminf(fmaxf(a.r[b * N + k], 1e-8f), 1.0f);
     beta_s[k] = a.beta[b * N + k];
-    float m = -INFINITY, s = 0.f;
-    const float2* pk = a.part + ((int64_t)b * N + k) * a.nchunks;
-    for (int j = 0; j < a.nchunks; ++j) agg_lse_merge(m, s, pk[j].x, pk[j].y);
-    lse_s[k] = m + logf(s);
+    if (a.rule == 0) {
+      // the per-expert constant of Eq. 2: gamma log r_k (plus the log-sum-exps
+      // when s_k are raw logits: z = lp + L)
+      const float btk = beta_s[k];
+      lse_s[k] = a.gamma * logf(w_s[k]) +
+                 (a.raw_logits ? (1.f + btk) * a.lse[b * n1 + 1 + k] - btk * a.lse[b * n1] : 0.f);
+    } else {
+      lse_s[k] = a.lse_k[(int64_t)b * N + k];
+    }
   }
   __syncthreads();
   if (tid == 0) {
@@ -93,69 +137,77 @@ __global__ void __launch_bounds__(AGG_THREADS) agg_select_kernel(AggArgs a) {
   __syncthreads();
   const float inv_w = 1.0f / wsum;
   const float* lp0 = a.lp + (int64_t)b * n1 * V;
-  float bv = -INFINITY;
+  // the chunk's best aggregate and token, and the best at another token
+  float bv = -INFINITY, b2 = -INFINITY;
   int bt = 0x7fffffff;
   const int v1 = min(V, (c + 1) * AGG_CHUNK);
   for (int v = c * AGG_CHUNK + tid; v < v1; v += AGG_THREADS) {
     const float l0 = lp0[v];
-    float acc = 0.f;
+    float acc = a.rule == 0 ? -INFINITY : 0.f;
     for (int k = 0; k < N; ++k) {
+      if (a.rule == 0) {
+        acc = fmaxf(acc, (1.f + beta_s[k]) * lp0[(int64_t)(k + 1) * V + v] - beta_s[k] * l0 + lse_s[k]);
+        continue;
+      }
       const float lpk = (1.f + beta_s[k]) * lp0[(int64_t)(k + 1) * V + v] - beta_s[k] * l0 - lse_s[k];  // log p_k(v)
       acc += a.rule == 1 ? w_s[k] * inv_w * expf(lpk) : w_s[k] * inv_w * lpk;
     }
     const float agg = a.rule == 1 ? logf(acc) : acc;
-    if (agg_better(agg, v, bv, bt)) {
-      bv = agg;
-      bt = v;
-    }
+    agg_top2(bv, bt, b2, agg, v, -INFINITY);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    const float v2 = __shfl_xor_sync(0xffffffffu, bv, o);
+    const float v2 = __shfl_xor_sync(0xffffffffu, bv, o), s2 = __shfl_xor_sync(0xffffffffu, b2, o);
     const int t2 = __shfl_xor_sync(0xffffffffu, bt, o);
-    if (agg_better(v2, t2, bv, bt)) {
-      bv = v2;
-      bt = t2;
-    }
+    agg_top2(bv, bt, b2, v2, t2, s2);
   }
   if (lane == 0) {
     bv_s[warp] = bv;
     bt_s[warp] = bt;
+    b2_s[warp] = b2;
   }
   __syncthreads();
   if (tid == 0) {
-    for (int w = 1; w < AGG_THREADS / 32; ++w)
-      if (agg_better(bv_s[w], bt_s[w], bv, bt)) {
-        bv = bv_s[w];
-        bt = bt_s[w];
-      }
+    for (int w = 1; w < AGG_THREADS / 32; ++w) agg_top2(bv, bt, b2, bv_s[w], bt_s[w], b2_s[w]);
     a.best[(int64_t)b * a.nchunks + c] = make_float2(bv, __int_as_float(bt));
+    a.best2[(int64_t)b * a.nchunks + c] = b2;
     __threadfence();
     last = atomicAdd(a.qdone + b, 1) == a.nchunks - 1;
   }
   __syncthreads();
-  if (!last || tid != 0) return;
+  if (!last || warp != 0) return;
   __threadfence();  // the other chunks' results of query b are visible
-  float sv = -INFINITY;
+  // best over the chunks (one warp, lanes over chunks, then a tree)
+  float sv = -INFINITY, sv2 = -INFINITY;
   int st = 0x7fffffff;
-  for (int j = 0; j < a.nchunks; ++j) {
+  for (int j = lane; j < a.nchunks; j += 32) {
     const float2 e = __ldcg(a.best + (int64_t)b * a.nchunks + j);
-    if (agg_better(e.x, __float_as_int(e.y), sv, st)) {
-      sv = e.x;
-      st = __float_as_int(e.y);
-    }
+    agg_top2(sv, st, sv2, e.x, __float_as_int(e.y), __ldcg(a.best2 + (int64_t)b * a.nchunks + j));
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float v2 = __shfl_xor_sync(0xffffffffu, sv, o), s2 = __shfl_xor_sync(0xffffffffu, sv2, o);
+    const int t2 = __shfl_xor_sync(0xffffffffu, st, o);
+    agg_top2(sv, st, sv2, v2, t2, s2);
   }
   if (st >= V) st = 0;  // no finite aggregate (degenerate rows): token 0
-  int bk = 0;
-  float bp = -INFINITY;
-  for (int k = 0; k < N; ++k) {  // the expert that puts the most weighted mass on the token
-    const float lpk = (1.f + beta_s[k]) * lp0[(int64_t)(k + 1) * V + st] - beta_s[k] * lp0[st] - lse_s[k];
-    const float pw = logf(w_s[k]) + lpk;
-    if (pw > bp) {
-      bp = pw;
-      bk = k;
-    }
+  // the expert: for Eq. 3 the best score at the token, for MoE / PoE the
+  // one that puts the most weighted mass on it (log(w p)); lowest k on
+  // ties, and the margin to the next one
+  float bp = -INFINITY, bp2 = -INFINITY;
+  int bk = 0x7fffffff;
+  for (int k = lane; k < N; k += 32) {
+    const float ck = (1.f + beta_s[k]) * lp0[(int64_t)(k + 1) * V + st] - beta_s[k] * lp0[st];
+    agg_top2(bp, bk, bp2, a.rule == 0 ? ck + lse_s[k] : logf(w_s[k]) + ck - lse_s[k], k, -INFINITY);
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float v2 = __shfl_xor_sync(0xffffffffu, bp, o), s2 = __shfl_xor_sync(0xffffffffu, bp2, o);
+    const int t2 = __shfl_xor_sync(0xffffffffu, bk, o);
+    agg_top2(bp, bk, bp2, v2, t2, s2);
+  }
+  if (bk >= N) bk = 0;
+  if (lane != 0) return;
   a.qdone[b] = 0;
   if (a.lse_out)
     for (int j = 0; j < n1; ++j) a.lse_out[b * n1 + j] = a.lse[b * n1 + j];
@@ -168,6 +220,7 @@ __global__ void __launch_bounds__(AGG_THREADS) agg_select_kernel(AggArgs a) {
       a.history[(int64_t)b * a.max_steps + t] = st;
       if (a.expert_trace) a.expert_trace[(int64_t)b * a.max_steps + t] = bk + 1;
       if (a.score_trace) a.score_trace[(int64_t)b * a.max_steps + t] = sv;
+      if (a.gap_trace) a.gap_trace[(int64_t)b * a.max_steps + t] = make_float2(sv - sv2, bp - bp2);
     } else {
       dev_flag(a.status, PCED_DEV_STEP_LIMIT);
     }

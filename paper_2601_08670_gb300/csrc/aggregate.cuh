@@ -10,9 +10,14 @@ struct AggArgs {
   const float* beta;    // [B][N]
   const float* r;       // [B][N] relevance scores
   const float* lse;     // [S] log-sum-exps of the rows (copied to lse_out)
-  int32_t B, N, V, rule, nchunks;  // rule 1 MoE, 2 PoE
+  int32_t B, N, V, rule, nchunks;  // rule 0 Eq. 3 (max over experts), 1 MoE, 2 PoE
+  float gamma;          // rule 0: weight of the retrieval prior
+  int raw_logits;       // rule 0: s_k of Eq. 2 are the raw logits lp + lse
   float2* part;         // [B][N][nchunks] (max, sum exp) of c_k over each chunk
+  int32_t* kdone;       // [B][N] chunks finished per expert (zero at launch; the last resets it)
+  float* lse_k;         // [B][N] log-sum-exp of c_k (the softmax normaliser of p_k)
   float2* best;         // [B][nchunks] (aggregate, token) of each chunk
+  float* best2;         // [B][nchunks] the chunk's best aggregate at another token
   int32_t* qdone;       // [B] chunks finished (zero at launch; the last resets it)
   int* tile_ctr;        // optional: the LM head's tile counter, reset for its next launch
   int32_t* token;       // optional [B]
@@ -24,6 +29,7 @@ struct AggArgs {
   int32_t* history;
   int32_t* expert_trace;
   float* score_trace;
+  float2* gap_trace;    // optional [B][max_steps]: (token gap, attribution margin)
   int32_t max_steps;
   int32_t* done_counter;
   int* status;

@@ -582,10 +582,10 @@ __device__ __forceinline__ float tv_value(uint64_t w) { return __uint_as_float((
 __device__ __forceinline__ bool tv_ok(uint64_t w, uint32_t tag) { return (uint32_t)(w >> 32) == tag; }
 
 // Bounded poll used by the tagged waits: false once the time limit is spent.
-__device__ __forceinline__ bool poll_again(uint64_t& t0, int* status) {
+__device__ __forceinline__ bool poll_again(uint64_t& t0, int* status, unsigned long long limit_ns = kWaitLimitNs) {
   const uint64_t now = globaltimer_ns();
   if (t0 == 0) t0 = now;
-  if (now - t0 > kWaitLimitNs) {
+  if (now - t0 > limit_ns) {
     dev_flag(status, PCED_DEV_TIMEOUT);
     return false;
   }
@@ -789,7 +789,7 @@ __device__ __forceinline__ void produce_tiles(const CUtensorMap* kmap, const CUt
   uint32_t it = 0, st = 0, ph = 0;
   bool ok = true;
   while (ld.ok) {
-    if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status)) {
+    if (!mbar_wait(bar_empty + 8 * st, ph ^ 1u, a.status, a.wait_ns)) {
       ok = false;
       break;
     }
@@ -823,7 +823,7 @@ __device__ __forceinline__ void produce_tiles(const CUtensorMap* kmap, const CUt
 // them): the same order in every warp and CTA, so every user gets the same
 // value bit for bit.  Whole warp.
 __device__ __forceinline__ bool wait_inv_rms(const uint64_t* part, int n, uint32_t tag, int d, float eps, int lane,
-                                             int* status, float& inv) {
+                                             int* status, unsigned long long limit_ns, float& inv) {
   uint64_t t0 = 0;
   while (true) {
     float t = 0.f;
@@ -839,7 +839,7 @@ __device__ __forceinline__ bool wait_inv_rms(const uint64_t* part, int n, uint32
       inv = 1.0f / sqrtf(t / (float)d + eps);
       return true;
     }
-    if (!poll_again(t0, status)) return false;
+    if (!poll_again(t0, status, limit_ns)) return false;
   }
 }
 
@@ -1096,7 +1096,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         }
         const uint32_t slot = p & 1u, u = p >> 1;
         ++p;
-        if (u > 0 && !mbar_wait(bar_qempty + 8 * slot, (u - 1u) & 1u, a.status)) {
+        if (u > 0 && !mbar_wait(bar_qempty + 8 * slot, (u - 1u) & 1u, a.status, a.wait_ns)) {
           ok = false;
           break;
         }
@@ -1145,7 +1145,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
               v[j][3] = tv_value(w3);
             }
             if (__all_sync(0xffffffffu, good)) break;
-            if (!poll_again(t0, a.status)) {
+            if (!poll_again(t0, a.status, a.wait_ns)) {
               ok = false;
               break;
             }
@@ -1210,7 +1210,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
               }
             }
             if (__all_sync(0xffffffffu, good)) break;
-            if (!poll_again(t0, a.status)) {
+            if (!poll_again(t0, a.status, a.wait_ns)) {
               ok = false;
               break;
             }
@@ -1259,7 +1259,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     // end marker for the consumers
     if (ok) {
       const uint32_t slot = p & 1u, u = p >> 1;
-      if (u == 0 || mbar_wait(bar_qempty + 8 * slot, (u - 1u) & 1u, a.status)) {
+      if (u == 0 || mbar_wait(bar_qempty + 8 * slot, (u - 1u) & 1u, a.status, a.wait_ns)) {
         if (lane == 0) {
           PieceDesc* dsc = reinterpret_cast<PieceDesc*>(gbase + SL.qbuf + slot * SL.qslot + SL.qdesc);
           dsc->end = 1;
@@ -1283,7 +1283,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
   for (;;) {
     const uint32_t slot = p & 1u, u = p >> 1;
     ++p;
-    if (!mbar_wait(bar_qfull + 8 * slot, u & 1u, a.status)) {
+    if (!mbar_wait(bar_qfull + 8 * slot, u & 1u, a.status, a.wait_ns)) {
       ok = false;
       break;
     }
@@ -1310,11 +1310,11 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     for (int32_t kt = pc.k0; kt < pc.k1; kt += ATT_BLOCK_N, ++it, cst = cst + 1 == NST ? (++cuse, 0u) : cst + 1) {
       if ((int)(it & 1u) != wg) continue;
       const uint32_t use = cuse, st = cst, ph = use & 1u;
-      if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status)) {
+      if (use > 0 && !mbar_wait(bar_empty + 8 * st, (use - 1u) & 1u, a.status, a.wait_ns)) {
         ok = false;
         break;
       }
-      if (!mbar_wait(bar_full + 8 * st, ph, a.status)) {
+      if (!mbar_wait(bar_full + 8 * st, ph, a.status, a.wait_ns)) {
         ok = false;
         break;
       }
@@ -1353,7 +1353,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     }
     // combine the eight warps' partials through a double-buffered slot;
     // afterwards thread tid < G*D/4 owns outputs idx0..idx0+3 (head hh)
-    if (u > 0 && !mbar_wait(bar_pempty + 8 * slot, (u - 1u) & 1u, a.status)) {
+    if (u > 0 && !mbar_wait(bar_pempty + 8 * slot, (u - 1u) & 1u, a.status, a.wait_ns)) {
       ok = false;
       break;
     }
@@ -1391,7 +1391,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(bar_pfull + 8 * slot);
-    if (!mbar_wait(bar_pfull + 8 * slot, u & 1u, a.status)) {
+    if (!mbar_wait(bar_pfull + 8 * slot, u & 1u, a.status, a.wait_ns)) {
       ok = false;
       break;
     }
@@ -1471,7 +1471,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           lv[q] = tv_value(wl);
         }
         if (__all_sync(0xffffffffu, good)) break;
-        if (!poll_again(t0, a.status)) {
+        if (!poll_again(t0, a.status, a.wait_ns)) {
           ok = false;
           break;
         }
@@ -1533,7 +1533,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
         if (part_cta(pa, gp.P[gi], align) != (int64_t)blockIdx.x) continue;  // completed by another CTA
         const uint64_t* ps = a.part_ss + ((int64_t)nx * S + pc.s) * Hkv * ATT_CONSUMERS;
         float inv;
-        if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, ntag, d, a.rms_eps, lane, a.status, inv)) {
+        if (!wait_inv_rms(ps, Hkv * ATT_CONSUMERS, ntag, d, a.rms_eps, lane, a.status, a.wait_ns, inv)) {
           ok = false;
           break;
         }

@@ -127,6 +127,7 @@ struct StepAttArgs {
   int32_t* done_cnt;          // [1] CTAs finished (zero between launches)
   __nv_bfloat16* hidden;      // [S][d] final hidden state
   __nv_bfloat16* hidden_copy; // optional copy of `hidden`
+  unsigned long long wait_ns; // limit of the kernel's waits on other warps and CTAs (PCED_DEV_TIMEOUT after it)
   int* status;
 };
 constexpr int ATT_MAX_LAYERS = 1000;  // layer index fits the 10-bit field of the tags

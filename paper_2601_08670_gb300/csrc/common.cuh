@@ -61,20 +61,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 // Wait for the phase with the given parity to complete; gives up after
 // kWaitLimitNs, flags PCED_DEV_TIMEOUT and returns false.  The first test is
 // inlined: on the hot paths the phase has usually completed already.
-static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int* status) {
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int* status,
+                                                   unsigned long long limit_ns) {
   const uint64_t t0 = globaltimer_ns();
   while (true) {
 #pragma unroll 1
     for (int i = 0; i < 32; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
       dev_flag(status, PCED_DEV_TIMEOUT);
       return false;
     }
   }
 }
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status) {
-  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, status);
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, status, limit_ns);
 }
 
 // Barrier among a subset of a CTA's threads built on an mbarrier initialised

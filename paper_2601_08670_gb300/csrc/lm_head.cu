@@ -70,6 +70,19 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
   return true;
 }
 
+// Top-2 over tokens of (value, token) candidates whose token sets are
+// disjoint: (b1, t1) the best (larger value, then lower token), b2 the best
+// value at another token; merges the candidate set (r1, rt, r2) into it.
+__device__ __forceinline__ void top2_merge(float& b1, int& t1, float& b2, float r1, int rt, float r2) {
+  if (r1 > b1 || (r1 == b1 && rt < t1)) {
+    b2 = fmaxf(b1, r2);
+    b1 = r1;
+    t1 = rt;
+  } else {
+    b2 = fmaxf(b2, r1);
+  }
+}
+
 struct FMax {
   __device__ __forceinline__ float operator()(float x, float y) const { return fmaxf(x, y); }
 };
@@ -111,7 +124,7 @@ __device__ __forceinline__ float bfly_reduce(float (&x)[NB], int lane, Op op) {
 // amateur logit from its query's first column to the expert columns.
 template <int NB>
 __device__ __forceinline__ void epi_block(const LmArgs& a, uint32_t taddr, int c0, int v, bool valid, int lane,
-                                          int q, float* bc, float2* wst, float2* wag, const float* sbeta,
+                                          int q, float* bc, float2* wst, float2* wag, float* wu2, const float* sbeta,
                                           float& z_am) {
   const int S = a.S, S_pad = a.S_pad, n1 = a.N + 1;
   float z[NB], t[NB];
@@ -159,10 +172,14 @@ __device__ __forceinline__ void epi_block(const LmArgs& a, uint32_t taddr, int c
     for (int i = 0; i < NB; ++i) {
       const unsigned hit = __ballot_sync(0xffffffffu, u[i] == bc[32 + i]);
       if (li == i) mine = hit;
+      // the runner-up of the column: every row but the (lowest) one holding the maximum
+      t[i] = hit && lane == __ffs(hit) - 1 ? -INFINITY : u[i];
     }
+    const float u2 = bfly_reduce<NB>(t, lane, FMax());
     if (lane < NB && mycol < S && mycol % n1 != 0) {
       const int r = mine ? __ffs(mine) - 1 : 0;
       wag[q * S_pad + mycol] = make_float2(um, __int_as_float(v - lane + r));
+      wu2[q * S_pad + mycol] = u2;
     }
   }
   __syncwarp();
@@ -206,6 +223,7 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
   int32_t* acc_tile = tring + LM_TRING;                        // [2] tile of each accumulator, MMA warp -> epilogue
   float2* wst = reinterpret_cast<float2*>(gbase + (bar_drain + 8 - base) + 96);  // [4][S_pad] per-warp stats
   float2* wag = wst + 4 * S_pad;                                                  // [4][S_pad] per-warp argmax
+  float* wu2 = reinterpret_cast<float*>(wag + 4 * S_pad);                         // [4][S_pad] per-warp runner-up
   float* sbeta = reinterpret_cast<float*>(wag + 6 * S_pad);  // [nbeta]
   float* bc = sbeta + ((a.nbeta + 3) & ~3);               // [8][64] per-warp column broadcast
 
@@ -402,9 +420,9 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       for (int kb = kb0; kb < kb1; ++kb) {
         const int c0 = 32 * kb;
         if (c0 + 32 <= S_pad)
-          epi_block<32>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, sbeta, z_am);
+          epi_block<32>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, sbeta, z_am);
         else
-          epi_block<16>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, sbeta, z_am);
+          epi_block<16>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, sbeta, z_am);
       }
       tc_fence_before();
       mbar_arrive(bar_tempty + 8 * buf);
@@ -421,14 +439,15 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
         }
         a.rec_stats[(int64_t)col * ntiles + tile] = make_float2(cm, cs);
         if (a.mode == 1 && col % n1 != 0) {
-          float bu = -INFINITY;
+          float bu = -INFINITY, b2 = -INFINITY;
           int bv = 0x7fffffff;
 #pragma unroll
           for (int qq = 0; qq < 4; ++qq) {
             const float2 r = wag[qq * S_pad + col];
-            argmax_merge(bu, bv, r.x, __float_as_int(r.y));
+            top2_merge(bu, bv, b2, r.x, __float_as_int(r.y), wu2[qq * S_pad + col]);
           }
           a.rec_arg[(int64_t)col * ntiles + tile] = make_float2(bu, __int_as_float(bv));
+          a.rec_u2[(int64_t)col * ntiles + tile] = b2;
         }
       }
       if (!bar_sync_bounded(bar_epi, ephase, a.status)) break;
@@ -468,7 +487,7 @@ cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, con
 // grid (chunks, S): every CTA of row s forms lse[s] from the row's tile
 // records (the same fixed order in each) and turns its chunk of logits into
 // log-probabilities in place; chunk 0 stores lse.
-constexpr int LSE_CHUNK = 16384;
+constexpr int LSE_CHUNK = 8192;  // (144 CTAs for 9 rows of 128K entries)
 
 __global__ void __launch_bounds__(256) lm_lse_finalize_kernel(float* logits, const float2* rec_stats, float* lse,
                                                               int32_t V, int32_t nrec) {
@@ -552,29 +571,41 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
   if (a.pdl) pdl_wait();  // the LM head's records are complete and visible
   if (j == 0 && b == 0 && tid == 0 && a.tile_ctr) *a.tile_ctr = 0;  // the next LM head claims its tiles from 0
   __shared__ float2 red[SEL_R_THREADS / 32];
-  __shared__ float sv[SEL_R_THREADS / 32];
+  __shared__ float sv[SEL_R_THREADS / 32], sv2[SEL_R_THREADS / 32];
   __shared__ int si[SEL_R_THREADS / 32];
   __shared__ int last;
+  __shared__ int pick[2];   // token, expert of the query (last CTA)
+  __shared__ float zy[LM_MAX_N1];  // z_s(token) of the query's rows (last CTA)
+  __shared__ uint4 wrow[LM_MAX_D / 8];  // W[token] (last CTA)
   float L = 0.f;
   lse_block(a.rec_stats + (int64_t)s * T, T, tid, red, L);
   if (j > 0) {
+    // the row's best u_k and its token, and the best u_k at any other token
     const float2* rec = a.rec_arg + (int64_t)s * T;
-    float bu = -INFINITY;
+    const float* rec2 = a.rec_u2 + (int64_t)s * T;
+    float bu = -INFINITY, b2 = -INFINITY;
     int bv = 0x7fffffff;
     for (int t = tid; t < T; t += SEL_R_THREADS) {
       const float2 r = rec[t];
-      argmax_merge(bu, bv, r.x, __float_as_int(r.y));
+      top2_merge(bu, bv, b2, r.x, __float_as_int(r.y), rec2[t]);
     }
-    warp_argmax(bu, bv);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float r1 = __shfl_xor_sync(0xffffffffu, bu, o), r2 = __shfl_xor_sync(0xffffffffu, b2, o);
+      const int rt = __shfl_xor_sync(0xffffffffu, bv, o);
+      top2_merge(bu, bv, b2, r1, rt, r2);
+    }
     if (lane == 0) {
       sv[warp] = bu;
       si[warp] = bv;
+      sv2[warp] = b2;
     }
     __syncthreads();
     if (tid == 0) {
-      for (int w = 1; w < SEL_R_THREADS / 32; ++w) argmax_merge(bu, bv, sv[w], si[w]);
+      for (int w = 1; w < SEL_R_THREADS / 32; ++w) top2_merge(bu, bv, b2, sv[w], si[w], sv2[w]);
       a.sel_u[s] = bu;
       a.sel_tok[s] = bv;
+      a.sel_u2[s] = b2;
     }
   }
   if (tid == 0) {
@@ -586,33 +617,89 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
   __syncthreads();
   if (!last) return;
   __threadfence();  // the other rows' results of query b are visible
-  if (warp != 0) return;
   const float L0 = __ldcg(a.sel_L + b * n1);
   float bs = -INFINITY;
   int bt = 0x7fffffff, bk = 0x7fffffff;
-  for (int k = lane; k < N; k += 32) {
-    const int sk = b * n1 + 1 + k;
-    const float btk = a.beta[b * N + k];
-    const float rr = fminf(fmaxf(a.r[b * N + k], 1e-8f), 1.0f);
-    const float c = (a.raw_logits ? 0.f : -(1.f + btk) * __ldcg(a.sel_L + sk) + btk * L0) + a.gamma * logf(rr);
-    const float sc = __ldcg(a.sel_u + sk) + c;
-    const int tk = __ldcg(a.sel_tok + sk);
-    if (sc > bs || (sc == bs && (tk < bt || (tk == bt && k < bk)))) {
-      bs = sc;
-      bt = tk;
-      bk = k;
+  if (warp == 0) {
+    for (int k = lane; k < N; k += 32) {
+      const int sk = b * n1 + 1 + k;
+      const float btk = a.beta[b * N + k];
+      const float rr = fminf(fmaxf(a.r[b * N + k], 1e-8f), 1.0f);
+      const float c = (a.raw_logits ? 0.f : -(1.f + btk) * __ldcg(a.sel_L + sk) + btk * L0) + a.gamma * logf(rr);
+      const float sc = __ldcg(a.sel_u + sk) + c;
+      const int tk = __ldcg(a.sel_tok + sk);
+      if (sc > bs || (sc == bs && (tk < bt || (tk == bt && k < bk)))) {
+        bs = sc;
+        bt = tk;
+        bk = k;
+      }
     }
-  }
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float s2 = __shfl_xor_sync(0xffffffffu, bs, o);
-    const int t2 = __shfl_xor_sync(0xffffffffu, bt, o), k2 = __shfl_xor_sync(0xffffffffu, bk, o);
-    if (s2 > bs || (s2 == bs && (t2 < bt || (t2 == bt && k2 < bk)))) {
-      bs = s2;
-      bt = t2;
-      bk = k2;
+    for (int o = 16; o > 0; o >>= 1) {
+      const float s2 = __shfl_xor_sync(0xffffffffu, bs, o);
+      const int t2 = __shfl_xor_sync(0xffffffffu, bt, o), k2 = __shfl_xor_sync(0xffffffffu, bk, o);
+      if (s2 > bs || (s2 == bs && (t2 < bt || (t2 == bt && k2 < bk)))) {
+        bs = s2;
+        bt = t2;
+        bk = k2;
+      }
+    }
+    if (lane == 0) {
+      pick[0] = bt;
+      pick[1] = bk;
     }
   }
+  float2 gaps = make_float2(INFINITY, INFINITY);
+  if (a.gap_trace) {
+    __syncthreads();
+    const int y = pick[0] >= 0 && pick[0] < a.V ? pick[0] : 0;
+    // W[y] into shared memory with 16-byte loads (one round trip), then
+    // z_s(y) = h_s . W[y] for the query's rows, one warp per row, fp32 sums
+    // of independent 8-element chunks
+    const int nv = a.d / 8;  // 16-byte chunks of a row (d % 64 == 0)
+    const uint4* wy = reinterpret_cast<const uint4*>(a.w_unembed + (int64_t)y * a.d);
+    for (int i = tid; i < nv; i += SEL_R_THREADS) wrow[i] = __ldg(wy + i);
+    __syncthreads();
+    for (int jr = warp; jr < n1; jr += SEL_R_THREADS / 32) {
+      const uint4* hr = reinterpret_cast<const uint4*>(a.hidden + (int64_t)(b * n1 + jr) * a.d);
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+      for (int i = lane; i < nv; i += 32) {
+        const uint4 hv = __ldcg(hr + i), wv = wrow[i];
+        const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w}, ww[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          acc[q] = fmaf(bf16_lo(hw[q]), bf16_lo(ww[q]), acc[q]);
+          acc[q] = fmaf(bf16_hi(hw[q]), bf16_hi(ww[q]), acc[q]);
+        }
+      }
+      const float t = warp_sum((acc[0] + acc[1]) + (acc[2] + acc[3]));
+      if (lane == 0) zy[jr] = t;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      // token gap: the best score at another token, over all experts
+      float other = -INFINITY, se_best = -INFINITY, se_other = -INFINITY;
+      for (int k = lane; k < N; k += 32) {
+        const int sk = b * n1 + 1 + k;
+        const float btk = a.beta[b * N + k];
+        const float rr = fminf(fmaxf(a.r[b * N + k], 1e-8f), 1.0f);
+        const float Lk = __ldcg(a.sel_L + sk);
+        const float c = (a.raw_logits ? 0.f : -(1.f + btk) * Lk + btk * L0) + a.gamma * logf(rr);
+        const float cand = __ldcg(a.sel_tok + sk) != bt ? __ldcg(a.sel_u + sk) : __ldcg(a.sel_u2 + sk);
+        other = fmaxf(other, cand + c);
+        // expert gap: every expert's score at the chosen token, from the recomputed logits
+        const float se = (1.f + btk) * zy[1 + k] - btk * zy[0] + c;
+        if (k == bk) se_best = se;
+        else se_other = fmaxf(se_other, se);
+      }
+      other = warp_max(other);
+      se_best = warp_max(se_best);
+      se_other = warp_max(se_other);
+      gaps = make_float2(bs - other, se_best - se_other);
+    }
+  }
+  if (warp != 0) return;
   if (lane == 0) {
     a.qdone[b] = 0;
     if (a.token) a.token[b] = bt;
@@ -624,6 +711,7 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
         a.history[(int64_t)b * a.max_steps + t] = bt;
         if (a.expert_trace) a.expert_trace[(int64_t)b * a.max_steps + t] = bk + 1;
         if (a.score_trace) a.score_trace[(int64_t)b * a.max_steps + t] = bs;
+        if (a.gap_trace) a.gap_trace[(int64_t)b * a.max_steps + t] = gaps;
       } else {
         dev_flag(a.status, PCED_DEV_STEP_LIMIT);
       }

@@ -10,6 +10,7 @@ constexpr int LM_THREADS = 64 + LM_EPI_THREADS;  // warp 0 TMA, warp 1 MMA + TME
 constexpr int LM_TILE_V = 128;   // vocabulary rows per tile (UMMA M)
 constexpr int LM_TILE_K = 64;    // hidden elements per stage (one 128-byte swizzle row)
 constexpr int LM_MAX_S = 512;
+constexpr int LM_MAX_D = 8192;   // hidden size of the fused step (the selection stages one W row)
 constexpr int LM_MAX_N1 = 256;   // experts + amateur per query in the selection kernels
 constexpr int LM_TRING = 16;     // claimed-tile ring between the TMA and MMA warps (> stages + 2 tiles in flight)
 
@@ -28,6 +29,7 @@ struct LmArgs {
   float* logits;      // mode 0
   float2* rec_stats;  // [S][ntiles] (max z, sum exp(z - max)) of each vocabulary tile
   float2* rec_arg;    // [S][ntiles] (max u, argmax v as int bits) for expert columns, mode 1
+  float* rec_u2;      // [S][ntiles] the tile's second-largest u (another token), mode 1
   int* tile_ctr;      // tiles claimed so far (zero at launch)
   const float* beta;  // [B][N]
   int pdl;            // launched as a programmatic dependent of the kernel that writes H
@@ -44,7 +46,9 @@ cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float
 struct SelectArgs {
   const float2* rec_stats;
   const float2* rec_arg;
+  const float* rec_u2;
   int32_t B, N, nrec;  // records per row (the LM head's vocabulary tiles)
+  int32_t V;
   int* tile_ctr;       // optional: the LM head's tile counter, reset here for its next launch
   const float* beta;
   const float* r;
@@ -65,6 +69,14 @@ struct SelectArgs {
   float* sel_L;       // [S] log-sum-exp of each row
   float* sel_u;       // [S] best u_k of each expert row
   int32_t* sel_tok;   // [S] its token
+  float* sel_u2;      // [S] the row's best u_k at another token
+  // near-tie margins of the choice (optional): gap_trace[b][t] = (token gap,
+  // expert gap); the expert gap recomputes z_s(y) = h_s . W[y] for the
+  // query's rows
+  float2* gap_trace;
+  const __nv_bfloat16* hidden;     // [S][d]
+  const __nv_bfloat16* w_unembed;  // [V][d]
+  int32_t d;
   int32_t* qdone;     // [B] rows of the query finished
   int pdl;            // launched as a programmatic dependent of the LM head
   int raw_logits;     // s_k of Eq. 2 are the raw logits: c_k = gamma log r_k alone

@@ -33,6 +33,9 @@ struct StepLayout {
   void* ada;              // scratch of the beta kernel (counters zero between uses)
   float2* agg_part;       // MoE / PoE: per (query, expert, chunk) statistics
   float2* agg_best;       // MoE / PoE: per (query, chunk) best
+  float* agg_best2;       // MoE / PoE: per (query, chunk) best at another token
+  int32_t* agg_kdone;     // MoE / PoE: chunks finished per (query, expert)
+  float* agg_lse;         // MoE / PoE: per (query, expert) log-sum-exp of the contrastive scores
   int32_t* agg_qdone;     // MoE / PoE: chunks finished per query
   uint64_t* part_ss;
   uint64_t* resid;
@@ -41,6 +44,8 @@ struct StepLayout {
   __nv_bfloat16* h;
   float2* lm_stats;
   float2* lm_arg;
+  float* lm_u2;
+  float* sel_u2;
   size_t bytes;
 };
 
@@ -63,6 +68,8 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   L.h = c.take<__nv_bfloat16>((size_t)S * d);
   L.lm_stats = c.take<float2>((size_t)(S * ntiles));
   L.lm_arg = c.take<float2>((size_t)(S * ntiles));
+  L.lm_u2 = c.take<float>((size_t)(S * ntiles));
+  L.sel_u2 = c.take<float>((size_t)S);
   L.lm_tile_ctr = c.take<int32_t>(1);
   L.sel_qdone = c.take<int32_t>((size_t)dm->B);
   L.sel_L = c.take<float>((size_t)S);
@@ -72,6 +79,9 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   L.ada = c.take<char>(adacad_scratch_bytes(dm->B, dm->N, dm->V));
   L.agg_part = c.take<float2>((size_t)dm->B * dm->N * agg_chunks(dm->V));
   L.agg_best = c.take<float2>((size_t)dm->B * agg_chunks(dm->V));
+  L.agg_best2 = c.take<float>((size_t)dm->B * agg_chunks(dm->V));
+  L.agg_kdone = c.take<int32_t>((size_t)dm->B * dm->N);
+  L.agg_lse = c.take<float>((size_t)dm->B * dm->N);
   L.agg_qdone = c.take<int32_t>((size_t)dm->B);
   L.bytes = c.used() + 4 * (4096 - 256);  // room for the 4 KB alignment of four arrays
   return L;
@@ -106,6 +116,8 @@ static int32_t step_plan(const pced_step_args* p, const char** kinds) {
   if (agg) {
     add("agg_partials");
     add("agg_select");
+  } else if (dyn) {
+    add("agg_select");  // Eq. 3 on the log-probabilities written for beta
   } else {
     add("lm_head");  // fused log-softmax statistics and contrastive tile maxima
     add("select");
@@ -247,6 +259,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   at.hidden = W.h;
   at.hidden_copy = (__nv_bfloat16*)p->hidden_out;
   at.status = W.status;
+  at.wait_ns = p->wait_limit_ns ? p->wait_limit_ns : kWaitLimitNs;
   e = att_step_launch(dm.D, kmap, vmap, at, att_grid(p->total_cap * dm.Hkv), s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "attention launch");
@@ -276,7 +289,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     lz.rec_stats = W.lm_stats;
     lz.tile_ctr = W.lm_tile_ctr;
     lz.status = W.status;
-    lz.pdl = 0;
+    lz.pdl = timed ? 0 : 1;  // streams weights while the attention kernel finishes
     e = lm_head_launch(wmap, hmap, g, lz, s);
     if (e == cudaSuccess) e = mark();
     if (e == cudaSuccess) e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
@@ -289,7 +302,9 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     if (e != cudaSuccess) return cuda_status(e, "log-probability launches");
     if (dyn) beta = p->beta_out;
   }
-  if (agg) {
+  if (agg || dyn) {
+    // MoE / PoE, or Eq. 3 on the log-probabilities the first step of a
+    // dynamic-beta decode has written anyway (no second LM-head pass)
     AggArgs ag = {};
     ag.lp = W.lp;
     ag.beta = beta;
@@ -299,9 +314,15 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ag.N = dm.N;
     ag.V = dm.V;
     ag.rule = p->aggregation;
+    ag.gamma = p->gamma;
+    ag.raw_logits = p->score_mode == PCED_SCORE_LOGIT;
     ag.nchunks = agg_chunks(dm.V);
     ag.part = W.agg_part;
     ag.best = W.agg_best;
+    ag.best2 = W.agg_best2;
+    ag.kdone = W.agg_kdone;
+    ag.lse_k = W.agg_lse;
+    ag.gap_trace = reinterpret_cast<float2*>(p->gap_trace);
     ag.qdone = W.agg_qdone;
     ag.tile_ctr = W.lm_tile_ctr;
     ag.lse_out = p->lse_out;
@@ -312,8 +333,10 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ag.max_steps = p->max_steps;
     ag.done_counter = W.done_counter;
     ag.status = W.status;
-    e = agg_partials_launch(ag, s);
-    if (e == cudaSuccess) e = mark();
+    if (agg) {
+      e = agg_partials_launch(ag, s);
+      if (e == cudaSuccess) e = mark();
+    }
     if (e == cudaSuccess) e = agg_select_launch(ag, s);
     if (e == cudaSuccess) e = mark();
     if (e != cudaSuccess) return cuda_status(e, "aggregation launches");
@@ -338,6 +361,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.tmem_cols = g.tmem_cols;
   la.rec_stats = W.lm_stats;
   la.rec_arg = W.lm_arg;
+  la.rec_u2 = W.lm_u2;
   la.tile_ctr = W.lm_tile_ctr;
   la.beta = beta;
   la.status = W.status;
@@ -349,6 +373,13 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   SelectArgs sa = {};
   sa.rec_stats = W.lm_stats;
   sa.rec_arg = W.lm_arg;
+  sa.rec_u2 = W.lm_u2;
+  sa.V = dm.V;
+  sa.sel_u2 = W.sel_u2;
+  sa.gap_trace = reinterpret_cast<float2*>(p->gap_trace);
+  sa.hidden = W.h;
+  sa.w_unembed = (const __nv_bfloat16*)p->w_unembed;
+  sa.d = d;
   sa.B = dm.B;
   sa.N = dm.N;
   sa.nrec = g.ntiles;

@@ -150,7 +150,7 @@ def test_launch_count_and_kinds_follow_the_mode(L):
     import paper_2601_08670_gb300 as pced
     assert pced.step_launch_kinds(step_args(pced)) == ["attention", "lm_head", "select"]
     assert pced.step_launch_kinds(step_args(pced, beta_from_step=1)) == [
-        "attention", "lm_head", "lse_finalize", "adacad_beta", "lm_head", "select"]
+        "attention", "lm_head", "lse_finalize", "adacad_beta", "agg_select"]
     for rule in (pced.AGG_MOE, pced.AGG_POE):
         assert pced.step_launch_kinds(step_args(pced, aggregation=rule)) == [
             "attention", "lm_head", "lse_finalize", "agg_partials", "agg_select"]
