@@ -308,6 +308,19 @@ typedef struct pced_step_args {
    * results.  0: 2 s.  A CTA still waits for its own tile copies in flight
    * (up to 2 s) before it exits. */
   uint64_t wait_limit_ns;
+  /* Expert-partitioned step (the experts of a query spread over several
+   * GPUs; each holds the amateur, W_U and its own experts): when key_out is
+   * not NULL the call computes the best choice of its experts per query as a
+   * packed key (pced_select_key, with expert index expert_base + k for its
+   * k-th expert) into key_out [B] (device int64) and appends nothing: t,
+   * history and the traces stay as they were (gap_trace is not written).
+   * After a max-reduction of the keys over the GPUs, pced_step_commit
+   * appends the common token on each.  Requires the max rule of Eq. 3
+   * (aggregation PCED_AGG_MAX), V <= 2^20 and expert_base + N <= 4096 (else
+   * PCED_ERR_UNSUPPORTED).  The cache appends of this step are made either
+   * way (every GPU appends the same input token). */
+  int32_t expert_base;
+  int64_t* key_out;
 } pced_step_args;
 
 #define PCED_SCORE_LOGPROB 0
@@ -315,6 +328,27 @@ typedef struct pced_step_args {
 #define PCED_AGG_MAX 0
 #define PCED_AGG_MOE 1
 #define PCED_AGG_POE 2
+
+/* ------------------------------------------------------------------------
+ * The choice of Eq. 3 as one int64 whose signed order is Eq. 3's order: the
+ * higher score first, then the lower token id, then the lower expert index
+ * (host; the device packs the same bits).  token in [0, 2^20), expert
+ * (1-based, global) in [1, 4096].  The maximum of the keys of disjoint sets
+ * of a query's experts is the key of the choice over their union (Eq. 3
+ * couples experts only through this max), so an all-reduce-max of int64
+ * (NCCL, gloo, torch.maximum) is the only exchange an expert-partitioned
+ * step needs.  Unpack returns the fp32 score exactly; NULL outputs are skipped.
+ * ------------------------------------------------------------------------ */
+int64_t pced_select_key(float score, int32_t token, int32_t expert);
+void pced_select_key_unpack(int64_t key, float* score, int32_t* token, int32_t* expert);
+
+/* Append the reduced choices of an expert-partitioned step: for each query
+ * b, history[b][t] = token, expert_trace / score_trace (may be NULL) from
+ * keys[b] (device int64 [B]), then t += 1 (step, device int32).  A t outside
+ * [0, max_steps) writes nothing and sets PCED_DEV_STEP_LIMIT in *status
+ * (device, may be NULL).  One launch on `stream`. */
+pced_status pced_step_commit(const int64_t* keys, int32_t B, int32_t* step, int32_t* history, int32_t* expert_trace,
+                             float* score_trace, int32_t max_steps, int* status, void* stream);
 
 size_t pced_step_workspace_size(const pced_dims* dims);
 pced_status pced_step(const pced_step_args* args, void* stream);

@@ -49,7 +49,7 @@ class StepArgs(ctypes.Structure):
                 ("n_stage_events", ctypes.c_int32), ("beta_from_step", ctypes.c_int32), ("beta_out", ctypes.c_void_p),
                 ("block_table", ctypes.c_void_p), ("block_rows", ctypes.c_int32), ("max_blocks", ctypes.c_int32),
                 ("rope_theta", ctypes.c_float), ("score_mode", ctypes.c_int32), ("aggregation", ctypes.c_int32),
-                ("wait_limit_ns", ctypes.c_uint64)]
+                ("wait_limit_ns", ctypes.c_uint64), ("expert_base", ctypes.c_int32), ("key_out", ctypes.c_void_p)]
 
 
 _lib = None
@@ -95,6 +95,12 @@ def lib(path: str = LIB_PATH):
         L.pced_step_launch_count.restype = I32
         L.pced_step_launch_kind.argtypes = [ctypes.POINTER(StepArgs), I32]
         L.pced_step_launch_kind.restype = ctypes.c_char_p
+        L.pced_select_key.argtypes = [F, I32, I32]
+        L.pced_select_key.restype = I64
+        L.pced_select_key_unpack.argtypes = [I64, ctypes.POINTER(F), ctypes.POINTER(I32), ctypes.POINTER(I32)]
+        L.pced_select_key_unpack.restype = None
+        L.pced_step_commit.argtypes = [P, I32, P, P, P, P, I32, P, P]
+        L.pced_step_commit.restype = I32
         _lib = L
     return _lib
 
@@ -252,6 +258,19 @@ def step_launch_count(args) -> int:
     return int(lib().pced_step_launch_count(ctypes.byref(args)))
 
 
+def select_key(score: float, token: int, expert: int) -> int:
+    """Eq. 3's choice as an int64 whose signed order is Eq. 3's order
+    (pced_select_key)."""
+    return int(lib().pced_select_key(float(score), int(token), int(expert)))
+
+
+def select_key_unpack(key: int):
+    """(fp32 score, token, expert) of a packed key."""
+    s, t, e = ctypes.c_float(), ctypes.c_int32(), ctypes.c_int32()
+    lib().pced_select_key_unpack(int(key), ctypes.byref(s), ctypes.byref(t), ctypes.byref(e))
+    return s.value, t.value, e.value
+
+
 def step_launch_kinds(args) -> list:
     return [lib().pced_step_launch_kind(ctypes.byref(args), i).decode() for i in range(step_launch_count(args))]
 
@@ -309,6 +328,27 @@ class Decoder:
     def step(self, stream=None):
         _check(lib().pced_step(ctypes.byref(self.args), _stream(stream)), "pced_step")
         self.args.beta_from_step = 0
+
+    def step_partial(self, keys, expert_base: int, stream=None):
+        """Expert-partitioned step: this decoder's experts are global experts
+        expert_base + 1 .. expert_base + N; writes their best choice per query
+        as packed keys (int64 [B] device tensor `keys`) and appends nothing.
+        Reduce the keys with a max over the decoders (NCCL / gloo all-reduce,
+        torch.maximum), then call commit()."""
+        assert keys.dtype == torch.int64 and keys.is_contiguous() and keys.numel() >= self.dm.B
+        self.args.key_out = _ptr(keys)
+        self.args.expert_base = int(expert_base)
+        try:
+            self.step(stream)
+        finally:
+            self.args.key_out = None
+            self.args.expert_base = 0
+
+    def commit(self, keys, stream=None):
+        """Append the reduced choices (int64 [B] device keys) and advance t."""
+        _check(lib().pced_step_commit(_ptr(keys), self.dm.B, _ptr(self.step_t), _ptr(self.history),
+                                      _ptr(self.expert_trace), _ptr(self.score_trace), self.max_steps,
+                                      _ptr(self.ws), _stream(stream)), "pced_step_commit")
 
     def set_stage_events(self, events):
         """Record one torch.cuda.Event before and after every launch of each

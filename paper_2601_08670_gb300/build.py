@@ -20,8 +20,7 @@ ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-I", os.path.join(ROOT, "include")]
 SOURCES = ["attention.cu", "attention_noalloc.cu", "lm_head.cu", "select.cu", "adacad.cu", "aggregate.cu", "relevance.cu",
-           "step.cu",
-           "host.cu"]
+           "step.cu", "partition.cu", "host.cu"]
 
 
 def _deps():

@@ -17,6 +17,7 @@
 #include <math.h>
 
 #include "aggregate.cuh"
+#include "select_key.cuh"
 
 namespace pced {
 
@@ -211,6 +212,10 @@ __global__ void __launch_bounds__(AGG_THREADS) agg_select_kernel(AggArgs a) {
   a.qdone[b] = 0;
   if (a.lse_out)
     for (int j = 0; j < n1; ++j) a.lse_out[b * n1 + j] = a.lse[b * n1 + j];
+  if (a.key_out) {  // expert-partitioned step (rule 0): the reduction and the append come after
+    a.key_out[b] = select_key(sv, st, a.expert_base + bk + 1);
+    return;
+  }
   if (a.token) a.token[b] = st;
   if (a.expert) a.expert[b] = bk + 1;
   if (a.score) a.score[b] = sv;

@@ -30,6 +30,8 @@ struct AggArgs {
   int32_t* expert_trace;
   float* score_trace;
   float2* gap_trace;    // optional [B][max_steps]: (token gap, attribution margin)
+  int64_t* key_out;     // rule 0, expert-partitioned step: packed choices [B], nothing appended
+  int32_t expert_base;
   int32_t max_steps;
   int32_t* done_counter;
   int* status;

@@ -22,6 +22,7 @@
 #include <stdlib.h>
 
 #include "lm_head.cuh"
+#include "select_key.cuh"
 
 namespace pced {
 
@@ -650,7 +651,7 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
     }
   }
   float2 gaps = make_float2(INFINITY, INFINITY);
-  if (a.gap_trace) {
+  if (a.gap_trace && !a.key_out) {
     __syncthreads();
     const int y = pick[0] >= 0 && pick[0] < a.V ? pick[0] : 0;
     // W[y] into shared memory with 16-byte loads (one round trip), then
@@ -700,6 +701,13 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
     }
   }
   if (warp != 0) return;
+  if (lane == 0 && a.key_out) {
+    // expert-partitioned step: this GPU's best, the reduction over GPUs and
+    // the append come after
+    a.qdone[b] = 0;
+    a.key_out[b] = select_key(bs, bt, a.expert_base + bk + 1);
+    return;
+  }
   if (lane == 0) {
     a.qdone[b] = 0;
     if (a.token) a.token[b] = bt;

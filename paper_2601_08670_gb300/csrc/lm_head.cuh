@@ -74,6 +74,8 @@ struct SelectArgs {
   // expert gap); the expert gap recomputes z_s(y) = h_s . W[y] for the
   // query's rows
   float2* gap_trace;
+  int64_t* key_out;   // expert-partitioned step: packed choices [B], nothing appended
+  int32_t expert_base;
   const __nv_bfloat16* hidden;     // [S][d]
   const __nv_bfloat16* w_unembed;  // [V][d]
   int32_t d;

@@ -16,6 +16,7 @@
 #include "aggregate.cuh"
 #include "attention.cuh"
 #include "lm_head.cuh"
+#include "select_key.cuh"
 
 namespace pced {
 
@@ -160,6 +161,10 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     return fail(PCED_ERR_INVALID_ARG, "pced_step: aggregation %d", p->aggregation);
   if (p->aggregation != PCED_AGG_MAX && dm.N > AGG_MAX_N)
     return fail(PCED_ERR_UNSUPPORTED, "pced_step: MoE / PoE take at most %d experts", AGG_MAX_N);
+  if (p->key_out && (p->aggregation != PCED_AGG_MAX || dm.V > KEY_MAX_TOKENS || p->expert_base < 0 ||
+                     p->expert_base + dm.N > KEY_MAX_EXPERTS))
+    return fail(PCED_ERR_UNSUPPORTED, "pced_step: expert-partitioned step needs the max rule, V <= 2^20 and "
+                                      "expert_base + N <= 4096");
   if (!(p->rope_theta >= 0.f) || !std::isfinite(p->rope_theta))
     return fail(PCED_ERR_INVALID_ARG, "pced_step: rope_theta must be finite and >= 0");
   int64_t num_blocks = 0;
@@ -322,7 +327,9 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ag.best2 = W.agg_best2;
     ag.kdone = W.agg_kdone;
     ag.lse_k = W.agg_lse;
-    ag.gap_trace = reinterpret_cast<float2*>(p->gap_trace);
+    ag.gap_trace = p->key_out ? nullptr : reinterpret_cast<float2*>(p->gap_trace);
+    ag.key_out = p->key_out;
+    ag.expert_base = p->expert_base;
     ag.qdone = W.agg_qdone;
     ag.tile_ctr = W.lm_tile_ctr;
     ag.lse_out = p->lse_out;
@@ -377,6 +384,8 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.V = dm.V;
   sa.sel_u2 = W.sel_u2;
   sa.gap_trace = reinterpret_cast<float2*>(p->gap_trace);
+  sa.key_out = p->key_out;
+  sa.expert_base = p->expert_base;
   sa.hidden = W.h;
   sa.w_unembed = (const __nv_bfloat16*)p->w_unembed;
   sa.d = d;

@@ -393,24 +393,41 @@ def host_normal_bf16(n: int, seed: int, sigma: float = 1.0) -> np.ndarray:
     return out
 
 
+def expert_part(w: Workload, e0: int, e1: int):
+    """The sequences of every query's amateur and contextual experts
+    [e0, e1) (0-based): the workload with N = e1 - e0, the global sequence
+    ids (query-major, amateur first) and the columns of beta / r."""
+    assert 0 <= e0 < e1 <= w.N
+    ids = np.array([b * (w.N + 1) + j for b in range(w.B) for j in [0] + list(range(1 + e0, 1 + e1))], np.int32)
+    return replace(w, N=e1 - e0), ids, slice(e0, e1)
+
+
 def device_inputs(w: Workload, device="cuda", extra_steps: int | None = None, stream=None,
-                  paged: int = 0) -> dict:
+                  paged: int = 0, part: tuple | None = None) -> dict:
     """All inputs of workload `w` as device tensors: caches with generated
     prefixes (zeros after), embedding, unembedding, lengths, layout tables,
     beta and r.  Generated on the device with the same bits as the host fills.
     paged = P > 0 stores the caches in the paged layout with P-row blocks
     (keys "block_table", "block_rows", "paged_layout"); the logical cache
-    contents are the same."""
+    contents are the same.  part = (e0, e1) keeps only the amateur and the
+    contextual experts [e0, e1) of every query (contents as in the full
+    workload; key "w" is the workload of the part)."""
     import torch
     stream = torch.cuda.current_stream() if stream is None else stream
     sp = stream.cuda_stream
-    bl = base_lengths(w)
+    full = w
+    if part is not None:
+        w, seq_ids, cols = expert_part(full, *part)
+        bl = base_lengths(full)[seq_ids]
+    else:
+        seq_ids, cols = np.arange(w.S, dtype=np.int32), slice(None)
+        bl = base_lengths(w)
     lay = paged_layout(w, bl, paged, extra_steps) if paged else cache_layout(w, bl, extra_steps)
     k = torch.zeros(lay.total_elems, dtype=torch.bfloat16, device=device)
     v = torch.zeros(lay.total_elems, dtype=torch.bfloat16, device=device)
     cap = torch.from_numpy(lay.cap).to(device)
     base = torch.from_numpy(bl).to(device)
-    ids = torch.arange(w.S, dtype=torch.int32, device=device)
+    ids = torch.from_numpy(seq_ids).to(device)
     extra = {}
     if paged:
         table = torch.from_numpy(lay.table).to(device)
@@ -430,5 +447,5 @@ def device_inputs(w: Workload, device="cuda", extra_steps: int | None = None, st
     dev_fill_matrix(w, T_EMBED, emb, sp)
     dev_fill_matrix(w, T_UNEMBED, wu, sp)
     return dict(k_cache=k, v_cache=v, kv_offset=kv_off, cap=cap, seq_len=base.clone(), base_len=bl, layout=lay,
-                embed=emb, w_unembed=wu, beta=torch.from_numpy(betas(w)).to(device),
-                r=torch.from_numpy(retrieval_scores(w)).to(device), **extra)
+                embed=emb, w_unembed=wu, beta=torch.from_numpy(np.ascontiguousarray(betas(full)[:, cols])).to(device),
+                r=torch.from_numpy(np.ascontiguousarray(retrieval_scores(full)[:, cols])).to(device), w=w, **extra)
