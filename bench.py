@@ -163,7 +163,7 @@ KERNEL_SOURCES = {
     "attention": ["paper_2601_08670_gb300/csrc/attention.cu", "paper_2601_08670_gb300/csrc/attention.cuh",
                    "paper_2601_08670_gb300/csrc/common.cuh"],
     "lm_head": ["paper_2601_08670_gb300/csrc/lm_head.cu", "paper_2601_08670_gb300/csrc/lm_head.cuh",
-                "paper_2601_08670_gb300/csrc/common.cuh"],
+                "paper_2601_08670_gb300/csrc/common.cuh", "paper_2601_08670_gb300/csrc/select_key.cuh"],
 }
 
 

@@ -10,6 +10,7 @@
 // the device, so one captured call replays as the next step.
 #include <cmath>
 #include <math.h>
+#include <nvtx3/nvToolsExt.h>
 #include <stdlib.h>
 
 #include "adacad.cuh"
@@ -87,6 +88,24 @@ static StepLayout step_layout(const pced_dims* dm, void* ws) {
   L.bytes = c.used() + 4 * (4096 - 256);  // room for the 4 KB alignment of four arrays
   return L;
 }
+
+// NVTX ranges on the host thread that enqueues a step, for timeline tools:
+// one over the call and, inside it, one per launch named by its kind (the
+// names of pced_step_launch_kind).  Without a tool attached they cost a
+// branch each.
+struct StepRanges {
+  bool open = false;
+  StepRanges() { nvtxRangePushA("pced_step"); }
+  void next(const char* kind) {
+    if (open) nvtxRangePop();
+    nvtxRangePushA(kind);
+    open = true;
+  }
+  ~StepRanges() {
+    if (open) nvtxRangePop();
+    nvtxRangePop();
+  }
+};
 
 }  // namespace pced
 
@@ -210,6 +229,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     return cap_status == cudaStreamCaptureStatusActive ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal)
                                                        : cudaEventRecord(ev, s);
   };
+  StepRanges ranges;
   cudaError_t e = mark();
   if (e != cudaSuccess) return cuda_status(e, "stage event");
 
@@ -265,6 +285,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   at.hidden_copy = (__nv_bfloat16*)p->hidden_out;
   at.status = W.status;
   at.wait_ns = p->wait_limit_ns ? p->wait_limit_ns : kWaitLimitNs;
+  ranges.next("attention");
   e = att_step_launch(dm.D, kmap, vmap, at, att_grid(p->total_cap * dm.Hkv), s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "attention launch");
@@ -295,12 +316,15 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     lz.tile_ctr = W.lm_tile_ctr;
     lz.status = W.status;
     lz.pdl = timed ? 0 : 1;  // streams weights while the attention kernel finishes
+    ranges.next("lm_head");
     e = lm_head_launch(wmap, hmap, g, lz, s);
     if (e == cudaSuccess) e = mark();
+    if (e == cudaSuccess) ranges.next("lse_finalize");
     if (e == cudaSuccess) e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
     if (e == cudaSuccess) e = mark();
     // the JSD kernel also re-arms the LM head's tile counter for the fused pass
     if (e == cudaSuccess && dyn) {
+      ranges.next("adacad_beta");
       e = adacad_beta_launch(W.lp, dm.B, dm.N, dm.V, p->beta_out, W.ada, W.lm_tile_ctr, s);
       if (e == cudaSuccess) e = mark();
     }
@@ -341,9 +365,11 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ag.done_counter = W.done_counter;
     ag.status = W.status;
     if (agg) {
+      ranges.next("agg_partials");
       e = agg_partials_launch(ag, s);
       if (e == cudaSuccess) e = mark();
     }
+    if (e == cudaSuccess) ranges.next("agg_select");
     if (e == cudaSuccess) e = agg_select_launch(ag, s);
     if (e == cudaSuccess) e = mark();
     if (e != cudaSuccess) return cuda_status(e, "aggregation launches");
@@ -373,6 +399,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.beta = beta;
   la.status = W.status;
   la.pdl = (timed || dyn) ? 0 : 1;  // stage events between the launches would break the overlap
+  ranges.next("lm_head");
   e = lm_head_launch(wmap, hmap, g, la, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "lm head launch");
@@ -410,6 +437,7 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.status = W.status;
   sa.pdl = (timed || dyn) ? 0 : 1;
   sa.raw_logits = p->score_mode == PCED_SCORE_LOGIT;
+  ranges.next("select");
   e = select_from_records_launch(sa, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "select launch");
