@@ -328,8 +328,9 @@ def time_dynamic_beta_first_step(w, dev, reps=3):
         del dec, t
     f, r = statistics.median(first), statistics.median(regular)
     return {"first_step_us": f, "next_step_us": r, "extra_us": f - r, "reps": reps,
-            "path": "pced_step with beta_from_step: LM head writes the log-probs, pced_adacad_beta kernel, "
-                    "then the fused LM head and selection with that beta"}, status
+            "path": "pced_step with beta_from_step: the LM head writes raw logits and per-tile log-sum-exp records, "
+                    "lse_finalize, the beta kernel, then Eq. 3 over the stored logits with that beta "
+                    "(no second LM-head pass)"}, status
 
 
 def cpu_baseline(w, budget_s=20.0, max_steps=3):
