@@ -374,6 +374,15 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
               umma_slabs<2>(dcol, ad0, bd0, bstep, idesc, first);
             else
               umma_slabs<1>(dcol, ad0, bd0, bstep, idesc, first);
+          } else if (a.nchunk == 2 && SL == 1) {
+            // more than 256 hidden rows: two N chunks per K-step, unrolled
+            // (the issuing thread, not the data, set the pace with a loop here)
+            const uint32_t coff = (uint32_t)(a.chunk_n * 128) >> 4, dc1 = dcol + a.chunk_n;
+#pragma unroll
+            for (int k = 0; k < LM_TILE_K / 16; ++k) {
+              umma_bf16(dcol, ad0 + 2 * k, bd0 + 2 * k, idesc, (ks | k) != 0);
+              umma_bf16(dc1, ad0 + 2 * k, bd0 + coff + 2 * k, idesc, (ks | k) != 0);
+            }
           } else {
             for (int j = 0; j < SL; ++j) {
 #pragma unroll
@@ -535,6 +544,7 @@ cudaError_t lm_lse_finalize_launch(float* logits, const float2* rec_stats, float
 // records t, t + 256, ... in four interleaved chains, then a fixed tree), so
 // the result does not depend on timing.
 constexpr int SEL_R_THREADS = 256;
+constexpr int SEL_ZROWS = 12;  // hidden rows per block of the near-tie dot products
 
 __device__ __forceinline__ void lse_block(const float2* rec, int T, int tid, float2* red, float& L) {
   float m[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY}, su[4] = {0.f, 0.f, 0.f, 0.f};
@@ -577,7 +587,7 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
   __shared__ int last;
   __shared__ int pick[2];   // token, expert of the query (last CTA)
   __shared__ float zy[LM_MAX_N1];  // z_s(token) of the query's rows (last CTA)
-  __shared__ uint4 wrow[LM_MAX_D / 8];  // W[token] (last CTA)
+  __shared__ float zpart[SEL_R_THREADS / 32][SEL_ZROWS];
   float L = 0.f;
   lse_block(a.rec_stats + (int64_t)s * T, T, tid, red, L);
   if (j > 0) {
@@ -654,30 +664,59 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
   if (a.gap_trace && !a.key_out) {
     __syncthreads();
     const int y = pick[0] >= 0 && pick[0] < a.V ? pick[0] : 0;
-    // W[y] into shared memory with 16-byte loads (one round trip), then
-    // z_s(y) = h_s . W[y] for the query's rows, one warp per row, fp32 sums
-    // of independent 8-element chunks
+    // z_s(y) = h_s . W[y] for the query's rows.  Thread t takes the 16-byte
+    // chunks i = t, t + 256 of W[y] and the same chunks of up to 16 rows at a
+    // time, all loads of a row block in flight together (one round trip for
+    // d <= 4096); per row the partial sums meet in a fixed order (warp tree,
+    // then the warps in order).
     const int nv = a.d / 8;  // 16-byte chunks of a row (d % 64 == 0)
     const uint4* wy = reinterpret_cast<const uint4*>(a.w_unembed + (int64_t)y * a.d);
-    for (int i = tid; i < nv; i += SEL_R_THREADS) wrow[i] = __ldg(wy + i);
-    __syncthreads();
-    for (int jr = warp; jr < n1; jr += SEL_R_THREADS / 32) {
-      const uint4* hr = reinterpret_cast<const uint4*>(a.hidden + (int64_t)(b * n1 + jr) * a.d);
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
-      for (int i = lane; i < nv; i += 32) {
-        const uint4 hv = __ldcg(hr + i), wv = wrow[i];
-        const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w}, ww[4] = {wv.x, wv.y, wv.z, wv.w};
+    const uint4* h0 = reinterpret_cast<const uint4*>(a.hidden + (int64_t)b * n1 * a.d);
+    for (int r0 = 0; r0 < n1; r0 += SEL_ZROWS) {
+      float acc[SEL_ZROWS];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          acc[q] = fmaf(bf16_lo(hw[q]), bf16_lo(ww[q]), acc[q]);
-          acc[q] = fmaf(bf16_hi(hw[q]), bf16_hi(ww[q]), acc[q]);
+      for (int r = 0; r < SEL_ZROWS; ++r) acc[r] = 0.f;
+      for (int i0 = tid; i0 < nv; i0 += 2 * SEL_R_THREADS) {
+        uint4 wv[2], hv[2][SEL_ZROWS];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int i = i0 + u * SEL_R_THREADS;
+          if (i < nv) wv[u] = __ldg(wy + i);
+#pragma unroll
+          for (int r = 0; r < SEL_ZROWS; ++r)
+            if (i < nv && r0 + r < n1) hv[u][r] = __ldcg(h0 + (int64_t)(r0 + r) * nv + i);
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          if (i0 + u * SEL_R_THREADS >= nv) continue;
+          const uint32_t ww[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
+#pragma unroll
+          for (int r = 0; r < SEL_ZROWS; ++r) {
+            if (r0 + r >= n1) continue;
+            const uint32_t hw[4] = {hv[u][r].x, hv[u][r].y, hv[u][r].z, hv[u][r].w};
+            float p = 0.f;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              p = fmaf(bf16_lo(hw[q]), bf16_lo(ww[q]), p);
+              p = fmaf(bf16_hi(hw[q]), bf16_hi(ww[q]), p);
+            }
+            acc[r] += p;
+          }
         }
       }
-      const float t = warp_sum((acc[0] + acc[1]) + (acc[2] + acc[3]));
-      if (lane == 0) zy[jr] = t;
+#pragma unroll
+      for (int r = 0; r < SEL_ZROWS; ++r) {
+        const float t = warp_sum(acc[r]);
+        if (lane == 0) zpart[warp][r] = t;
+      }
+      __syncthreads();
+      if (tid < SEL_ZROWS && r0 + tid < n1) {
+        float z = 0.f;
+        for (int w = 0; w < SEL_R_THREADS / 32; ++w) z += zpart[w][tid];
+        zy[r0 + tid] = z;
+      }
+      __syncthreads();
     }
-    __syncthreads();
     if (warp == 0) {
       // token gap: the best score at another token, over all experts
       float other = -INFINITY, se_best = -INFINITY, se_other = -INFINITY;

@@ -10,7 +10,6 @@ constexpr int LM_THREADS = 64 + LM_EPI_THREADS;  // warp 0 TMA, warp 1 MMA + TME
 constexpr int LM_TILE_V = 128;   // vocabulary rows per tile (UMMA M)
 constexpr int LM_TILE_K = 64;    // hidden elements per stage (one 128-byte swizzle row)
 constexpr int LM_MAX_S = 512;
-constexpr int LM_MAX_D = 8192;   // hidden size of the fused step (the selection stages one W row)
 constexpr int LM_MAX_N1 = 256;   // experts + amateur per query in the selection kernels
 constexpr int LM_TRING = 16;     // claimed-tile ring between the TMA and MMA warps (> stages + 2 tiles in flight)
 
