@@ -31,6 +31,7 @@ sys.path.insert(0, ROOT)
 METRIC = "PCED decode tokens/s at N=8/32 experts; achieved HBM GB/s vs ~8 TB/s peak"
 UNIT = "tokens/s"
 NOMINAL_HBM_GBS = 8000.0
+GRAPH_STEPS = 8  # decode steps per captured CUDA graph (at most)
 
 
 def parse_args():
@@ -214,20 +215,37 @@ def build_decoder(w, dev, capacity_steps, paged=0, rope_theta=0.0, aggregation="
     return dec, t
 
 
+def steps_per_graph(steps, most=GRAPH_STEPS):
+    """Decode steps captured in one CUDA graph: the largest divisor of the
+    timed step count up to `most`, so the timed region is exactly `steps`."""
+    return max(k for k in range(1, most + 1) if steps % k == 0)
+
+
+def graph_capacity(steps, warmup):
+    """Steps time_graph runs: eager warm-up, warm-up graph replays, timed steps."""
+    k = steps_per_graph(steps)
+    return max(1, warmup) + k * (-(-warmup // k)) + steps
+
+
 def time_graph(dec, dist, steps, warmup, dev, clocks=None):
-    """Returns (elapsed ms of `steps` graph replays, lengths before the timed region)."""
+    """Returns (elapsed ms of `steps` decode steps replayed from CUDA graphs of
+    steps_per_graph(steps) steps each, lengths before the timed region).  Every
+    step in a graph is a full pced_step; several per graph only save the
+    launch of a graph between steps, as a serving loop would."""
     import torch
     s = torch.cuda.Stream(device=dev)
     for _ in range(max(1, warmup)):  # eager warm-up (also configures the kernels)
         dec.step()
     torch.cuda.synchronize(dev)
+    k = steps_per_graph(steps)
     s.wait_stream(torch.cuda.current_stream(dev))
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=s):
-        dec.step()
+        for _ in range(k):
+            dec.step()
     # capture does not execute: state is unchanged
     with torch.cuda.stream(s):
-        for _ in range(warmup):
+        for _ in range(-(-warmup // k)):
             g.replay()
     torch.cuda.synchronize(dev)
     lens0 = dec.seq_len.cpu().numpy().copy()
@@ -238,7 +256,7 @@ def time_graph(dec, dist, steps, warmup, dev, clocks=None):
     torch.cuda.synchronize(dev)
     with torch.cuda.stream(s):
         e0.record(s)
-        for _ in range(steps):
+        for _ in range(steps // k):
             g.replay()
         e1.record(s)
     torch.cuda.synchronize(dev)
@@ -378,7 +396,7 @@ def run_ours(args):
     hbm_peak = peaks.get("hbm_gbs")
     w = synth.get(args.workload)
     e2e_steps = 0 if args.no_e2e else min(args.steps, 16)
-    cap_steps = args.warmup * 2 + 1 + args.steps + args.profile_steps + e2e_steps + 2
+    cap_steps = graph_capacity(args.steps, args.warmup) + 1 + args.profile_steps + e2e_steps + 2
     dec, _ = build_decoder(w, dev, cap_steps, paged=args.paged, rope_theta=args.rope_theta,
                            aggregation=args.aggregation, raw_logits=args.raw_logits)
     launches = dec.launches_per_step()
@@ -454,7 +472,7 @@ def run_ours(args):
     if args.secondary != "none":
         w2 = synth.get(args.secondary)
         k2 = min(args.steps, 32)
-        dec2, _ = build_decoder(w2, dev, args.warmup * 2 + 1 + k2 + 1)
+        dec2, _ = build_decoder(w2, dev, graph_capacity(k2, args.warmup) + 2)
         ms2, l2, g2, s2, _ = time_graph(dec2, dist, k2, args.warmup, dev)
         ms2 = dist.max(ms2)
         b2 = sum(step_bytes(w2, l2 + 1 + i) for i in range(k2))
@@ -474,8 +492,9 @@ def run_ours(args):
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded counter-based generator)",
-            "config": workload_config(w, paged=args.paged, rope_theta=args.rope_theta, aggregation=args.aggregation,
-                                      raw_logits=args.raw_logits),
+            "config": dict(workload_config(w, paged=args.paged, rope_theta=args.rope_theta,
+                                           aggregation=args.aggregation, raw_logits=args.raw_logits),
+                           steps_per_graph=steps_per_graph(args.steps)),
             "step_hbm": {"achieved_gbs": step_gbs,
                                                        "frac_of_8tbps": step_gbs / NOMINAL_HBM_GBS,
                                                        "frac_of_measured": step_gbs / hbm_peak if hbm_peak else None,

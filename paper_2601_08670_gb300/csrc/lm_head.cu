@@ -45,10 +45,9 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g) {
   g->tmem_cols = cols;
   g->ntiles = (V + LM_TILE_V - 1) / LM_TILE_V;
   g->nks = d / LM_TILE_K;
-  g->nbeta = S;  // beta has B*N < S entries
   const size_t slab = LM_A_BYTES + (size_t)g->S_pad * 128;
   const size_t fixed = 1024 + 64 * 8 + 16 + (size_t)2 * 4 * g->S_pad * sizeof(float2) +
-                       (size_t)2 * g->S_pad * sizeof(float2) + (size_t)(g->nbeta + 3) * 4 + 8 * 64 * 4 + 64 + 128;
+                       (size_t)2 * g->S_pad * sizeof(float2) + (size_t)g->S_pad * sizeof(float2) + 32 * 4 + 8 * 64 * 4 + 64 + 128;
   // several consecutive K-slabs per stage so each row is fetched in longer
   // runs and the tensor cores get longer bursts per stage; keep at least
   // three stages in flight
@@ -117,20 +116,69 @@ __device__ __forceinline__ float bfly_reduce(float (&x)[NB], int lane, Op op) {
   return x[0];
 }
 
-// Epilogue of NB accumulator columns c0.. of one warp's 32 vocabulary rows:
-// mode 0 stores the logits; both modes record the per-column (max, sum of
-// exp) of the 32 rows; mode 1 also records per expert column the max of
-// u_k = (1 + beta) z_k - beta z_0 and its first (lowest) vocabulary index.
-// `bc` is this warp's 64-float broadcast buffer; z_am carries the row's
-// amateur logit from its query's first column to the expert columns.
+// Top-2 over the 32 lanes (vocabulary rows) of NB columns held one per
+// register, in the transposed form of bfly_reduce: (best value, its token,
+// best value at another token) travel together, ties to the lower token.
+// NB = 32: lane l ends with column l; NB = 16: lanes l and l ^ 16 both end
+// with column l & 15.  `tok` is this lane's token.
+template <int NB>
+__device__ __forceinline__ void bfly_top2(const float (&u)[NB], int tok, int lane, float& r1, int& rt, float& r2) {
+  float b1[16], b2[16];
+  int bt[16];
+  const int ptok = tok + ((lane ^ 16) - lane);  // the row across lane bit 4
+  const bool hi16 = (lane & 16) != 0;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    // NB = 32: the first halving level; NB = 16: a full exchange
+    const float send = NB == 32 ? (hi16 ? u[i] : u[i + 16 * (NB / 32)]) : u[i];
+    const float keep = NB == 32 ? (hi16 ? u[i + 16 * (NB / 32)] : u[i]) : u[i];
+    const float o = __shfl_xor_sync(0xffffffffu, send, 16);
+    const bool take = o > keep || (o == keep && ptok < tok);
+    b1[i] = take ? o : keep;
+    bt[i] = take ? ptok : tok;
+    b2[i] = take ? keep : o;
+  }
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1) {
+    const bool hi = (lane & w) != 0;
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      const float s1 = hi ? b1[i] : b1[i + w], s2 = hi ? b2[i] : b2[i + w];
+      const int st = hi ? bt[i] : bt[i + w];
+      float k1 = hi ? b1[i + w] : b1[i], k2 = hi ? b2[i + w] : b2[i];
+      int kt = hi ? bt[i + w] : bt[i];
+      const float o1 = __shfl_xor_sync(0xffffffffu, s1, w), o2 = __shfl_xor_sync(0xffffffffu, s2, w);
+      const int ot = __shfl_xor_sync(0xffffffffu, st, w);
+      top2_merge(k1, kt, k2, o1, ot, o2);
+      b1[i] = k1;
+      bt[i] = kt;
+      b2[i] = k2;
+    }
+  }
+  r1 = b1[0];
+  rt = bt[0];
+  r2 = b2[0];
+}
+
+// Epilogue of NB accumulator columns c0.. (c0 a multiple of 32) of one
+// warp's 32 vocabulary rows: mode 0 stores the logits; both modes record the
+// per-column (max, sum of exp) of the 32 rows; mode 1 also records per expert
+// column the max of u_k = (1 + beta) z_k - beta z_0, its first (lowest)
+// vocabulary index and the best value at another index.  `bc` is this warp's
+// broadcast buffer; z_am carries the row's amateur logit from its query's
+// first column to the expert columns; ccoef / cmask hold each column's
+// (1 + beta, beta) and the amateur / expert column bits of each 32-column
+// block (the same for every tile).
 template <int NB>
 __device__ __forceinline__ void epi_block(const LmArgs& a, uint32_t taddr, int c0, int v, bool valid, int lane,
-                                          int q, float* bc, float2* wst, float2* wag, float* wu2, const float* sbeta,
-                                          float& z_am) {
-  const int S = a.S, S_pad = a.S_pad, n1 = a.N + 1;
+                                          int q, float* bc, float2* wst, float2* wag, float* wu2, const float2* ccoef,
+                                          const uint32_t* cmask, float& z_am) {
+  const int S = a.S, S_pad = a.S_pad;
   float z[NB], t[NB];
-  tmem_ld16(taddr, z);
-  if (NB == 32) tmem_ld16(taddr + 16, z + 16);
+  if (NB == 32)
+    tmem_ld32(taddr, z);
+  else
+    tmem_ld16(taddr, z);
   if (a.mode == 0 && valid) {
 #pragma unroll
     for (int i = 0; i < NB; ++i)
@@ -138,49 +186,34 @@ __device__ __forceinline__ void epi_block(const LmArgs& a, uint32_t taddr, int c
   }
 #pragma unroll
   for (int i = 0; i < NB; ++i) t[i] = valid ? z[i] : -INFINITY;
+  float u[NB];
+  const uint32_t em = a.mode == 1 ? cmask[16 + (c0 >> 5)] : 0u;
+  if (a.mode == 1) {
+    const uint32_t am = cmask[c0 >> 5];
+    float za = z_am;
+#pragma unroll
+    for (int i = 0; i < NB; ++i) {
+      if ((am >> i) & 1u) za = z[i];
+      const float2 cf = ccoef[c0 + i];
+      u[i] = valid && ((em >> i) & 1u) ? cf.x * z[i] - cf.y * za : -INFINITY;
+    }
+    z_am = za;
+  }
   const float m = bfly_reduce<NB>(t, lane, FMax());
+  float b1 = -INFINITY, b2 = -INFINITY;
+  int bt = 0;
+  if (a.mode == 1) bfly_top2<NB>(u, v, lane, b1, bt, b2);
   const int li = lane & (NB - 1), mycol = c0 + li;
   if (lane < NB) bc[lane] = m;
   __syncwarp();
 #pragma unroll
   for (int i = 0; i < NB; ++i) t[i] = valid ? __expf(z[i] - bc[i]) : 0.f;
   const float sm = bfly_reduce<NB>(t, lane, FAdd());
-  if (lane < NB && mycol < S) wst[q * S_pad + mycol] = make_float2(m, sm);
-  if (a.mode == 1) {
-    float u[NB];
-#pragma unroll
-    for (int i = 0, j = c0 % n1, b = c0 / n1; i < NB; ++i) {
-      u[i] = -INFINITY;
-      if (c0 + i < S) {
-        if (j == 0) {
-          z_am = z[i];
-        } else {
-          const float bt = sbeta[b * a.N + j - 1];
-          if (valid) u[i] = (1.f + bt) * z[i] - bt * z_am;
-        }
-      }
-      t[i] = u[i];
-      if (++j == n1) {
-        j = 0;
-        ++b;
-      }
-    }
-    const float um = bfly_reduce<NB>(t, lane, FMax());
-    if (lane < NB) bc[32 + lane] = um;
-    __syncwarp();
-    unsigned mine = 0;
-#pragma unroll
-    for (int i = 0; i < NB; ++i) {
-      const unsigned hit = __ballot_sync(0xffffffffu, u[i] == bc[32 + i]);
-      if (li == i) mine = hit;
-      // the runner-up of the column: every row but the (lowest) one holding the maximum
-      t[i] = hit && lane == __ffs(hit) - 1 ? -INFINITY : u[i];
-    }
-    const float u2 = bfly_reduce<NB>(t, lane, FMax());
-    if (lane < NB && mycol < S && mycol % n1 != 0) {
-      const int r = mine ? __ffs(mine) - 1 : 0;
-      wag[q * S_pad + mycol] = make_float2(um, __int_as_float(v - lane + r));
-      wu2[q * S_pad + mycol] = u2;
+  if (lane < NB && mycol < S) {
+    wst[q * S_pad + mycol] = make_float2(m, sm);
+    if ((em >> li) & 1u) {
+      wag[q * S_pad + mycol] = make_float2(b1, __int_as_float(bt));
+      wu2[q * S_pad + mycol] = b2;
     }
   }
   __syncwarp();
@@ -225,8 +258,9 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
   float2* wst = reinterpret_cast<float2*>(gbase + (bar_drain + 8 - base) + 96);  // [4][S_pad] per-warp stats
   float2* wag = wst + 4 * S_pad;                                                  // [4][S_pad] per-warp argmax
   float* wu2 = reinterpret_cast<float*>(wag + 4 * S_pad);                         // [4][S_pad] per-warp runner-up
-  float* sbeta = reinterpret_cast<float*>(wag + 6 * S_pad);  // [nbeta]
-  float* bc = sbeta + ((a.nbeta + 3) & ~3);               // [8][64] per-warp column broadcast
+  float2* ccoef = wag + 6 * S_pad;                                 // [S_pad] (1 + beta, beta) per column
+  uint32_t* cmask = reinterpret_cast<uint32_t*>(ccoef + S_pad);     // [2][16] amateur / expert column bits
+  float* bc = reinterpret_cast<float*>(cmask + 32);                // [8][64] per-warp column broadcast
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
@@ -252,8 +286,27 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
     tmem_alloc(smem_u32(tmem_slot), a.tmem_cols);
     tmem_relinquish();
   }
-  if (a.mode == 1)
-    for (int i = tid; i < a.nbeta; i += LM_THREADS) sbeta[i] = a.beta[i];
+  if (a.mode == 1) {
+    // per column: expert columns carry (1 + beta_k, beta_k), the amateur
+    // column of each query starts its group; bit i of block kb is column 32 kb + i
+    const int n1 = a.N + 1;
+    for (int c = tid; c < S_pad; c += LM_THREADS) {
+      const int j = c % n1, bq = c / n1;
+      const float bt = c < a.S && j > 0 ? a.beta[bq * a.N + j - 1] : 0.f;
+      ccoef[c] = make_float2(1.f + bt, bt);
+    }
+    if (warp == 0)
+      for (int kb = 0; kb < 16; ++kb) {
+        const int c = 32 * kb + lane;
+        const bool in = c < a.S;
+        const uint32_t am = __ballot_sync(0xffffffffu, in && c % n1 == 0);
+        const uint32_t em = __ballot_sync(0xffffffffu, in && c % n1 != 0);
+        if (lane == 0) {
+          cmask[kb] = am;
+          cmask[16 + kb] = em;
+        }
+      }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -430,9 +483,9 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       for (int kb = kb0; kb < kb1; ++kb) {
         const int c0 = 32 * kb;
         if (c0 + 32 <= S_pad)
-          epi_block<32>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, sbeta, z_am);
+          epi_block<32>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, ccoef, cmask, z_am);
         else
-          epi_block<16>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, sbeta, z_am);
+          epi_block<16>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, ccoef, cmask, z_am);
       }
       tc_fence_before();
       mbar_arrive(bar_tempty + 8 * buf);
@@ -828,7 +881,6 @@ extern "C" pced_status pced_lm_head_logprobs(const void* hidden, const void* w_u
   a.nks = g.nks;
   a.slabs = g.slabs;
   a.nst = g.nst;
-  a.nbeta = 0;
   a.stages = g.stages;
   a.acc_bufs = g.acc_bufs;
   a.S_pad = g.S_pad;

@@ -14,7 +14,7 @@ constexpr int LM_MAX_N1 = 256;   // experts + amateur per query in the selection
 constexpr int LM_TRING = 16;     // claimed-tile ring between the TMA and MMA warps (> stages + 2 tiles in flight)
 
 struct LmGeom {
-  int32_t S, S_pad, nchunk, chunk_n, d, V, ntiles, nks, slabs, nst, stages, acc_bufs, grid, nbeta;
+  int32_t S, S_pad, nchunk, chunk_n, d, V, ntiles, nks, slabs, nst, stages, acc_bufs, grid;
   uint32_t tmem_cols;
   size_t smem;
 };
@@ -23,7 +23,7 @@ bool lm_geometry(int32_t S, int32_t d, int32_t V, LmGeom* g);
 
 struct LmArgs {
   int mode;  // 0: write logits[S][V]; 1: contrastive records (needs N, beta)
-  int32_t S, N, V, ntiles, nks, slabs, nst, stages, acc_bufs, S_pad, nchunk, chunk_n, nbeta;
+  int32_t S, N, V, ntiles, nks, slabs, nst, stages, acc_bufs, S_pad, nchunk, chunk_n;
   uint32_t tmem_cols;
   float* logits;      // mode 0
   float2* rec_stats;  // [S][ntiles] (max z, sum exp(z - max)) of each vocabulary tile

@@ -304,7 +304,6 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     lz.nks = g.nks;
     lz.slabs = g.slabs;
     lz.nst = g.nst;
-    lz.nbeta = 0;
     lz.stages = g.stages;
     lz.acc_bufs = g.acc_bufs;
     lz.S_pad = g.S_pad;
@@ -385,7 +384,6 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   la.nks = g.nks;
   la.slabs = g.slabs;
   la.nst = g.nst;
-  la.nbeta = dm.B * dm.N;
   la.stages = g.stages;
   la.acc_bufs = g.acc_bufs;
   la.S_pad = g.S_pad;

@@ -56,3 +56,18 @@ def test_single_rank_needs_no_process_group():
     assert d.max(3.5) == 3.5 and d.sum(2.0) == 2.0
     d.barrier()
     d.close()
+
+
+def test_timed_steps_are_exact_with_several_steps_per_graph():
+    sys.path.insert(0, ROOT)
+    import bench
+    for steps in (1, 4, 7, 11, 16, 32, 64, 100):
+        k = bench.steps_per_graph(steps)
+        assert 1 <= k <= bench.GRAPH_STEPS and steps % k == 0
+        assert (steps // k) * k == steps
+        # eager warm-up, whole graphs of warm-up, then the timed steps
+        for warmup in (1, 3, 5):
+            cap = bench.graph_capacity(steps, warmup)
+            assert cap == warmup + k * -(-warmup // k) + steps
+            assert k * -(-warmup // k) >= warmup
+    assert bench.steps_per_graph(64) == 8 and bench.steps_per_graph(7) == 7 and bench.steps_per_graph(11) == 1
