@@ -319,33 +319,41 @@ def run_e2e(dec, w, dev, steps):
 
 
 def time_dynamic_beta_first_step(w, dev, reps=3):
-    """Device time of the first step of a decode with dynamic contrast strength
-    and of the regular step after it (eager calls, CUDA events), median of
-    `reps` fresh decoders."""
+    """Device time of the first step of a decode with dynamic contrast strength,
+    of the regular step after it, and of the first step of a decode with a
+    fixed beta (eager calls, CUDA events), median of `reps` fresh decoders
+    each.  The extra cost of dynamic beta is the difference of the two first
+    steps: both start on freshly written caches, which the second step of a
+    decode does not."""
     import torch
     import paper_2601_08670_gb300 as pced
     import synth
     S = w.B * (w.N + 1)
     pced.adacad_beta(torch.zeros((S, w.V), dtype=torch.float32, device=dev), w.B, w.N)  # load the kernel
-    first, regular, status = [], [], 0
+    first, regular, fixed_first, status = [], [], [], 0
     for _ in range(reps):
-        t = synth.device_inputs(w, dev, extra_steps=4)
-        dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
-        dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=4, bos=w.bos, dynamic_beta=True)
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-        torch.cuda.synchronize()
-        ev[0].record()
-        dec.step()
-        ev[1].record()
-        dec.step()
-        ev[2].record()
-        torch.cuda.synchronize()
-        first.append(ev[0].elapsed_time(ev[1]) * 1e3)
-        regular.append(ev[1].elapsed_time(ev[2]) * 1e3)
-        status |= dec.status()
-        del dec, t
-    f, r = statistics.median(first), statistics.median(regular)
-    return {"first_step_us": f, "next_step_us": r, "extra_us": f - r, "reps": reps,
+        for dyn in (True, False):
+            t = synth.device_inputs(w, dev, extra_steps=4)
+            dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
+            dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=4, bos=w.bos, dynamic_beta=dyn)
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            torch.cuda.synchronize()
+            ev[0].record()
+            dec.step()
+            ev[1].record()
+            dec.step()
+            ev[2].record()
+            torch.cuda.synchronize()
+            if dyn:
+                first.append(ev[0].elapsed_time(ev[1]) * 1e3)
+                regular.append(ev[1].elapsed_time(ev[2]) * 1e3)
+            else:
+                fixed_first.append(ev[0].elapsed_time(ev[1]) * 1e3)
+            status |= dec.status()
+            del dec, t
+    f, r, ff = statistics.median(first), statistics.median(regular), statistics.median(fixed_first)
+    return {"first_step_us": f, "fixed_beta_first_step_us": ff, "next_step_us": r, "extra_us": f - ff,
+            "extra_vs_next_step_us": f - r, "reps": reps,
             "path": "pced_step with beta_from_step: the LM head writes raw logits and per-tile log-sum-exp records, "
                     "lse_finalize, the beta kernel, then Eq. 3 over the stored logits with that beta "
                     "(no second LM-head pass)"}, status

@@ -57,6 +57,7 @@ typedef enum pced_status {
 #define PCED_DEV_BAD_TOKEN 0x8u   /* history token outside [0, V) */
 #define PCED_DEV_STEP_LIMIT 0x10u /* step counter reached max_steps */
 #define PCED_DEV_BAD_BLOCK 0x20u  /* paged caches: a needed block-table entry is missing or outside the pool */
+#define PCED_DEV_BOUNDS 0x40u     /* bounds-checked build only: an index outside its buffer (the access was skipped) */
 
 /* Static description of a status code (host). */
 const char* pced_status_string(int32_t status);

@@ -14,7 +14,8 @@ import os
 import torch
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(HERE, "_lib", "libpced.so")
+# PCED_LIB=checked selects the bounds-checked build (build.build(checked=True))
+LIB_PATH = os.path.join(HERE, "_lib_checked" if os.environ.get("PCED_LIB") == "checked" else "_lib", "libpced.so")
 
 PCED_DEV_BAD_LENGTH = 0x1
 PCED_DEV_CACHE_FULL = 0x2
@@ -22,6 +23,7 @@ PCED_DEV_TIMEOUT = 0x4
 PCED_DEV_BAD_TOKEN = 0x8
 PCED_DEV_STEP_LIMIT = 0x10
 PCED_DEV_BAD_BLOCK = 0x20
+PCED_DEV_BOUNDS = 0x40
 
 
 class PcedError(RuntimeError):

@@ -15,6 +15,10 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIBDIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(LIBDIR, "libpced.so")
+# the bounds-checked build: every guarded index outside its buffer sets
+# PCED_DEV_BOUNDS in the status word and skips the access
+CHECKED_LIBDIR = os.path.join(HERE, "_lib_checked")
+CHECKED_LIB = os.path.join(CHECKED_LIBDIR, "libpced.so")
 ROOT = os.path.dirname(HERE)
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
@@ -28,16 +32,20 @@ def _deps():
     return max(os.path.getmtime(f) for f in files)
 
 
-def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
-    os.makedirs(LIBDIR, exist_ok=True)
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= _deps():
-        return LIB
+def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False, checked: bool = False) -> str:
+    """Compiles libpced.so if a source is newer; `checked` builds the
+    bounds-checked library (-DPCED_BOUNDS_CHECK) into its own folder."""
+    libdir, lib = (CHECKED_LIBDIR, CHECKED_LIB) if checked else (LIBDIR, LIB)
+    os.makedirs(libdir, exist_ok=True)
+    if not force and os.path.exists(lib) and os.path.getmtime(lib) >= _deps():
+        return lib
     procs = []
     objs = []
     for src in SOURCES:
-        obj = os.path.join(LIBDIR, src.replace(".cu", ".o"))
+        obj = os.path.join(libdir, src.replace(".cu", ".o"))
         objs.append(obj)
-        cmd = ["nvcc", *ARCH, *FLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
+        cmd = ["nvcc", *ARCH, *FLAGS, *(["-DPCED_BOUNDS_CHECK"] if checked else []), "-c", os.path.join(CSRC, src),
+               "-o", obj]
         if ptxas_info:
             cmd += ["-Xptxas", "-v"]
         procs.append((src, subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)))
@@ -50,10 +58,10 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
             failed.append(src)
     if failed:
         raise RuntimeError(f"nvcc failed for {failed}")
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = lib + f".tmp{os.getpid()}"
     subprocess.check_call(["nvcc", *ARCH, "-shared", "-o", tmp, *objs, "-cudart", "static"])
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":

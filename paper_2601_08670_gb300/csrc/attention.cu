@@ -1187,7 +1187,12 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
             arow = (int64_t)l * a.rows_per_layer + (a.kv_offset[pc.s] + (int64_t)pc.h * a.cap[pc.s] * D) / D +
                    lens[pc.s] - 1;
           }
-          const bool wrow = arow >= 0;  // a bad block id was flagged: keep the cache untouched
+          // a bad block id was flagged: keep the cache untouched
+          const bool wrow = arow >= 0 &&
+                            PCED_IN_BOUNDS(arow >= (int64_t)l * a.rows_per_layer &&
+                                               arow < (int64_t)(l + 1) * a.rows_per_layer &&
+                                               (a.block_table || lens[pc.s] - 1 < a.cap[pc.s]),
+                                           a.status);
           const int64_t grow = (wrow ? arow : 0) * D;
           constexpr int RQ = (D / 4 + 31) / 32;  // rotary quads per lane (as for the queries)
           float kx[RQ][4], vx[RQ][4];
@@ -1429,7 +1434,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     if (!merges) {
       // the segment continues in an earlier CTA: publish this CTA's record
       const int64_t rs = rbase + (int64_t)blockIdx.x + seg;
-      if (own) {
+      if (own && PCED_IN_BOUNDS(rs >= 0 && rs < (int64_t)a.groups * (gridDim.x + S * Hkv), a.status)) {
         uint64_t* ro = a.rec_o + rs * GD + idx0;
 #pragma unroll
         for (int j = 0; j < 4; ++j) st_tagged(ro + j, acc[j], tag);
@@ -1456,6 +1461,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
           for (int j = 0; j < 4; ++j) ov[q][j] = 0.f;
           if (!own || c + q > c1) continue;
           const int64_t rs = rbase + c + q + seg;
+          if (!PCED_IN_BOUNDS(rs >= 0 && rs < (int64_t)a.groups * (gridDim.x + S * Hkv), a.status)) continue;
           const uint64_t wm = ld_tagged(a.rec_ml + (rs * G + hh) * 2);
           const uint64_t wl = ld_tagged(a.rec_ml + (rs * G + hh) * 2 + 1);
           uint64_t wo[4];
@@ -1495,7 +1501,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     uint64_t* xn = a.resid + ((int64_t)nx * S + pc.s) * d + (int64_t)pc.h * GD;
     float xv[4] = {0.f, 0.f, 0.f, 0.f};
     float ss = 0.f;
-    if (own) {
+    if (own && PCED_IN_BOUNDS(pc.s >= 0 && pc.s < S && (int64_t)pc.h * GD + idx0 + 4 <= d, a.status)) {
       const float4 x4 = *reinterpret_cast<const float4*>(xr + idx0);
       const float xo[4] = {x4.x, x4.y, x4.z, x4.w};
 #pragma unroll

@@ -21,6 +21,19 @@ __device__ __forceinline__ void dev_flag(int* status, unsigned bit) {
   if (status) atomicOr(status, (int)bit);
 }
 
+// Bounds checks of the bounds-checked build (compiled with -DPCED_BOUNDS_CHECK):
+// an index outside its buffer sets PCED_DEV_BOUNDS and the guarded access is
+// skipped; the release build compiles the check away.
+__device__ __forceinline__ bool bounds_ok(bool in, int* status) {
+  if (!in) dev_flag(status, PCED_DEV_BOUNDS);
+  return in;
+}
+#ifdef PCED_BOUNDS_CHECK
+#define PCED_IN_BOUNDS(cond, status) ::pced::bounds_ok((cond), (status))
+#else
+#define PCED_IN_BOUNDS(cond, status) true
+#endif
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));

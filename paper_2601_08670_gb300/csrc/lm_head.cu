@@ -493,7 +493,8 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       // this tile's records: the four lane quarters' results folded in a fixed
       // order, stored per tile so the cross-tile merge order does not depend
       // on which CTA took the tile
-      for (int col = etid; col < S; col += LM_EPI_THREADS) {
+      const bool tile_ok = PCED_IN_BOUNDS(tile < ntiles, a.status);
+      for (int col = etid; col < S && tile_ok; col += LM_EPI_THREADS) {
         float cm = -INFINITY, cs = 0.f;
 #pragma unroll
         for (int qq = 0; qq < 4; ++qq) {
@@ -632,6 +633,7 @@ __device__ __forceinline__ void lse_block(const float2* rec, int T, int tid, flo
 __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(SelectArgs a) {
   const int j = blockIdx.x, b = blockIdx.y, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int N = a.N, n1 = N + 1, s = b * n1 + j, T = a.nrec;
+  if (!PCED_IN_BOUNDS(s < a.B * n1, a.status)) return;
   if (a.pdl) pdl_wait();  // the LM head's records are complete and visible
   if (j == 0 && b == 0 && tid == 0 && a.tile_ctr) *a.tile_ctr = 0;  // the next LM head claims its tiles from 0
   __shared__ float2 red[SEL_R_THREADS / 32];
