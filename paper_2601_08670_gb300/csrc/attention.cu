@@ -1605,7 +1605,7 @@ static int env_int(const char* name, int dflt, int lo, int hi) {
 int att_step_seg_cost(int D) { return env_int("PCED_ATT_SEGCOST", 512, 0, 1 << 20); }
 int att_step_pf_tiles() { return env_int("PCED_ATT_PF", 6, 0, 64); }
 int att_step_groups() { return env_int("PCED_ATT_GROUPS", 2, 1, ATT_MAX_GROUPS); }
-int att_step_seg_lead(int seg_cost) { return env_int("PCED_ATT_LEAD", 0, 0, seg_cost); }
+int att_step_seg_lead(int seg_cost) { return env_int("PCED_ATT_LEAD", seg_cost / 2, 0, seg_cost); }
 
 // cudaFuncSetAttribute once per kernel and device
 template <typename K>

@@ -95,13 +95,14 @@ struct FAdd {
 // held to the partner lane, so NB columns cost NB - 1 shuffles instead of
 // 5 NB.  The pairing (lane bit 4 first, bit 0 last) is that of a per-column
 // xor tree, so sums round identically.  NB = 32: lane l ends with column l;
-// NB = 16: after a full exchange across lane bit 4, lanes l and l ^ 16 both
-// end with column l & 15.
+// NB = 16 or 8: full exchanges across the lane bits at and above NB first, so
+// every lane l ends with column l & (NB - 1).
 template <int NB, class Op>
 __device__ __forceinline__ float bfly_reduce(float (&x)[NB], int lane, Op op) {
-  if (NB == 16) {
 #pragma unroll
-    for (int i = 0; i < 16; ++i) x[i] = op(x[i], __shfl_xor_sync(0xffffffffu, x[i], 16));
+  for (int w = 16; w >= NB; w >>= 1) {
+#pragma unroll
+    for (int i = 0; i < NB; ++i) x[i] = op(x[i], __shfl_xor_sync(0xffffffffu, x[i], w));
   }
 #pragma unroll
   for (int w = NB / 2; w >= 1; w >>= 1) {
@@ -119,27 +120,37 @@ __device__ __forceinline__ float bfly_reduce(float (&x)[NB], int lane, Op op) {
 // Top-2 over the 32 lanes (vocabulary rows) of NB columns held one per
 // register, in the transposed form of bfly_reduce: (best value, its token,
 // best value at another token) travel together, ties to the lower token.
-// NB = 32: lane l ends with column l; NB = 16: lanes l and l ^ 16 both end
-// with column l & 15.  `tok` is this lane's token.
+// Lane l ends with column l & (NB - 1).  `tok` is this lane's token.
 template <int NB>
 __device__ __forceinline__ void bfly_top2(const float (&u)[NB], int tok, int lane, float& r1, int& rt, float& r2) {
-  float b1[16], b2[16];
-  int bt[16];
+  constexpr int K = NB == 32 ? 16 : NB;  // slots after the first level
+  float b1[K], b2[K];
+  int bt[K];
   const int ptok = tok + ((lane ^ 16) - lane);  // the row across lane bit 4
   const bool hi16 = (lane & 16) != 0;
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    // NB = 32: the first halving level; NB = 16: a full exchange
-    const float send = NB == 32 ? (hi16 ? u[i] : u[i + 16 * (NB / 32)]) : u[i];
-    const float keep = NB == 32 ? (hi16 ? u[i + 16 * (NB / 32)] : u[i]) : u[i];
+  for (int i = 0; i < K; ++i) {
+    // NB = 32: the first halving level; NB <= 16: a full exchange
+    const float send = NB == 32 ? (hi16 ? u[i] : u[(i + 16) % NB]) : u[i];
+    const float keep = NB == 32 ? (hi16 ? u[(i + 16) % NB] : u[i]) : u[i];
     const float o = __shfl_xor_sync(0xffffffffu, send, 16);
     const bool take = o > keep || (o == keep && ptok < tok);
     b1[i] = take ? o : keep;
     bt[i] = take ? ptok : tok;
     b2[i] = take ? keep : o;
   }
+  // NB = 8: one more full exchange, across lane bit 3
 #pragma unroll
-  for (int w = 8; w >= 1; w >>= 1) {
+  for (int w = 8; w >= NB; w >>= 1) {
+#pragma unroll
+    for (int i = 0; i < K; ++i) {
+      const float o1 = __shfl_xor_sync(0xffffffffu, b1[i], w), o2 = __shfl_xor_sync(0xffffffffu, b2[i], w);
+      const int ot = __shfl_xor_sync(0xffffffffu, bt[i], w);
+      top2_merge(b1[i], bt[i], b2[i], o1, ot, o2);
+    }
+  }
+#pragma unroll
+  for (int w = (NB == 32 ? 8 : NB / 2); w >= 1; w >>= 1) {
     const bool hi = (lane & w) != 0;
 #pragma unroll
     for (int i = 0; i < w; ++i) {
@@ -160,7 +171,7 @@ __device__ __forceinline__ void bfly_top2(const float (&u)[NB], int tok, int lan
   r2 = b2[0];
 }
 
-// Epilogue of NB accumulator columns c0.. (c0 a multiple of 32) of one
+// Epilogue of NB accumulator columns c0.. (c0 a multiple of NB) of one
 // warp's 32 vocabulary rows: mode 0 stores the logits; both modes record the
 // per-column (max, sum of exp) of the 32 rows; mode 1 also records per expert
 // column the max of u_k = (1 + beta) z_k - beta z_0, its first (lowest)
@@ -177,8 +188,10 @@ __device__ __forceinline__ void epi_block(const LmArgs& a, uint32_t taddr, int c
   float z[NB], t[NB];
   if (NB == 32)
     tmem_ld32(taddr, z);
-  else
+  else if (NB == 16)
     tmem_ld16(taddr, z);
+  else
+    tmem_ld8(taddr, z);
   if (a.mode == 0 && valid) {
 #pragma unroll
     for (int i = 0; i < NB; ++i)
@@ -187,9 +200,9 @@ __device__ __forceinline__ void epi_block(const LmArgs& a, uint32_t taddr, int c
 #pragma unroll
   for (int i = 0; i < NB; ++i) t[i] = valid ? z[i] : -INFINITY;
   float u[NB];
-  const uint32_t em = a.mode == 1 ? cmask[16 + (c0 >> 5)] : 0u;
+  const uint32_t em = a.mode == 1 ? cmask[16 + (c0 >> 5)] >> (c0 & 31) : 0u;
   if (a.mode == 1) {
-    const uint32_t am = cmask[c0 >> 5];
+    const uint32_t am = cmask[c0 >> 5] >> (c0 & 31);
     float za = z_am;
 #pragma unroll
     for (int i = 0; i < NB; ++i) {
@@ -473,16 +486,20 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
       const int v = tile * LM_TILE_V + 32 * q + lane;
       const bool valid = v < a.V;
       const uint32_t trow = tmem_base + ((uint32_t)(32 * q) << 16) + buf * S_pad;
-      // column blocks of 32 (the last one may be 16 wide); the first half of
-      // the blocks goes to warps 2-5, the rest to warps 6-9
-      const int nb = (S + 31) / 32, kb0 = half ? (nb + 1) / 2 : 0, kb1 = half ? nb : (nb + 1) / 2;
+      // column blocks of W = 32 (the last one may be 16 wide), or of S_pad / 2
+      // when S_pad <= 32 so that both warp halves work; the first half of the
+      // blocks goes to warps 2-5, the rest to warps 6-9
+      const int W = S_pad <= 32 ? S_pad / 2 : 32;
+      const int nb = (S + W - 1) / W, kb0 = half ? (nb + 1) / 2 : 0, kb1 = half ? nb : (nb + 1) / 2;
       float z_am = 0.f;
-      if (a.mode == 1 && kb0 < kb1 && (32 * kb0) % n1 != 0)
-        z_am = tmem_ld1(trow + 32 * kb0 - (32 * kb0) % n1);  // the row's amateur logit of the open query
+      if (a.mode == 1 && kb0 < kb1 && (W * kb0) % n1 != 0)
+        z_am = tmem_ld1(trow + W * kb0 - (W * kb0) % n1);  // the row's amateur logit of the open query
       float* wbc = bc + 64 * (warp - 2);
       for (int kb = kb0; kb < kb1; ++kb) {
-        const int c0 = 32 * kb;
-        if (c0 + 32 <= S_pad)
+        const int c0 = W * kb;
+        if (W == 8)
+          epi_block<8>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, ccoef, cmask, z_am);
+        else if (c0 + 32 <= S_pad && W == 32)
           epi_block<32>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, ccoef, cmask, z_am);
         else
           epi_block<16>(a, trow + c0, c0, v, valid, lane, q, wbc, wst, wag, wu2, ccoef, cmask, z_am);
