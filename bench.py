@@ -41,6 +41,9 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="llama8")
+    p.add_argument("--layers", type=int, default=0,
+                   help="override the workload's layer count (small cases for multi-pass ncu captures; "
+                        "not the headline configuration)")
     p.add_argument("--secondary", default="llama32", help="second workload timed on the value path ('none' skips)")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
@@ -402,7 +405,7 @@ def run_ours(args):
     dist = Dist(world, local)
     peaks = measured_peaks()
     hbm_peak = peaks.get("hbm_gbs")
-    w = synth.get(args.workload)
+    w = synth.get(args.workload, **({"L": args.layers} if args.layers > 0 else {}))
     e2e_steps = 0 if args.no_e2e else min(args.steps, 16)
     cap_steps = graph_capacity(args.steps, args.warmup) + 1 + args.profile_steps + e2e_steps + 2
     dec, _ = build_decoder(w, dev, cap_steps, paged=args.paged, rope_theta=args.rope_theta,
@@ -524,7 +527,7 @@ def run_reference(args):
     import oracle
     import synth
     from oracle.run import OracleRun
-    w = synth.get(args.workload)
+    w = synth.get(args.workload, **({"L": args.layers} if args.layers > 0 else {}))
     run = OracleRun(w, extra_steps=args.warmup + args.steps + 1)
     t0 = time.perf_counter()
     run.step()

@@ -53,3 +53,10 @@ def test_two_mma_chunks_s272(cuda_ok):
 def test_larger_logits_scale(cuda_ok):
     # logits with std ~ 6: exercises the max-subtracted sums
     assert run_case(17, 1024, 3000, wscale=0.2) < 1e-3
+
+
+@pytest.mark.parametrize("S", [272, 300, 340])
+def test_many_tiles_per_cta_with_two_n_chunks(cuda_ok, S):
+    # more than 256 hidden rows: two N chunks in one TMEM accumulator, several
+    # vocabulary tiles per CTA (the accumulator is reused), ragged tail
+    assert run_case(S, 256, 48000 + 77) < 1e-4
