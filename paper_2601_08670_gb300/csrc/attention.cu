@@ -589,7 +589,7 @@ __device__ __forceinline__ bool poll_again(uint64_t& t0, int* status, unsigned l
     dev_flag(status, PCED_DEV_TIMEOUT);
     return false;
   }
-  __nanosleep(32);
+  __nanosleep(128);  // fewer polls of L2 while the data is on its way (measured 1-4 us faster per step than 32 ns)
   return true;
 }
 
@@ -925,18 +925,42 @@ __device__ void embed_sequence(const StepAttArgs& a, int s, uint32_t tag, int la
     tok = 0;
   }
   if (s == 0 && lane == 0 && t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
-  const __nv_bfloat162* e = reinterpret_cast<const __nv_bfloat162*>(a.embed + (int64_t)tok * d);
+  // the row in 16-byte chunks, CPG per head group; every load of a batch of
+  // head groups is issued before its stores (a tagged store orders memory,
+  // so a load after it would wait a whole round trip: with one load per
+  // store this loop took ~36 us per sequence, the start of every layer 0)
+  const uint4* e = reinterpret_cast<const uint4*>(a.embed + (int64_t)tok * d);
   uint64_t* x = a.resid + (int64_t)s * d;
-  for (int h = 0; h < a.Hkv; ++h) {
-    float ss = 0.f;
-    for (int i = lane; i < GD / 2; i += 32) {
-      const float2 v = __bfloat1622float2(e[h * GD / 2 + i]);
-      st_tagged(x + h * GD + 2 * i, v.x, tag);
-      st_tagged(x + h * GD + 2 * i + 1, v.y, tag);
-      ss += v.x * v.x + v.y * v.y;
+  constexpr int EB = 8;  // chunks per lane in flight
+  const int cpg = GD / 8;  // <= ATT_MAX_G * D / 8 = 128 <= 32 * EB
+  const int hpb = (32 * EB) / cpg;
+  for (int h0 = 0; h0 < a.Hkv; h0 += hpb) {
+    const int h1 = min(a.Hkv, h0 + hpb), cb = h0 * cpg, ce = h1 * cpg;
+    uint4 v[EB];
+#pragma unroll
+    for (int j = 0; j < EB; ++j) {
+      const int c = cb + lane + 32 * j;
+      v[j] = c < ce ? __ldg(e + c) : make_uint4(0u, 0u, 0u, 0u);
     }
-    ss = warp_sum(ss);
-    if (lane < ATT_CONSUMERS) st_tagged(a.part_ss + ((int64_t)s * a.Hkv + h) * ATT_CONSUMERS + lane, lane == 0 ? ss : 0.f, tag);
+    for (int h = h0; h < h1; ++h) {
+      float ss = 0.f;
+#pragma unroll
+      for (int j = 0; j < EB; ++j) {
+        const int c = cb + lane + 32 * j;
+        if (c >= ce || c / cpg != h) continue;
+        const uint32_t w[4] = {v[j].x, v[j].y, v[j].z, v[j].w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float lo = bf16_lo(w[k]), hi = bf16_hi(w[k]);
+          st_tagged(x + 8 * (int64_t)c + 2 * k, lo, tag);
+          st_tagged(x + 8 * (int64_t)c + 2 * k + 1, hi, tag);
+          ss += lo * lo + hi * hi;
+        }
+      }
+      ss = warp_sum(ss);
+      if (lane < ATT_CONSUMERS)
+        st_tagged(a.part_ss + ((int64_t)s * a.Hkv + h) * ATT_CONSUMERS + lane, lane == 0 ? ss : 0.f, tag);
+    }
   }
 }
 
