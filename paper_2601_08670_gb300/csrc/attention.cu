@@ -912,55 +912,52 @@ __host__ __device__ inline StepSmem step_smem(int D, int G) {
   return L;
 }
 
-// x_0[s] = E[y_{t-1}] (tagged, residual buffer 0) and its per-group sums of
-// squares (in partial slot 0 of each group; slots 1..7 hold 0).  One warp.
+// x_0[s] = E[y_{t-1}] for every sequence (tagged, residual buffer 0) and its
+// per-group sums of squares.  The rows are cut into (sequence, kv-head group,
+// eighth) slices of GD / 8 elements, spread over the CTAs' input warps: each
+// lane loads one 16-byte chunk, so a warp's share is one memory round trip
+// (one warp embedding a whole row waited on the load traffic of the whole
+// grid at the start of a launch), and each slice's sum of squares goes to its
+// own partial-sum slot (ATT_CONSUMERS per head group, the layout the layers'
+// merges use).  Whole warp.
 template <int D>
-__device__ void embed_sequence(const StepAttArgs& a, int s, uint32_t tag, int lane) {
-  const int d = a.Hq * D, GD = a.G * D, b = s / a.n1;
+__device__ void embed_slices(const StepAttArgs& a, uint32_t tag, int lane) {
+  const int d = a.Hq * D, GD = a.G * D, S = a.S, Hkv = a.Hkv;
+  const int cps = GD / (8 * ATT_CONSUMERS);  // chunks of a slice: G*D/64, in [2, 16]
+  int lps = 1;                               // lanes per slice: cps rounded up to a power of two
+  while (lps < cps) lps <<= 1;
+  const int per_pass = 32 / lps;             // slices a warp covers at once
+  const int nslices = S * Hkv * ATT_CONSUMERS;
   const int t = *a.step;
-  int tok = a.bos;
-  if (t > 0 && t <= a.max_steps) tok = a.history[(int64_t)b * a.max_steps + t - 1];
-  if (tok < 0 || tok >= a.V) {
-    if (lane == 0) dev_flag(a.status, PCED_DEV_BAD_TOKEN);
-    tok = 0;
-  }
-  if (s == 0 && lane == 0 && t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
-  // the row in 16-byte chunks, CPG per head group; every load of a batch of
-  // head groups is issued before its stores (a tagged store orders memory,
-  // so a load after it would wait a whole round trip: with one load per
-  // store this loop took ~36 us per sequence, the start of every layer 0)
-  const uint4* e = reinterpret_cast<const uint4*>(a.embed + (int64_t)tok * d);
-  uint64_t* x = a.resid + (int64_t)s * d;
-  constexpr int EB = 8;  // chunks per lane in flight
-  const int cpg = GD / 8;  // <= ATT_MAX_G * D / 8 = 128 <= 32 * EB
-  const int hpb = (32 * EB) / cpg;
-  for (int h0 = 0; h0 < a.Hkv; h0 += hpb) {
-    const int h1 = min(a.Hkv, h0 + hpb), cb = h0 * cpg, ce = h1 * cpg;
-    uint4 v[EB];
-#pragma unroll
-    for (int j = 0; j < EB; ++j) {
-      const int c = cb + lane + 32 * j;
-      v[j] = c < ce ? __ldg(e + c) : make_uint4(0u, 0u, 0u, 0u);
+  if (blockIdx.x == 0 && lane == 0 && t >= a.max_steps) dev_flag(a.status, PCED_DEV_STEP_LIMIT);
+  for (int q0 = blockIdx.x * per_pass; q0 < nslices; q0 += gridDim.x * per_pass) {
+    const int q = q0 + lane / lps, k = lane % lps;
+    const bool on = q < nslices && k < cps;
+    const int s = on ? q / (Hkv * ATT_CONSUMERS) : 0, h = on ? (q / ATT_CONSUMERS) % Hkv : 0, j = q % ATT_CONSUMERS;
+    int tok = a.bos;
+    if (t > 0 && t <= a.max_steps) tok = a.history[(int64_t)(s / a.n1) * a.max_steps + t - 1];
+    if (tok < 0 || tok >= a.V) {
+      if (on) dev_flag(a.status, PCED_DEV_BAD_TOKEN);
+      tok = 0;
     }
-    for (int h = h0; h < h1; ++h) {
-      float ss = 0.f;
+    const int64_t e0 = (int64_t)h * GD + (int64_t)j * (GD / ATT_CONSUMERS) + 8 * k;  // first element of the chunk
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (on) v = __ldg(reinterpret_cast<const uint4*>(a.embed + (int64_t)tok * d + e0));
+    float ss = 0.f;
+    if (on) {
+      uint64_t* x = a.resid + (int64_t)s * d + e0;
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-      for (int j = 0; j < EB; ++j) {
-        const int c = cb + lane + 32 * j;
-        if (c >= ce || c / cpg != h) continue;
-        const uint32_t w[4] = {v[j].x, v[j].y, v[j].z, v[j].w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float lo = bf16_lo(w[k]), hi = bf16_hi(w[k]);
-          st_tagged(x + 8 * (int64_t)c + 2 * k, lo, tag);
-          st_tagged(x + 8 * (int64_t)c + 2 * k + 1, hi, tag);
-          ss += lo * lo + hi * hi;
-        }
+      for (int i = 0; i < 4; ++i) {
+        const float lo = bf16_lo(w[i]), hi = bf16_hi(w[i]);
+        st_tagged(x + 2 * i, lo, tag);
+        st_tagged(x + 2 * i + 1, hi, tag);
+        ss += lo * lo + hi * hi;
       }
-      ss = warp_sum(ss);
-      if (lane < ATT_CONSUMERS)
-        st_tagged(a.part_ss + ((int64_t)s * a.Hkv + h) * ATT_CONSUMERS + lane, lane == 0 ? ss : 0.f, tag);
     }
+    // the slice's lanes are an aligned group of lps: a xor tree over them
+    for (int o = 1; o < lps; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if (on && k == 0) st_tagged(a.part_ss + ((int64_t)s * Hkv + h) * ATT_CONSUMERS + j, ss, tag);
   }
 }
 
@@ -1096,7 +1093,7 @@ __global__ void __launch_bounds__(STEP_THREADS, 1)
     // group sums of x_l[s], then hand the consumers q = bf16(x_l * inv_rms)
     // (and, for the piece holding the row appended this step, that row's K
     // and V, also written to the caches) through a double-buffered slot.
-    for (int s = blockIdx.x; s < S; s += gridDim.x) embed_sequence<D>(a, s, step_tag(epoch, 0), lane);
+    embed_slices<D>(a, step_tag(epoch, 0), lane);
     uint32_t p = 0;
     bool ok = true;
     for (int l = 0; l < a.L && ok; ++l) {
