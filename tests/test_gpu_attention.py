@@ -12,7 +12,7 @@ from gpu_util import to_dev_bf16
 
 pytestmark = pytest.mark.gpu
 
-# Spec tolerance for attention outputs (bf16 in, fp32 accumulate): 2e-2
+# Attention tolerance (bf16 in, fp32 accumulate): 2e-2
 # relative.  The kernel keeps QK^T exact in fp32 and P to ~16 bits, so the
 # observed error is far below; the bound is applied per (sequence, head) row
 # relative to that row's largest magnitude.

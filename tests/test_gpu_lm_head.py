@@ -9,7 +9,7 @@ from gpu_util import to_dev_bf16
 
 pytestmark = pytest.mark.gpu
 
-# Spec tolerance for log-probs: 1e-2 absolute (bf16 inputs, fp32
+# Log-prob tolerance: 1e-2 absolute (bf16 inputs, fp32
 # accumulation).  Products of bf16 operands are exact in fp32 and the sums run
 # over d <= 4096 terms, so the observed error is ~1e-5.
 ABS_TOL = 1e-2

@@ -17,9 +17,9 @@ from oracle.run import OracleRun
 
 pytestmark = pytest.mark.gpu
 
-LSE_TOL = 1e-2  # spec log-prob tolerance (absolute)
+LSE_TOL = 1e-2  # log-prob tolerance (absolute)
 # Hidden state h = bf16(rmsnorm(x_L)) after the whole attention chain: every
-# element within the spec attention bound, 2e-2 of the largest
+# element within the attention tolerance, 2e-2 of the largest
 # magnitude of its (sequence, head) block, and most elements bit-equal (fp32
 # accumulation against fp64 moves a bf16 rounding only near a midpoint).
 H_REL_TOL = 2e-2
