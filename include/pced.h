@@ -226,7 +226,8 @@ typedef struct pced_step_args {
   const int32_t* cap;       /* [S] rows per slab */
   int64_t total_cap;        /* host: sum of cap */
   int32_t* seq_len;         /* [S] live rows; +1 per step */
-  int32_t* step;            /* [1] step counter t; +1 per step */
+  int32_t* step;            /* [1] step counter t; +1 per step while t < max_steps (at the
+                               limit nothing is appended and PCED_DEV_STEP_LIMIT is set) */
   int32_t* history;         /* [B][max_steps] chosen tokens */
   int32_t* expert_trace;    /* [B][max_steps] winning expert (1-based), may be NULL */
   float* score_trace;       /* [B][max_steps] winning score, may be NULL */

@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(AGG_THREADS) agg_select_kernel(AggArgs a) {
     }
     __threadfence();
     if (atomicAdd(a.done_counter, 1) == a.B - 1) {
-      *a.step = t + 1;
+      if (t >= 0 && t < a.max_steps) *a.step = t + 1;  // at the limit t stays (as the commit does)
       *a.done_counter = 0;
       __threadfence();
     }

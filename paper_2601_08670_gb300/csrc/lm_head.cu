@@ -836,7 +836,7 @@ __global__ void __launch_bounds__(SEL_R_THREADS) select_from_records_kernel(Sele
       }
       __threadfence();
       if (atomicAdd(a.done_counter, 1) == a.B - 1) {
-        *a.step = t + 1;
+        if (t >= 0 && t < a.max_steps) *a.step = t + 1;  // at the limit t stays (as the commit does)
         *a.done_counter = 0;
         __threadfence();
       }

@@ -99,11 +99,11 @@ def check_stats(stats, name=""):
     assert nt <= MAX_NEAR_TIE_FRAC * stats["compared"], f"{name}: {nt} near ties in {stats['compared']} selections"
 
 
-def run_parity(name, steps, queries=None, graph=False, min_ram_gb=0.0):
+def run_parity(name, steps, queries=None, graph=False, min_ram_gb=0.0, **overrides):
     if host_ram_gb() < min_ram_gb:
         pytest.skip(f"needs {min_ram_gb} GB of free host memory for the oracle's caches")
     dev = torch.device("cuda")
-    w = synth.get(name)
+    w = synth.get(name, **overrides)
     dec, _ = make_decoder(w, dev)
     run = OracleRun(w, queries=queries)
     stats = new_stats()
@@ -138,6 +138,13 @@ def test_tiny_all_steps(cuda_ok):
 
 def test_tiny_graph_replay(cuda_ok):
     run_parity("tiny", 4, graph=True)
+
+
+@pytest.mark.parametrize("V", [8192 + 77, 1000, 128 * 300 + 1])
+def test_tiny_ragged_vocabularies(cuda_ok, V):
+    # the last vocabulary tile of the fused LM head is partly outside V:
+    # its rows must neither win Eq. 3 nor enter the log-sum-exps
+    run_parity("tiny", 3, V=V)
 
 
 def test_llama8_full_size(cuda_ok):
@@ -196,6 +203,44 @@ def test_cache_full_is_flagged_not_faulted(cuda_ok):
     torch.cuda.synchronize()
     assert dec.status() & pced.PCED_DEV_CACHE_FULL
     assert np.array_equal(dec.seq_len.cpu().numpy(), synth.base_lengths(w) + 1)
+
+
+def test_history_token_outside_the_vocabulary_is_flagged(cuda_ok):
+    # the embedding of y_{t-1} checks the token: outside [0, V) it sets
+    # PCED_DEV_BAD_TOKEN and embeds token 0 instead (no out-of-range read)
+    import paper_2601_08670_gb300 as pced
+    dev = torch.device("cuda")
+    w = synth.get("tiny")
+    dec, _ = make_decoder(w, dev)
+    dec.step()
+    torch.cuda.synchronize()
+    assert dec.status() == 0
+    dec.history[:, 0] = w.V + 5
+    dec.step()
+    torch.cuda.synchronize()
+    assert dec.status() & pced.PCED_DEV_BAD_TOKEN
+    assert int(dec.step_t.item()) == 2
+    assert np.all((dec.history[:, 1].cpu().numpy() >= 0) & (dec.history[:, 1].cpu().numpy() < w.V))
+
+
+def test_step_limit_is_flagged_and_appends_nothing(cuda_ok):
+    # a step at t = max_steps writes no history entry and leaves t unchanged
+    import paper_2601_08670_gb300 as pced
+    dev = torch.device("cuda")
+    w = synth.get("tiny")
+    t = synth.device_inputs(w, dev, extra_steps=4)
+    dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
+    dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=2, bos=w.bos)
+    dec.step()
+    dec.step()
+    torch.cuda.synchronize()
+    assert dec.status() == 0
+    hist = dec.history.clone()
+    dec.step()
+    torch.cuda.synchronize()
+    assert dec.status() & pced.PCED_DEV_STEP_LIMIT
+    assert int(dec.step_t.item()) == 2
+    assert torch.equal(dec.history, hist)
 
 
 def test_expired_waits_report_timeout_and_leave_the_device_usable(cuda_ok):
