@@ -16,12 +16,12 @@ pytestmark = pytest.mark.gpu
 SCORE_TOL = 2e-2
 
 
-def run_variant(name, steps, ram, **kw):
+def run_variant(name, steps, ram, paged=0, overrides=None, **kw):
     import paper_2601_08670_gb300 as pced
     if host_ram_gb() < ram:
         pytest.skip(f"needs {ram} GB of free host memory for the oracle's caches")
-    w = synth.get(name)
-    t = synth.device_inputs(w, "cuda")
+    w = synth.get(name, **(overrides or {}))
+    t = synth.device_inputs(w, "cuda", paged=paged)
     dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
     dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=w.steps, bos=w.bos, keep_hidden=True, **kw)
     run = OracleRun(w, **kw)
@@ -53,6 +53,19 @@ def test_moe_poe_llama8(cuda_ok, rule):
 def test_raw_logit_mode(cuda_ok):
     run_variant("tiny", 4, 0, score_mode=1)
     run_variant("llama8", 2, 8, score_mode=1)
+
+
+@pytest.mark.parametrize("rule,paged,theta", [(1, 64, 0.0), (2, 128, 5e5), (1, 0, 1e4)])
+def test_aggregation_with_paged_caches_and_rotary(cuda_ok, rule, paged, theta):
+    # the aggregation kernels after attention over paged caches and / or
+    # rotary positions (the options compose: they touch different stages)
+    run_variant("tiny", 3, 0, paged=paged, aggregation=rule, rope_theta=theta)
+    run_variant("llama8", 2, 2, paged=paged, overrides={"L": 4}, aggregation=rule, rope_theta=theta)
+
+
+def test_dynamic_beta_with_rotary_and_raw_logits(cuda_ok):
+    run_variant("tiny", 3, 0, dynamic_beta=True, rope_theta=1e4)
+    run_variant("tiny", 3, 0, score_mode=1, rope_theta=1e4)
 
 
 def test_moe_with_dynamic_beta_and_graph_replay(cuda_ok):

@@ -96,7 +96,9 @@ def check_stats(stats, name=""):
     assert eq >= H_BITS_MIN, f"{name}: only {eq:.4f} of the hidden-state elements bit-equal"
     nt = stats["near_ties"]
     assert nt < stats["compared"], f"{name}: every selection was a near tie"
-    assert nt <= MAX_NEAR_TIE_FRAC * stats["compared"], f"{name}: {nt} near ties in {stats['compared']} selections"
+    # near ties occur at a rate set by the inputs; a run of a few selections
+    # may hold one
+    assert nt <= max(1.0, MAX_NEAR_TIE_FRAC * stats["compared"]), f"{name}: {nt} near ties in {stats['compared']} selections"
 
 
 def run_parity(name, steps, queries=None, graph=False, min_ram_gb=0.0, **overrides):
@@ -145,6 +147,25 @@ def test_tiny_ragged_vocabularies(cuda_ok, V):
     # the last vocabulary tile of the fused LM head is partly outside V:
     # its rows must neither win Eq. 3 nor enter the log-sum-exps
     run_parity("tiny", 3, V=V)
+
+
+@pytest.mark.parametrize("Hq,Hkv,D", [(4, 2, 64), (6, 2, 128), (16, 2, 64), (16, 2, 128), (12, 4, 128)])
+def test_tiny_head_shapes(cuda_ok, Hq, Hkv, D):
+    # query heads per kv head G = 2, 3, 8, 8, 3 with D = 64 / 128: the packed
+    # (G <= 4) and unpacked MMA layouts, odd G, the embedding slices' widths
+    run_parity("tiny", 4, Hq=Hq, Hkv=Hkv, D=D)
+
+
+@pytest.mark.parametrize("env", [{"PCED_ATT_LEAD": "0"}, {"PCED_ATT_SEGCOST": "0"},
+                                 {"PCED_ATT_SEGCOST": "1024", "PCED_ATT_LEAD": "1024"}, {"PCED_ATT_PF": "0"},
+                                 {"PCED_ATT_PF": "16"}])
+def test_partition_tunables_keep_parity(cuda_ok, monkeypatch, env):
+    # the attention partition's launch tunables move piece boundaries and
+    # prefetch distances, never results beyond the summation order
+    for k, v in env.items():
+        monkeypatch.setenv(k, v)
+    run_parity("llama8", 2, min_ram_gb=2, L=4)
+    run_parity("tiny", 3)
 
 
 def test_llama8_full_size(cuda_ok):
