@@ -294,31 +294,50 @@ def profile_launches(dec, g_unused, dev, reps):
 
 
 def run_e2e(dec, w, dev, steps):
-    """Public-API steps with host buffers: per step the retrieval scores and
-    contrastive weights are uploaded from pinned host memory, pced_step runs,
-    and the chosen token / expert / score are read back."""
+    """End to end through the C ABI with host buffers (pced_step_host_io), as a
+    serving loop runs it: every step uploads beta and r from page-locked host
+    memory, runs the decode step and copies the chosen token / expert / score
+    back; the host reads each step's choice while the next step runs (two
+    host slots used in turn).  Timed twice by the wall clock over `steps`
+    steps: with one captured CUDA graph of the call per slot (a replay is one
+    step with its copies) and with eager calls.  Returns both times, the
+    bytes copied per step and whether the tokens read on the host are the
+    device history."""
     import torch
+    B = w.B
     beta_h = dec.beta.cpu().pin_memory()
     r_h = dec.r.cpu().pin_memory()
-    out_tok = torch.empty(w.B, dtype=torch.int32).pin_memory()
-    out_exp = torch.empty(w.B, dtype=torch.int32).pin_memory()
-    out_sc = torch.empty(w.B, dtype=torch.float32).pin_memory()
-    torch.cuda.synchronize(dev)
-    t_first = int(dec.step_t.item())
-    t0 = time.perf_counter()
-    for i in range(steps):
-        dec.beta.copy_(beta_h, non_blocking=True)
-        dec.r.copy_(r_h, non_blocking=True)
-        dec.step()
-        t = t_first + i
-        out_tok.copy_(dec.history[:, t], non_blocking=True)
-        out_exp.copy_(dec.expert_trace[:, t], non_blocking=True)
-        out_sc.copy_(dec.score_trace[:, t], non_blocking=True)
-    torch.cuda.synchronize(dev)
-    el = time.perf_counter() - t0
+    slots = [dict(token=torch.zeros(B, dtype=torch.int32).pin_memory(),
+                  expert=torch.zeros(B, dtype=torch.int32).pin_memory(),
+                  score=torch.zeros(B, dtype=torch.float32).pin_memory()) for _ in range(2)]
+    graphs = [dec.capture_host_io(beta_h, r_h, **sl) for sl in slots]
+    events = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def loop(run):
+        run(0)  # warm-up steps (a graph's first replay also uploads it)
+        run(1)
+        torch.cuda.synchronize(dev)
+        t_first = int(dec.step_t.item())
+        got = []
+        t0 = time.perf_counter()
+        for i in range(steps + 1):
+            if i < steps:
+                run(i % 2)
+                events[i % 2].record()
+            if i:  # the previous step's choice, read while this one runs
+                events[(i - 1) % 2].synchronize()
+                sl = slots[(i - 1) % 2]
+                got.append((sl["token"].tolist(), sl["expert"].tolist(), sl["score"].tolist()))
+        el = time.perf_counter() - t0
+        hist = dec.history[:, t_first:t_first + steps].cpu().T.tolist()
+        return el, [g[0] for g in got] == hist
+
+    el_graph, ok_graph = loop(lambda k: graphs[k].replay())
+    el_eager, ok_eager = loop(lambda k: dec.step_host_io(beta_h, r_h, **slots[k]))
+    del graphs
     h2d = beta_h.numel() * 4 + r_h.numel() * 4
-    d2h = w.B * (4 + 4 + 4)
-    return el, h2d, d2h
+    d2h = B * (4 + 4 + 4)
+    return el_graph, el_eager, h2d, d2h, ok_graph and ok_eager
 
 
 def time_dynamic_beta_first_step(w, dev, reps=3):
@@ -406,8 +425,8 @@ def run_ours(args):
     peaks = measured_peaks()
     hbm_peak = peaks.get("hbm_gbs")
     w = synth.get(args.workload, **({"L": args.layers} if args.layers > 0 else {}))
-    e2e_steps = 0 if args.no_e2e else min(args.steps, 16)
-    cap_steps = graph_capacity(args.steps, args.warmup) + 1 + args.profile_steps + e2e_steps + 2
+    e2e_steps = 0 if args.no_e2e else min(args.steps, 32)
+    cap_steps = graph_capacity(args.steps, args.warmup) + 1 + args.profile_steps + 2 * (e2e_steps + 2) + 2
     dec, _ = build_decoder(w, dev, cap_steps, paged=args.paged, rope_theta=args.rope_theta,
                            aggregation=args.aggregation, raw_logits=args.raw_logits)
     launches = dec.launches_per_step()
@@ -461,12 +480,18 @@ def run_ours(args):
 
     e2e = None
     if e2e_steps:
-        el, h2d, d2h = run_e2e(dec, w, dev, e2e_steps)
-        el = dist.max(el)
+        el, el_eager, h2d, d2h, same = run_e2e(dec, w, dev, e2e_steps)
+        el, el_eager = dist.max(el), dist.max(el_eager)
         e2e = {"value": dist.sum(w.B * e2e_steps) / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-               "path": "Decoder.step (pced_step C ABI, no graph) + pinned host copies of beta/r in and "
-                       "token/expert/score out, wall clock"}
+               "path": "pced_step_host_io (C ABI, host buffers): beta and r uploaded from page-locked host "
+                       "memory, the step, token / expert / score copied back, one captured CUDA graph of "
+                       "the call per step; the host reads each step's choice while the next runs; wall clock",
+               "host_tokens_equal_device_history": same,
+               "eager": {"value": dist.sum(w.B * e2e_steps) / el_eager, "unit": UNIT,
+                         "path": "the same loop with eager pced_step_host_io calls"}}
+        if not same:
+            status |= 1 << 16
     status |= dec.status()
     del dec, g
     torch.cuda.empty_cache()

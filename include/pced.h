@@ -323,6 +323,15 @@ typedef struct pced_step_args {
    * way (every GPU appends the same input token). */
   int32_t expert_base;
   int64_t* key_out;
+  /* Optional per-call outputs at fixed device addresses (each may be NULL):
+   * this call's chosen token, its expert (1-based) and its score per query
+   * ([B] each), the values history / expert_trace / score_trace receive at t.
+   * The traces move with t; these do not, so a captured CUDA graph of the call
+   * (or of pced_step_host_io) finds each step's choice at the same address.
+   * An expert-partitioned call (key_out) does not write them. */
+  int32_t* token_out;
+  int32_t* expert_out;
+  float* score_out;
 } pced_step_args;
 
 #define PCED_SCORE_LOGPROB 0
@@ -354,6 +363,32 @@ pced_status pced_step_commit(const int64_t* keys, int32_t B, int32_t* step, int3
 
 size_t pced_step_workspace_size(const pced_dims* dims);
 pced_status pced_step(const pced_step_args* args, void* stream);
+
+/* One decode step with its per-step inputs and outputs in host memory, as a
+ * serving loop runs it (Sec. 3: every step scores the experts with their
+ * retrieval-derived weights r_k and contrast strengths beta_k of Eq. 2, and
+ * the chosen token leaves the GPU to be emitted).  In stream order:
+ *   1. beta_host, r_host (host fp32 [B][N] each; NULL: leave the device
+ *      values) are copied into the device arrays args->beta and args->r
+ *      point to (this call writes them);
+ *   2. pced_step(args, stream);
+ *   3. the step's choice is copied from args->token_out / expert_out /
+ *      score_out into token_host / expert_host / score_host (host [B] each;
+ *      NULL: not copied).
+ * The call returns without waiting: the host outputs hold the step's values
+ * once the stream has passed the call (synchronise it or an event recorded
+ * after it).  Host buffers should be page-locked (cudaHostAlloc or
+ * cudaHostRegister): the copies are then asynchronous, and a stream capture
+ * of the call records them as graph nodes, so one graph replay is one step
+ * with its uploads and read-backs; pageable buffers are staged by the CUDA
+ * runtime and may block the calling thread.  Errors (nothing is enqueued):
+ * PCED_ERR_INVALID_ARG for a host output without its device output in args,
+ * for an expert-partitioned call (key_out set) and, outside a stream capture,
+ * for a "host" pointer that is device memory; any error pced_step reports
+ * for args.  With beta_from_step the step overwrites beta_out after the
+ * upload (upload nothing then, or a starting beta that is ignored). */
+pced_status pced_step_host_io(const pced_step_args* args, const float* beta_host, const float* r_host,
+                              int32_t* token_host, int32_t* expert_host, float* score_host, void* stream);
 
 /* Number of kernel launches one pced_step call with these arguments makes:
  * 3 for the max rule with a fixed beta (attention, LM head, selection); a

@@ -51,7 +51,8 @@ class StepArgs(ctypes.Structure):
                 ("n_stage_events", ctypes.c_int32), ("beta_from_step", ctypes.c_int32), ("beta_out", ctypes.c_void_p),
                 ("block_table", ctypes.c_void_p), ("block_rows", ctypes.c_int32), ("max_blocks", ctypes.c_int32),
                 ("rope_theta", ctypes.c_float), ("score_mode", ctypes.c_int32), ("aggregation", ctypes.c_int32),
-                ("wait_limit_ns", ctypes.c_uint64), ("expert_base", ctypes.c_int32), ("key_out", ctypes.c_void_p)]
+                ("wait_limit_ns", ctypes.c_uint64), ("expert_base", ctypes.c_int32), ("key_out", ctypes.c_void_p),
+                ("token_out", ctypes.c_void_p), ("expert_out", ctypes.c_void_p), ("score_out", ctypes.c_void_p)]
 
 
 _lib = None
@@ -93,6 +94,8 @@ def lib(path: str = LIB_PATH):
         L.pced_step_workspace_size.restype = SZ
         L.pced_step.argtypes = [ctypes.POINTER(StepArgs), P]
         L.pced_step.restype = I32
+        L.pced_step_host_io.argtypes = [ctypes.POINTER(StepArgs), P, P, P, P, P, P]
+        L.pced_step_host_io.restype = I32
         L.pced_step_launch_count.argtypes = [ctypes.POINTER(StepArgs)]
         L.pced_step_launch_count.restype = I32
         L.pced_step_launch_kind.argtypes = [ctypes.POINTER(StepArgs), I32]
@@ -298,6 +301,10 @@ class Decoder:
         self.score_trace = torch.zeros((B, max_steps), dtype=torch.float32, device=dev)
         # near-tie margins of every choice: [B, max_steps, 2] (token gap, expert gap)
         self.gap_trace = torch.zeros((B, max_steps, 2), dtype=torch.float32, device=dev) if track_gaps else None
+        # this step's choice at fixed addresses (the traces move with t)
+        self.token_out = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.expert_out = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.score_out = torch.zeros(B, dtype=torch.float32, device=dev)
         self.hidden = torch.zeros((S, d), dtype=torch.bfloat16, device=dev) if keep_hidden else None
         self.lse = torch.zeros(S, dtype=torch.float32, device=dev)
         self.ws = workspace(step_workspace_size(dm), dev)
@@ -312,6 +319,9 @@ class Decoder:
             float(1.0 / math.sqrt(dm.D) if attn_scale is None else attn_scale), float(rms_eps), int(bos),
             _ptr(self.hidden), _ptr(self.lse), _ptr(self.ws), self.ws.numel())
         self.max_steps = max_steps
+        self.args.token_out = _ptr(self.token_out)
+        self.args.expert_out = _ptr(self.expert_out)
+        self.args.score_out = _ptr(self.score_out)
         self.args.rope_theta = float(rope_theta)  # rotary base, 0: none
         self.args.score_mode = int(score_mode)     # SCORE_LOGPROB / SCORE_LOGIT
         self.args.aggregation = int(aggregation)   # AGG_MAX / AGG_MOE / AGG_POE
@@ -330,6 +340,38 @@ class Decoder:
     def step(self, stream=None):
         _check(lib().pced_step(ctypes.byref(self.args), _stream(stream)), "pced_step")
         self.args.beta_from_step = 0
+
+    def step_host_io(self, beta=None, r=None, token=None, expert=None, score=None, stream=None):
+        """One step with host buffers (pced_step_host_io): uploads `beta` / `r`
+        (host fp32 [B, N], None: keep the device values), steps, and copies
+        the choice into `token` / `expert` / `score` (host [B] int32 / int32 /
+        fp32, None: skip).  Asynchronous on the stream; use page-locked
+        tensors (pin_memory()) for asynchronous copies and graph capture."""
+        B, N = self.dm.B, self.dm.N
+
+        def host(t, dtype, n):
+            if t is None:
+                return None
+            assert t.device.type == "cpu" and t.dtype == dtype and t.is_contiguous() and t.numel() == n
+            return t.data_ptr()
+
+        _check(lib().pced_step_host_io(ctypes.byref(self.args), host(beta, torch.float32, B * N),
+                                       host(r, torch.float32, B * N), host(token, torch.int32, B),
+                                       host(expert, torch.int32, B), host(score, torch.float32, B),
+                                       _stream(stream)), "pced_step_host_io")
+        self.args.beta_from_step = 0
+
+    def capture_host_io(self, beta=None, r=None, token=None, expert=None, score=None):
+        """A CUDA graph of one step_host_io call: each replay is one decode
+        step with its uploads and read-backs (page-locked host tensors
+        required; the decoder's dynamic-beta first step must already be done)."""
+        assert not self.args.beta_from_step, "run the dynamic-beta first step before capturing"
+        for t in (beta, r, token, expert, score):
+            assert t is None or t.is_pinned(), "graph capture needs page-locked host tensors"
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.step_host_io(beta, r, token, expert, score)
+        return g
 
     def step_partial(self, keys, expert_base: int, stream=None):
         """Expert-partitioned step: this decoder's experts are global experts

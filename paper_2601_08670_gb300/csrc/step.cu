@@ -153,7 +153,9 @@ extern "C" const char* pced_step_launch_kind(const pced_step_args* p, int32_t i)
   return kinds[i];
 }
 
-extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
+// Host-side validation of a pced_step call; on success *g and *num_blocks
+// hold the LM-head geometry and the paged pool's block count.
+static pced_status step_check(const pced_step_args* p, LmGeom* g_out, int64_t* num_blocks_out) {
   if (!p) return fail(PCED_ERR_INVALID_ARG, "pced_step: null args");
   const pced_dims dm = p->dims;
   const bool paged = p->block_table != nullptr;
@@ -205,6 +207,19 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   if (((uintptr_t)p->workspace) & 255u || p->workspace_bytes < pced_step_workspace_size(&dm))
     return fail(PCED_ERR_WORKSPACE, "pced_step: workspace too small or misaligned");
   if (num_sms() <= 0) return fail(PCED_ERR_NO_DEVICE, "pced_step: no CUDA device");
+  *g_out = g;
+  *num_blocks_out = num_blocks;
+  return PCED_OK;
+}
+
+extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
+  LmGeom g;
+  int64_t num_blocks = 0;
+  const pced_status chk = step_check(p, &g, &num_blocks);
+  if (chk != PCED_OK) return chk;
+  const pced_dims dm = p->dims;
+  const bool paged = p->block_table != nullptr;
+  const int32_t S = dm.B * (dm.N + 1), d = dm.Hq * dm.D, G = dm.Hq / dm.Hkv;
 
   const StepLayout W = step_layout(&dm, p->workspace);
   CUtensorMap kmap, vmap, wmap, hmap;
@@ -362,6 +377,9 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ag.score_trace = p->score_trace;
     ag.max_steps = p->max_steps;
     ag.done_counter = W.done_counter;
+    ag.token = p->token_out;
+    ag.expert = p->expert_out;
+    ag.score = p->score_out;
     ag.status = W.status;
     if (agg) {
       ranges.next("agg_partials");
@@ -432,6 +450,9 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   sa.score_trace = p->score_trace;
   sa.max_steps = p->max_steps;
   sa.done_counter = W.done_counter;
+  sa.token = p->token_out;
+  sa.expert = p->expert_out;
+  sa.score = p->score_out;
   sa.status = W.status;
   sa.pdl = (timed || dyn) ? 0 : 1;
   sa.raw_logits = p->score_mode == PCED_SCORE_LOGIT;
@@ -439,5 +460,54 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
   e = select_from_records_launch(sa, s);
   if (e == cudaSuccess) e = mark();
   if (e != cudaSuccess) return cuda_status(e, "select launch");
+  return PCED_OK;
+}
+
+// A "host" buffer that is device memory would make the copy device to
+// device; refuse it where the runtime can say (not inside a stream capture,
+// where a pointer query is not a capturable call).
+static bool is_device_memory(const void* ptr) {
+  cudaPointerAttributes at = {};
+  if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice;
+}
+
+extern "C" pced_status pced_step_host_io(const pced_step_args* p, const float* beta_host, const float* r_host,
+                                         int32_t* token_host, int32_t* expert_host, float* score_host,
+                                         void* stream) {
+  if (!p) return fail(PCED_ERR_INVALID_ARG, "pced_step_host_io: null args");
+  if (p->key_out) return fail(PCED_ERR_INVALID_ARG, "pced_step_host_io: not for an expert-partitioned step");
+  if ((token_host && !p->token_out) || (expert_host && !p->expert_out) || (score_host && !p->score_out))
+    return fail(PCED_ERR_INVALID_ARG, "pced_step_host_io: a host output needs its device output in args");
+  LmGeom g;
+  int64_t num_blocks = 0;
+  const pced_status chk = step_check(p, &g, &num_blocks);
+  if (chk != PCED_OK) return chk;
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cap) != cudaSuccess) return cuda_status(cudaGetLastError(), "capture query");
+  if (cap == cudaStreamCaptureStatusNone) {
+    const void* host[5] = {beta_host, r_host, token_host, expert_host, score_host};
+    for (const void* h : host)
+      if (h && is_device_memory(h))
+        return fail(PCED_ERR_INVALID_ARG, "pced_step_host_io: a host buffer is device memory");
+  }
+  const size_t BN = (size_t)p->dims.B * p->dims.N, B = (size_t)p->dims.B;
+  cudaError_t e = cudaSuccess;
+  if (beta_host) e = cudaMemcpyAsync((void*)p->beta, beta_host, BN * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess && r_host)
+    e = cudaMemcpyAsync((void*)p->r, r_host, BN * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_status(e, "pced_step_host_io: upload");
+  const pced_status st = pced_step(p, stream);
+  if (st != PCED_OK) return st;
+  if (token_host) e = cudaMemcpyAsync(token_host, p->token_out, B * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess && expert_host)
+    e = cudaMemcpyAsync(expert_host, p->expert_out, B * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess && score_host)
+    e = cudaMemcpyAsync(score_host, p->score_out, B * sizeof(float), cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return cuda_status(e, "pced_step_host_io: read-back");
   return PCED_OK;
 }

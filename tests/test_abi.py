@@ -146,6 +146,21 @@ def test_step_rejects_bad_arguments(L):
     assert f(step_args(pced, workspace_bytes=100)) == 2
 
 
+def test_step_host_io_rejects_bad_arguments(L):
+    import paper_2601_08670_gb300 as pced
+    f = lambda a, tok=None, exp=None, sc=None: L.pced_step_host_io(ctypes.byref(a), None, None, tok, exp, sc, None)
+    assert L.pced_step_host_io(None, None, None, None, None, None, None) == 1
+    # a host output needs its device output
+    assert f(step_args(pced), tok=FAKE) == 1
+    assert f(step_args(pced), exp=FAKE) == 1
+    assert f(step_args(pced), sc=FAKE) == 1
+    # not for an expert-partitioned call
+    assert f(step_args(pced, key_out=FAKE, token_out=FAKE), tok=FAKE) == 1
+    # the step's own validation applies
+    assert f(step_args(pced, embed=None, token_out=FAKE), tok=FAKE) == 1
+    assert f(step_args(pced, D=96)) == 3
+
+
 def test_launch_count_and_kinds_follow_the_mode(L):
     import paper_2601_08670_gb300 as pced
     assert pced.step_launch_kinds(step_args(pced)) == ["attention", "lm_head", "select"]
