@@ -305,11 +305,11 @@ def run_e2e(dec, w, dev, steps):
     device history."""
     import torch
     B = w.B
-    beta_h = dec.beta.cpu().pin_memory()
-    r_h = dec.r.cpu().pin_memory()
-    slots = [dict(token=torch.zeros(B, dtype=torch.int32).pin_memory(),
-                  expert=torch.zeros(B, dtype=torch.int32).pin_memory(),
-                  score=torch.zeros(B, dtype=torch.float32).pin_memory()) for _ in range(2)]
+    # beta and r side by side, and the choice as one [3, B] block, as on the
+    # device: one upload and one read-back per step
+    beta_r = torch.stack([dec.beta.cpu(), dec.r.cpu()]).pin_memory()
+    beta_h, r_h = beta_r[0], beta_r[1]
+    slots = [dict(zip(("token", "expert", "score"), dec.choice_buffers())) for _ in range(2)]
     graphs = [dec.capture_host_io(beta_h, r_h, **sl) for sl in slots]
     events = [torch.cuda.Event(), torch.cuda.Event()]
 
@@ -485,8 +485,9 @@ def run_ours(args):
         e2e = {"value": dist.sum(w.B * e2e_steps) / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "steps": e2e_steps,
                "path": "pced_step_host_io (C ABI, host buffers): beta and r uploaded from page-locked host "
-                       "memory, the step, token / expert / score copied back, one captured CUDA graph of "
-                       "the call per step; the host reads each step's choice while the next runs; wall clock",
+                       "memory (one copy), the step, token / expert / score copied back (one copy), one "
+                       "captured CUDA graph of the call per step; the host reads each step's choice while the "
+                       "next runs; wall clock",
                "host_tokens_equal_device_history": same,
                "eager": {"value": dist.sum(w.B * e2e_steps) / el_eager, "unit": UNIT,
                          "path": "the same loop with eager pced_step_host_io calls"}}

@@ -11,8 +11,9 @@
  * then appends y_t to the shared history of all experts.
  *
  * Conventions shared by every entry point
- *   - All tensor pointers are DEVICE pointers owned by the caller; the
- *     library allocates nothing and never synchronises.  `stream` is a
+ *   - All tensor pointers are DEVICE pointers owned by the caller (the one
+ *     exception: the *_host buffers of pced_step_host_io, in host memory);
+ *     the library allocates nothing and never synchronises.  `stream` is a
  *     cudaStream_t (NULL = legacy default stream).
  *   - bf16 tensors are raw bf16 arrays (2 bytes per element).
  *   - Sequences are query-major: sequence s = b*(N+1) + j belongs to query b;
@@ -381,7 +382,10 @@ pced_status pced_step(const pced_step_args* args, void* stream);
  * cudaHostRegister): the copies are then asynchronous, and a stream capture
  * of the call records them as graph nodes, so one graph replay is one step
  * with its uploads and read-backs; pageable buffers are staged by the CUDA
- * runtime and may block the calling thread.  Errors (nothing is enqueued):
+ * runtime and may block the calling thread.  Each copy adds a few
+ * microseconds of latency to the step: buffers that lie side by side on both
+ * sides (r right after beta; expert right after token, score right after
+ * expert) move in one copy each way.  Errors (nothing is enqueued):
  * PCED_ERR_INVALID_ARG for a host output without its device output in args,
  * for an expert-partitioned call (key_out set) and, outside a stream capture,
  * for a "host" pointer that is device memory; any error pced_step reports

@@ -302,9 +302,10 @@ class Decoder:
         # near-tie margins of every choice: [B, max_steps, 2] (token gap, expert gap)
         self.gap_trace = torch.zeros((B, max_steps, 2), dtype=torch.float32, device=dev) if track_gaps else None
         # this step's choice at fixed addresses (the traces move with t)
-        self.token_out = torch.zeros(B, dtype=torch.int32, device=dev)
-        self.expert_out = torch.zeros(B, dtype=torch.int32, device=dev)
-        self.score_out = torch.zeros(B, dtype=torch.float32, device=dev)
+        # (one [3, B] block, so that reading all three back is one copy)
+        self._choice = torch.zeros((3, B), dtype=torch.int32, device=dev)
+        self.token_out, self.expert_out = self._choice[0], self._choice[1]
+        self.score_out = self._choice[2].view(torch.float32)
         self.hidden = torch.zeros((S, d), dtype=torch.bfloat16, device=dev) if keep_hidden else None
         self.lse = torch.zeros(S, dtype=torch.float32, device=dev)
         self.ws = workspace(step_workspace_size(dm), dev)
@@ -346,7 +347,10 @@ class Decoder:
         (host fp32 [B, N], None: keep the device values), steps, and copies
         the choice into `token` / `expert` / `score` (host [B] int32 / int32 /
         fp32, None: skip).  Asynchronous on the stream; use page-locked
-        tensors (pin_memory()) for asynchronous copies and graph capture."""
+        tensors (pin_memory()) for asynchronous copies and graph capture.
+        Adjacent buffers on both sides (r right after beta; expert after
+        token, score after expert, as choice_buffers() lays them out) move
+        in one copy each way."""
         B, N = self.dm.B, self.dm.N
 
         def host(t, dtype, n):
@@ -360,6 +364,12 @@ class Decoder:
                                        host(expert, torch.int32, B), host(score, torch.float32, B),
                                        _stream(stream)), "pced_step_host_io")
         self.args.beta_from_step = 0
+
+    def choice_buffers(self):
+        """Page-locked host (token, expert, score) tensors laid out like the
+        device outputs, so step_host_io reads them back in one copy."""
+        blk = torch.zeros((3, self.dm.B), dtype=torch.int32).pin_memory()
+        return blk[0], blk[1], blk[2].view(torch.float32)
 
     def capture_host_io(self, beta=None, r=None, token=None, expert=None, score=None):
         """A CUDA graph of one step_host_io call: each replay is one decode

@@ -496,18 +496,37 @@ extern "C" pced_status pced_step_host_io(const pced_step_args* p, const float* b
         return fail(PCED_ERR_INVALID_ARG, "pced_step_host_io: a host buffer is device memory");
   }
   const size_t BN = (size_t)p->dims.B * p->dims.N, B = (size_t)p->dims.B;
+  // Each copy costs a few microseconds of copy-engine latency on the step's
+  // critical path, far more than its bytes: buffers that lie side by side on
+  // both sides (r after beta; expert after token, score after expert) move
+  // in one copy.
+  auto adjacent = [](const void* a, const void* b, size_t bytes) {
+    return (const char*)b == (const char*)a + bytes;
+  };
+  const bool one_in = beta_host && r_host && adjacent(beta_host, r_host, BN * 4) && adjacent(p->beta, p->r, BN * 4);
+  const bool one_out = token_host && expert_host && score_host && adjacent(token_host, expert_host, B * 4) &&
+                       adjacent(expert_host, score_host, B * 4) && adjacent(p->token_out, p->expert_out, B * 4) &&
+                       adjacent(p->expert_out, p->score_out, B * 4);
   cudaError_t e = cudaSuccess;
-  if (beta_host) e = cudaMemcpyAsync((void*)p->beta, beta_host, BN * sizeof(float), cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess && r_host)
-    e = cudaMemcpyAsync((void*)p->r, r_host, BN * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (one_in) {
+    e = cudaMemcpyAsync((void*)p->beta, beta_host, 2 * BN * sizeof(float), cudaMemcpyHostToDevice, s);
+  } else {
+    if (beta_host) e = cudaMemcpyAsync((void*)p->beta, beta_host, BN * sizeof(float), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess && r_host)
+      e = cudaMemcpyAsync((void*)p->r, r_host, BN * sizeof(float), cudaMemcpyHostToDevice, s);
+  }
   if (e != cudaSuccess) return cuda_status(e, "pced_step_host_io: upload");
   const pced_status st = pced_step(p, stream);
   if (st != PCED_OK) return st;
-  if (token_host) e = cudaMemcpyAsync(token_host, p->token_out, B * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess && expert_host)
-    e = cudaMemcpyAsync(expert_host, p->expert_out, B * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess && score_host)
-    e = cudaMemcpyAsync(score_host, p->score_out, B * sizeof(float), cudaMemcpyDeviceToHost, s);
+  if (one_out) {
+    e = cudaMemcpyAsync(token_host, p->token_out, 3 * B * 4, cudaMemcpyDeviceToHost, s);
+  } else {
+    if (token_host) e = cudaMemcpyAsync(token_host, p->token_out, B * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && expert_host)
+      e = cudaMemcpyAsync(expert_host, p->expert_out, B * sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && score_host)
+      e = cudaMemcpyAsync(score_host, p->score_out, B * sizeof(float), cudaMemcpyDeviceToHost, s);
+  }
   if (e != cudaSuccess) return cuda_status(e, "pced_step_host_io: read-back");
   return PCED_OK;
 }

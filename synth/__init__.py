@@ -446,6 +446,9 @@ def device_inputs(w: Workload, device="cuda", extra_steps: int | None = None, st
     wu = torch.empty((w.V, w.d), dtype=torch.bfloat16, device=device)
     dev_fill_matrix(w, T_EMBED, emb, sp)
     dev_fill_matrix(w, T_UNEMBED, wu, sp)
+    # beta and r side by side in one allocation, so a per-step upload of both
+    # can be one copy
+    beta_r = torch.from_numpy(np.ascontiguousarray(np.stack([betas(full)[:, cols],
+                                                             retrieval_scores(full)[:, cols]]))).to(device)
     return dict(k_cache=k, v_cache=v, kv_offset=kv_off, cap=cap, seq_len=base.clone(), base_len=bl, layout=lay,
-                embed=emb, w_unembed=wu, beta=torch.from_numpy(np.ascontiguousarray(betas(full)[:, cols])).to(device),
-                r=torch.from_numpy(np.ascontiguousarray(retrieval_scores(full)[:, cols])).to(device), w=w, **extra)
+                embed=emb, w_unembed=wu, beta=beta_r[0], r=beta_r[1], w=w, **extra)

@@ -39,6 +39,16 @@ def host_buffers(w, beta, r):
                 score=torch.zeros(w.B, dtype=torch.float32).pin_memory())
 
 
+def adjacent_host_buffers(dec, beta, r):
+    # r right after beta and the choice as one block, as on the device: the
+    # call moves each side in one copy
+    br = torch.stack([beta.cpu(), r.cpu()]).pin_memory()
+    tok, exp, sc = dec.choice_buffers()
+    assert exp.data_ptr() == tok.data_ptr() + 4 * tok.numel() and sc.data_ptr() == exp.data_ptr() + 4 * tok.numel()
+    assert dec.r.data_ptr() == dec.beta.data_ptr() + 4 * dec.beta.numel()
+    return dict(beta=br[0], r=br[1], token=tok, expert=exp, score=sc)
+
+
 def per_query_beta(w):
     # a different contrast strength per (query, expert), so a lost upload shows
     return torch.from_numpy(np.random.default_rng(5).uniform(0.1, 0.9, (w.B, w.N)).astype(np.float32))
@@ -96,7 +106,7 @@ def test_graph_of_one_host_io_step_replays_step_after_step(cuda_ok):
     ref = decoder(w, dev)
     ref.beta.copy_(beta)
     dec = decoder(w, dev)
-    hb = host_buffers(w, beta, ref.r)
+    hb = adjacent_host_buffers(dec, beta, ref.r)
     dec.beta.fill_(float("nan"))
     dec.r.fill_(float("nan"))
     g = dec.capture_host_io(**hb)
@@ -136,7 +146,7 @@ def test_host_io_with_dynamic_beta_and_moe(cuda_ok):
     # MoE: the aggregation kernels write the fixed-address outputs too
     ref = decoder(w, dev, aggregation=pced.AGG_MOE)
     dec = decoder(w, dev, aggregation=pced.AGG_MOE)
-    hb = host_buffers(w, ref.beta, ref.r)
+    hb = adjacent_host_buffers(dec, ref.beta, ref.r)
     for t in range(2):
         ref.step()
         dec.step_host_io(hb["beta"], hb["r"], hb["token"], hb["expert"], hb["score"])
