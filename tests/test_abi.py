@@ -144,6 +144,9 @@ def test_step_rejects_bad_arguments(L):
     assert f(step_args(pced, D=96)) == 3
     assert f(step_args(pced, bos_token=128256)) == 1
     assert f(step_args(pced, workspace_bytes=100)) == 2
+    # beyond the maxima: S = B (N + 1) > 512, N + 1 > 256 sequences per query
+    assert f(step_args(pced, B=3, N=170)) == 3
+    assert f(step_args(pced, B=1, N=256)) == 3
 
 
 def test_step_host_io_rejects_bad_arguments(L):

@@ -55,8 +55,9 @@ def test_larger_logits_scale(cuda_ok):
     assert run_case(17, 1024, 3000, wscale=0.2) < 1e-3
 
 
-@pytest.mark.parametrize("S", [272, 300, 340])
+@pytest.mark.parametrize("S", [272, 300, 340, 512])
 def test_many_tiles_per_cta_with_two_n_chunks(cuda_ok, S):
     # more than 256 hidden rows: two N chunks in one TMEM accumulator, several
-    # vocabulary tiles per CTA (the accumulator is reused), ragged tail
+    # vocabulary tiles per CTA (the accumulator is reused), ragged tail; 512
+    # rows is the maximum (two 256-column chunks in all 512 TMEM columns)
     assert run_case(S, 256, 48000 + 77) < 1e-4

@@ -142,6 +142,18 @@ def test_tiny_graph_replay(cuda_ok):
     run_parity("tiny", 4, graph=True)
 
 
+def test_largest_batch_and_empty_caches(cuda_ok):
+    # The library's limits at once: S = 512 sequences (the LM head's maximum:
+    # two 256-column MMA chunks filling all 512 TMEM columns) and 256
+    # sequences per query (255 experts and the amateur, the selection's
+    # maximum).  Documents of 0-3 tokens and empty amateurs: 129 of the 512
+    # caches start empty, so their first step attends to its own appended
+    # row only.
+    w = synth.get("tiny", B=2, N=255, doc_len=("uniform", 0, 3), query_tokens=0, amateur_len=0, seed=11)
+    assert w.S == 512 and int((synth.base_lengths(w) == 0).sum()) > 100
+    run_parity("tiny", 3, B=2, N=255, doc_len=("uniform", 0, 3), query_tokens=0, amateur_len=0, seed=11)
+
+
 @pytest.mark.parametrize("V", [8192 + 77, 1000, 128 * 300 + 1])
 def test_tiny_ragged_vocabularies(cuda_ok, V):
     # the last vocabulary tile of the fused LM head is partly outside V:
