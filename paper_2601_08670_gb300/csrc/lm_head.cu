@@ -544,12 +544,16 @@ __global__ void __launch_bounds__(LM_THREADS, 1)
 
 cudaError_t lm_head_launch(const CUtensorMap& wmap, const CUtensorMap& hmap, const LmGeom& g, const LmArgs& a,
                            cudaStream_t stream) {
-  static size_t configured = 0;
-  if (configured < g.smem) {
-    cudaError_t e = cudaFuncSetAttribute(lm_head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)LM_SMEM_BUDGET);
+  // the shared-memory limit is an attribute of the kernel on each device
+  static bool configured[64];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!configured[dev]) {
+    e = cudaFuncSetAttribute(lm_head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LM_SMEM_BUDGET);
     if (e != cudaSuccess) return e;
-    configured = LM_SMEM_BUDGET;
+    configured[dev] = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(g.grid);
