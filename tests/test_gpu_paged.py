@@ -33,15 +33,20 @@ def test_paged_pool_holds_the_logical_cache(cuda_ok):
                     assert np.array_equal(pool_v[l, blk, h, pos % lay.P], want_v)
 
 
-@pytest.mark.parametrize("name,P,steps,queries,ram", [("tiny", 64, 4, None, 0), ("tiny", 192, 3, None, 0),
-                                                       ("llama8", 256, 2, None, 8), ("manydoc", 64, 1, [0, 15], 8)])
-def test_paged_step_matches_oracle(cuda_ok, name, P, steps, queries, ram):
+@pytest.mark.parametrize("name,P,steps,queries,ram,over", [
+    ("tiny", 64, 4, None, 0, {}), ("tiny", 192, 3, None, 0, {}),
+    # seven query heads per kv head at D = 128 (the Qwen grouping) in 128-row blocks
+    ("tiny", 128, 3, None, 0, dict(Hq=14, Hkv=2, D=128)),
+    ("llama8", 256, 2, None, 8, {}), ("manydoc", 64, 1, [0, 15], 8, {}),
+    # Qwen2-7B shapes (28 layers, G = 7, 4096 + 32 keys) over 64-row blocks
+    ("qwen_flat", 64, 1, None, 8, {})])
+def test_paged_step_matches_oracle(cuda_ok, name, P, steps, queries, ram, over):
     import paper_2601_08670_gb300 as pced
     from oracle.run import OracleRun
     from test_gpu_step import check_stats, compare_step, host_ram_gb, new_stats
     if host_ram_gb() < ram:
         pytest.skip(f"needs {ram} GB of free host memory for the oracle's caches")
-    w = synth.get(name)
+    w = synth.get(name, **over)
     t = synth.device_inputs(w, "cuda", paged=P)
     dm = pced.dims(w.B, w.N, w.L, w.Hq, w.Hkv, w.D, w.V)
     dec = pced.decoder_from_inputs(dm, t, gamma=w.gamma, max_steps=w.steps, bos=w.bos, keep_hidden=True)

@@ -154,6 +154,13 @@ def test_largest_batch_and_empty_caches(cuda_ok):
     run_parity("tiny", 3, B=2, N=255, doc_len=("uniform", 0, 3), query_tokens=0, amateur_len=0, seed=11)
 
 
+def test_largest_hidden_size(cuda_ok):
+    # d = Hq * D = 8192, the largest hidden size pced_step takes (64 query /
+    # 8 kv heads of 128): 128 K-slabs per LM-head tile, 1024 16-byte chunks
+    # per row in the embedding slices and the near-tie dot products
+    run_parity("tiny", 3, Hq=64, Hkv=8, D=128)
+
+
 @pytest.mark.parametrize("V", [8192 + 77, 1000, 128 * 300 + 1])
 def test_tiny_ragged_vocabularies(cuda_ok, V):
     # the last vocabulary tile of the fused LM head is partly outside V:
