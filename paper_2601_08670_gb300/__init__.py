@@ -116,6 +116,12 @@ def _check(rc: int, what: str):
         raise PcedError(rc, f"{what}: {L.pced_status_string(rc).decode()}: {L.pced_last_error().decode()}")
 
 
+def _require(cond: bool, what: str):
+    """Argument check of the binding (raises even under python -O)."""
+    if not cond:
+        raise ValueError(what)
+
+
 def _ptr(t):
     return None if t is None else t.data_ptr()
 
@@ -240,10 +246,10 @@ def relevance(ret_scores, ret_mode: int = RET_DENSE, rer_logits=None, eps: float
     """pced_relevance: relevance scores in [0, 1) from raw retrieval scores
     (dense/ColBERT or sparse) and optional reranker logits, fused by the
     harmonic mean (fp32 tensors of one shape on the device)."""
-    assert ret_scores.dtype == torch.float32 and ret_scores.is_contiguous()
+    _require(ret_scores.dtype == torch.float32 and ret_scores.is_contiguous(), "ret_scores: contiguous fp32")
     if rer_logits is not None:
-        assert rer_logits.dtype == torch.float32 and rer_logits.is_contiguous()
-        assert rer_logits.shape == ret_scores.shape
+        _require(rer_logits.dtype == torch.float32 and rer_logits.is_contiguous(), "rer_logits: contiguous fp32")
+        _require(rer_logits.shape == ret_scores.shape, "rer_logits: the shape of ret_scores")
     r = torch.empty_like(ret_scores)
     _check(lib().pced_relevance(_ptr(ret_scores), int(ret_mode), _ptr(rer_logits), ret_scores.numel(), float(eps),
                                 _ptr(r), _stream(stream)), "pced_relevance")
@@ -327,14 +333,15 @@ class Decoder:
         self.args.score_mode = int(score_mode)     # SCORE_LOGPROB / SCORE_LOGIT
         self.args.aggregation = int(aggregation)   # AGG_MAX / AGG_MOE / AGG_POE
         if block_table is not None:  # paged caches
-            assert block_table.dtype == torch.int32 and block_table.is_contiguous() and block_table.dim() == 2
+            _require(block_table.dtype == torch.int32 and block_table.is_contiguous() and block_table.dim() == 2,
+                     "block_table: contiguous int32 [S, max_blocks]")
             self.args.block_table = _ptr(block_table)
             self.args.block_rows = int(block_rows)
             self.args.max_blocks = int(block_table.shape[1])
         # dynamic contrast strength: the first step computes beta (into the
         # `beta` tensor, which the later steps read) from its distributions
         if dynamic_beta:
-            assert beta.dtype == torch.float32 and beta.is_contiguous()
+            _require(beta.dtype == torch.float32 and beta.is_contiguous(), "beta: contiguous fp32 (dynamic beta writes it)")
             self.args.beta_from_step = 1
             self.args.beta_out = _ptr(beta)
 
@@ -356,7 +363,8 @@ class Decoder:
         def host(t, dtype, n):
             if t is None:
                 return None
-            assert t.device.type == "cpu" and t.dtype == dtype and t.is_contiguous() and t.numel() == n
+            _require(t.device.type == "cpu" and t.dtype == dtype and t.is_contiguous() and t.numel() == n,
+                     f"host buffers: contiguous {dtype} CPU tensors of {n} elements")
             return t.data_ptr()
 
         _check(lib().pced_step_host_io(ctypes.byref(self.args), host(beta, torch.float32, B * N),
@@ -375,9 +383,9 @@ class Decoder:
         """A CUDA graph of one step_host_io call: each replay is one decode
         step with its uploads and read-backs (page-locked host tensors
         required; the decoder's dynamic-beta first step must already be done)."""
-        assert not self.args.beta_from_step, "run the dynamic-beta first step before capturing"
+        _require(not self.args.beta_from_step, "run the dynamic-beta first step before capturing")
         for t in (beta, r, token, expert, score):
-            assert t is None or t.is_pinned(), "graph capture needs page-locked host tensors"
+            _require(t is None or t.is_pinned(), "graph capture needs page-locked host tensors")
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
             self.step_host_io(beta, r, token, expert, score)
@@ -389,7 +397,8 @@ class Decoder:
         as packed keys (int64 [B] device tensor `keys`) and appends nothing.
         Reduce the keys with a max over the decoders (NCCL / gloo all-reduce,
         torch.maximum), then call commit()."""
-        assert keys.dtype == torch.int64 and keys.is_contiguous() and keys.numel() >= self.dm.B
+        _require(keys.dtype == torch.int64 and keys.is_contiguous() and keys.numel() >= self.dm.B,
+                 "keys: contiguous int64 of at least B elements")
         self.args.key_out = _ptr(keys)
         self.args.expert_base = int(expert_base)
         try:

@@ -194,3 +194,16 @@ def test_workspace_sizes(L):
 def test_valid_call_without_device_reports_no_device(L):
     import torch  # noqa: F401
     assert L.pced_contrastive_select(FAKE, FAKE, FAKE, 2.5, 1, 4, 100, FAKE, FAKE, FAKE, FAKE, 1 << 30, None) == 5
+
+
+def test_binding_rejects_bad_tensors_before_any_call(L):
+    # the binding's own checks raise ValueError (also under python -O),
+    # before the library or a device is touched
+    import torch
+    import paper_2601_08670_gb300 as pced
+    with pytest.raises(ValueError):
+        pced.relevance(torch.zeros(4, dtype=torch.float64))
+    with pytest.raises(ValueError):
+        pced.relevance(torch.zeros(4), rer_logits=torch.zeros(5))
+    with pytest.raises(ValueError):
+        pced.relevance(torch.zeros(4, 2).t())  # not contiguous
