@@ -302,8 +302,8 @@ typedef struct pced_step_args {
    * argmax_v log sum_k w_k p_k(v), PoE argmax_v sum_k w_k log p_k(v); the
    * expert reported is argmax_k w_k p_k(token), the score the aggregate;
    * gamma and score_mode do not enter (a per-expert constant drops out of the
-   * softmax).  These rules materialise the log-probabilities (S x V fp32 in
-   * the workspace) and take five launches (see pced_step_launch_kind). */
+   * softmax).  These rules materialise the logits (S x V fp32 in the
+   * workspace) and take four launches (see pced_step_launch_kind). */
   int32_t aggregation;
   /* How long (ns) a warp of the attention kernel waits for another warp or
    * CTA (a layer's input, a partial record, a pipeline stage) before it sets
@@ -398,8 +398,9 @@ pced_status pced_step_host_io(const pced_step_args* args, const float* beta_host
  * 3 for the max rule with a fixed beta (attention, LM head, selection); a
  * first step with beta_from_step runs attention, a logits pass, its
  * log-sum-exp finalise, the beta kernel and a selection from the
- * log-probabilities (5); MoE / PoE run attention, the logits pass, the
- * finalise and two aggregation kernels (5; 6 with beta_from_step).  Only the
+ * log-probabilities (5); MoE / PoE run attention, the logits pass and two
+ * aggregation kernels, which read the raw logits (4; with beta_from_step
+ * also the finalise and the beta kernel, 6).  Only the
  * fields dims, beta_from_step and aggregation are read; NULL gives 0. */
 int32_t pced_step_launch_count(const pced_step_args* args);
 /* Kind of launch i (0-based) of such a call: "attention", "lm_head",

@@ -59,6 +59,20 @@ __global__ void __launch_bounds__(AGG_THREADS) agg_partials_kernel(AggArgs a) {
     __syncthreads();
     return make_float2(M, Sm);
   };
+  if (a.rec_stats && c == 0) {
+    // raw logits: the log-sum-exps of expert k's row (and, for k = 0, the
+    // amateur's) from the LM head's tile records, in a fixed order
+    for (int r = 0; r < (k == 0 ? 2 : 1); ++r) {
+      const int64_t row = (int64_t)b * (N + 1) + (r == 0 ? k + 1 : 0);
+      float mm = -INFINITY, ss = 0.f;
+      for (int j = tid; j < a.nrec; j += AGG_THREADS) {
+        const float2 e = a.rec_stats[row * a.nrec + j];
+        agg_lse_merge(mm, ss, e.x, e.y);
+      }
+      const float2 t = block_merge(mm, ss);
+      if (tid == 0) a.lse_rows[row] = t.x + logf(t.y);
+    }
+  }
   float m = -INFINITY, s = 0.f;
   const int v1 = min(V, (c + 1) * AGG_CHUNK);
   for (int v = c * AGG_CHUNK + tid; v < v1; v += AGG_THREADS) {

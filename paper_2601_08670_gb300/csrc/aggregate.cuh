@@ -6,7 +6,14 @@
 namespace pced {
 
 struct AggArgs {
-  const float* lp;      // [S][V] log-probabilities, query-major, amateur first
+  // [S][V] log-probabilities, query-major, amateur first; or, with rec_stats
+  // set (MoE / PoE only), the raw logits z: p_k and the aggregates do not
+  // depend on the rows' log-sum-exps L (the constant (1+beta) L_k - beta L_0
+  // cancels in the softmax of the contrastive scores)
+  const float* lp;
+  const float2* rec_stats;  // raw logits: the LM head's per-tile (max, sum exp) of every row, [S][nrec]
+  int32_t nrec;
+  float* lse_rows;      // raw logits: [S] log-sum-exps formed from rec_stats (what lse points to)
   const float* beta;    // [B][N]
   const float* r;       // [B][N] relevance scores
   const float* lse;     // [S] log-sum-exps of the rows (copied to lse_out)

@@ -129,9 +129,11 @@ static int32_t step_plan(const pced_step_args* p, const char** kinds) {
   const bool dyn = p->beta_from_step != 0, agg = p->aggregation != PCED_AGG_MAX;
   add("attention");
   if (dyn || agg) {
-    add("lm_head");  // logits mode: log-probabilities materialised
-    add("lse_finalize");
-    if (dyn) add("adacad_beta");
+    add("lm_head");  // logits mode: the logits materialised
+    if (dyn) {
+      add("lse_finalize");  // normalised to log-probabilities for beta
+      add("adacad_beta");
+    }
   }
   if (agg) {
     add("agg_partials");
@@ -333,9 +335,14 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     ranges.next("lm_head");
     e = lm_head_launch(wmap, hmap, g, lz, s);
     if (e == cudaSuccess) e = mark();
-    if (e == cudaSuccess) ranges.next("lse_finalize");
-    if (e == cudaSuccess) e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
-    if (e == cudaSuccess) e = mark();
+    // MoE / PoE alone need no log-probabilities (the aggregation kernels
+    // read the raw logits and form the rows' log-sum-exps themselves); beta
+    // needs the normalised rows
+    if (e == cudaSuccess && dyn) {
+      ranges.next("lse_finalize");
+      e = lm_lse_finalize_launch(W.lp, W.lm_stats, W.sel_L, S, dm.V, g.ntiles, s);
+      if (e == cudaSuccess) e = mark();
+    }
     // the JSD kernel also re-arms the LM head's tile counter for the fused pass
     if (e == cudaSuccess && dyn) {
       ranges.next("adacad_beta");
@@ -350,6 +357,11 @@ extern "C" pced_status pced_step(const pced_step_args* p, void* stream) {
     // dynamic-beta decode has written anyway (no second LM-head pass)
     AggArgs ag = {};
     ag.lp = W.lp;
+    if (!dyn) {  // raw logits (MoE / PoE without a dynamic beta)
+      ag.rec_stats = W.lm_stats;
+      ag.nrec = g.ntiles;
+      ag.lse_rows = W.sel_L;
+    }
     ag.beta = beta;
     ag.r = p->r;
     ag.lse = W.sel_L;

@@ -170,13 +170,14 @@ def test_launch_count_and_kinds_follow_the_mode(L):
     assert pced.step_launch_kinds(step_args(pced, beta_from_step=1)) == [
         "attention", "lm_head", "lse_finalize", "adacad_beta", "agg_select"]
     for rule in (pced.AGG_MOE, pced.AGG_POE):
+        # the aggregation kernels read the raw logits: no finalise launch
         assert pced.step_launch_kinds(step_args(pced, aggregation=rule)) == [
-            "attention", "lm_head", "lse_finalize", "agg_partials", "agg_select"]
+            "attention", "lm_head", "agg_partials", "agg_select"]
         assert pced.step_launch_kinds(step_args(pced, aggregation=rule, beta_from_step=1)) == [
             "attention", "lm_head", "lse_finalize", "adacad_beta", "agg_partials", "agg_select"]
     a = step_args(pced, aggregation=pced.AGG_MOE)
-    assert pced.step_launch_count(a) == 5
-    assert L.pced_step_launch_kind(ctypes.byref(a), 5) is None
+    assert pced.step_launch_count(a) == 4
+    assert L.pced_step_launch_kind(ctypes.byref(a), 4) is None
     assert L.pced_step_launch_kind(ctypes.byref(a), -1) is None
     assert L.pced_step_launch_count(None) == 0
 
