@@ -624,6 +624,30 @@ def test_aggregate_single_expert_is_contrastive_greedy_and_permutation_invariant
         assert perm[b["expert"][0] - 1] + 1 == a["expert"][0]
 
 
+def test_aggregate_depends_on_each_row_only_up_to_a_constant():
+    # MoE and PoE take p_k as the softmax of the contrastive scores, so a
+    # constant added to any row (raw logits z = lp + L instead of lp) shifts
+    # each expert's scores by a constant that the softmax removes: the choice,
+    # the aggregate and both margins stay the same
+    rng = np.random.default_rng(11)
+    B, N, V = 2, 3, 64
+    z = rng.normal(size=(B * (N + 1), V)) * 2
+    lp = z - np.log(np.exp(z).sum(1, keepdims=True))
+    beta = rng.uniform(0.1, 0.9, (B, N)).astype(np.float32)
+    r = rng.uniform(0.05, 0.95, (B, N)).astype(np.float32)
+    shifted = lp + rng.normal(size=(B * (N + 1), 1)) * 7
+    for rule in (oracle.MOE, oracle.POE):
+        a = oracle.aggregate_select(lp, beta, r, rule)
+        b = oracle.aggregate_select(shifted, beta, r, rule)
+        assert np.array_equal(a["token"], b["token"]) and np.array_equal(a["expert"], b["expert"])
+        for key in ("score", "token_gap", "expert_gap"):
+            assert np.allclose(a[key], b[key], rtol=0, atol=1e-9), key
+    # Eq. 3 itself is not invariant: its per-expert constants carry the L_k
+    a = oracle.contrastive_select(lp, beta, r, 2.5, B, N)
+    b = oracle.contrastive_select(shifted, beta, r, 2.5, B, N)
+    assert not np.allclose(a["score"], b["score"])
+
+
 def test_step_raw_logit_mode_and_moe_in_closed_form():
     # one expert over an empty prefix: expert and amateur see the same single
     # token, so lp_1 = lp_0 and (1 + beta) s_1 - beta s_0 = s_1.  Log-prob mode
