@@ -71,3 +71,23 @@ def test_timed_steps_are_exact_with_several_steps_per_graph():
             assert cap == warmup + k * -(-warmup // k) + steps
             assert k * -(-warmup // k) >= warmup
     assert bench.steps_per_graph(64) == 8 and bench.steps_per_graph(7) == 7 and bench.steps_per_graph(11) == 1
+
+
+def test_reference_arm_prints_one_json_line_on_the_cpu():
+    # the reference arm is the oracle on the host cores: one JSON line with
+    # the contract's keys, its e2e equal to its value (no device copies)
+    import json
+    import subprocess
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                          "--steps", "2", "--warmup", "3"], capture_output=True, text=True, timeout=600, cwd=ROOT)
+    assert out.returncode == 0, out.stderr
+    lines = [l for l in out.stdout.splitlines() if l.strip()]
+    assert len(lines) == 1
+    rec = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+                "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert key in rec, key
+    assert rec["impl"] == "reference" and rec["value"] > 0 and rec["higher_is_better"] is True
+    assert rec["cpu_baseline"]["kind"] == "oracle" and rec["cpu_baseline"]["cores"] >= 1
+    assert rec["e2e"]["value"] == rec["value"] and rec["e2e"]["h2d_bytes_per_step"] == 0
+    assert rec["config"]["workload"].startswith("tiny")
