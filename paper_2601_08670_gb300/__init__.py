@@ -341,7 +341,8 @@ class Decoder:
         # dynamic contrast strength: the first step computes beta (into the
         # `beta` tensor, which the later steps read) from its distributions
         if dynamic_beta:
-            _require(beta.dtype == torch.float32 and beta.is_contiguous(), "beta: contiguous fp32 (dynamic beta writes it)")
+            _require(beta.dtype == torch.float32 and beta.is_contiguous(),
+                     "beta: contiguous fp32 (dynamic beta writes it)")
             self.args.beta_from_step = 1
             self.args.beta_out = _ptr(beta)
 
